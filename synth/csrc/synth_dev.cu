@@ -1,0 +1,135 @@
+// Device side of the synthetic workload generator (harness).  Same recipe and
+// same source of truth as the host side: synth_core.h.  Build with
+// --fmad=false so that no multiply-add is fused.
+#include <cuda_runtime.h>
+
+#include "synth_core.h"
+
+namespace {
+
+__device__ __forceinline__ void store(const syn_workload &w, void *out, int64_t i, float v) {
+  if (w.dtype == SYN_BF16)
+    ((uint16_t *)out)[i] = syn_bf16_bits(v);
+  else
+    ((float *)out)[i] = v;
+}
+
+// grid: x = row block, y = layer * H_kv + kvh, z = sequence; one thread per element
+__global__ void fill_cache_kernel(syn_workload w, const syn_seq *seqs, const int64_t *seq_off,
+                                  const int32_t *n_rows, int64_t S_total, void *K, void *V) {
+  const int b = blockIdx.z, lh = blockIdx.y;
+  const int layer = lh / w.H_kv, kvh = lh % w.H_kv;
+  const int rows_per_block = blockDim.x / w.d;
+  const int r = threadIdx.x / w.d, e = threadIdx.x % w.d;
+  const syn_seq s = seqs[b];
+  const int64_t nr = n_rows[b];
+  for (int64_t p = (int64_t)blockIdx.x * rows_per_block + r; p < nr;
+       p += (int64_t)gridDim.x * rows_per_block) {
+    int64_t i = ((int64_t)lh * S_total + seq_off[b] + p) * w.d + e;
+    store(w, K, i, syn_row_value(&w, &s, 0, layer, kvh, b, p, e));
+    store(w, V, i, syn_row_value(&w, &s, 1, layer, kvh, b, p, e));
+  }
+}
+
+// one thread per (layer, sequence, query head) for q, per (layer, sequence, kv-head, element)
+// for the new K/V rows.  mode 0: as the sequence state says; 1: every sequence loop-free;
+// 2: as if no sequence had been intervened on.
+__global__ void step_q_kernel(syn_workload w, const syn_seq *seqs, int batch, const int64_t *pos,
+                              int mode, void *q) {
+  int t = blockIdx.x * blockDim.x + threadIdx.x;
+  int total = w.L * batch * w.H_q;
+  if (t >= total) return;
+  int h = t % w.H_q, b = (t / w.H_q) % batch, layer = t / (w.H_q * batch);
+  syn_seq s = seqs[b];
+  if (mode == 1) s.fresh_from = 0;
+  if (mode == 2) s.fresh_from = SYN_NEVER;
+  float qv[128];
+  syn_query(&w, &s, layer, h, b, pos[b], qv);
+  for (int e = 0; e < w.d; ++e) store(w, q, (int64_t)t * w.d + e, qv[e]);
+}
+
+__global__ void step_kv_kernel(syn_workload w, const syn_seq *seqs, int batch,
+                               const int64_t *pos, int mode, void *k_new, void *v_new) {
+  int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  int64_t total = (int64_t)w.L * batch * w.H_kv * w.d;
+  if (t >= total) return;
+  int e = t % w.d;
+  int kvh = (t / w.d) % w.H_kv;
+  int b = (t / ((int64_t)w.d * w.H_kv)) % batch;
+  int layer = t / ((int64_t)w.d * w.H_kv * batch);
+  syn_seq s = seqs[b];
+  if (mode == 1) s.fresh_from = 0;
+  if (mode == 2) s.fresh_from = SYN_NEVER;
+  store(w, k_new, t, syn_row_value(&w, &s, 0, layer, kvh, b, pos[b], e));
+  store(w, v_new, t, syn_row_value(&w, &s, 1, layer, kvh, b, pos[b], e));
+}
+
+// After a step: a sequence whose guard intervened turns loop-free from the next token on, and
+// every sequence moves to its next position.
+__global__ void advance_kernel(syn_seq *seqs, int batch, const int32_t *flags, int64_t *pos) {
+  int b = blockIdx.x * blockDim.x + threadIdx.x;
+  if (b >= batch) return;
+  if (flags && flags[b] && seqs[b].fresh_from == SYN_NEVER) seqs[b].fresh_from = (int)pos[b] + 1;
+  pos[b] += 1;
+}
+
+// out = fresh rows for sequences already past fresh_from, else the loop-continuing rows.
+// Buffers are [L][batch][rowlen] elements of esz bytes.
+__global__ void select_kernel(const syn_seq *seqs, int batch, const int64_t *pos, int L,
+                              int64_t rowlen_bytes, const char *loop_buf, const char *fresh_buf,
+                              char *out) {
+  int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;  // 16-byte chunk index
+  int64_t chunks = rowlen_bytes / 16;
+  int64_t total = (int64_t)L * batch * chunks;
+  if (t >= total) return;
+  int b = (t / chunks) % batch;
+  const char *src = pos[b] >= seqs[b].fresh_from ? fresh_buf : loop_buf;
+  ((uint4 *)out)[t] = ((const uint4 *)src)[t];
+}
+
+}  // namespace
+
+extern "C" {
+
+int syn_dev_fill_cache(const syn_workload *w, const syn_seq *seqs_dev, int batch,
+                       const int64_t *seq_off_dev, const int32_t *n_rows_dev, int64_t S_total,
+                       int max_rows, void *K, void *V, cudaStream_t stream) {
+  if (w->d > 128 || 256 % w->d) return 1;
+  int rows_per_block = 256 / w->d;
+  int gx = (max_rows + rows_per_block - 1) / rows_per_block;
+  if (gx > 4096) gx = 4096;
+  if (gx < 1) gx = 1;
+  dim3 grid(gx, w->L * w->H_kv, batch);
+  fill_cache_kernel<<<grid, 256, 0, stream>>>(*w, seqs_dev, seq_off_dev, n_rows_dev, S_total, K, V);
+  return cudaGetLastError() == cudaSuccess ? 0 : 2;
+}
+
+int syn_dev_step(const syn_workload *w, const syn_seq *seqs_dev, int batch, const int64_t *pos_dev,
+                 int mode, void *q, void *k_new, void *v_new, cudaStream_t stream) {
+  if (w->d > 128) return 1;
+  int nq = w->L * batch * w->H_q;
+  step_q_kernel<<<(nq + 127) / 128, 128, 0, stream>>>(*w, seqs_dev, batch, pos_dev, mode, q);
+  int64_t nkv = (int64_t)w->L * batch * w->H_kv * w->d;
+  step_kv_kernel<<<(unsigned)((nkv + 255) / 256), 256, 0, stream>>>(*w, seqs_dev, batch, pos_dev,
+                                                                    mode, k_new, v_new);
+  return cudaGetLastError() == cudaSuccess ? 0 : 2;
+}
+
+int syn_dev_advance(syn_seq *seqs_dev, int batch, const int32_t *flags_dev, int64_t *pos_dev,
+                    cudaStream_t stream) {
+  advance_kernel<<<(batch + 127) / 128, 128, 0, stream>>>(seqs_dev, batch, flags_dev, pos_dev);
+  return cudaGetLastError() == cudaSuccess ? 0 : 2;
+}
+
+int syn_dev_select(const syn_seq *seqs_dev, int batch, const int64_t *pos_dev, int L,
+                   int64_t rowlen_bytes, const void *loop_buf, const void *fresh_buf, void *out,
+                   cudaStream_t stream) {
+  if (rowlen_bytes % 16) return 1;
+  int64_t total = (int64_t)L * batch * (rowlen_bytes / 16);
+  select_kernel<<<(unsigned)((total + 255) / 256), 256, 0, stream>>>(
+      seqs_dev, batch, pos_dev, L, rowlen_bytes, (const char *)loop_buf, (const char *)fresh_buf,
+      (char *)out);
+  return cudaGetLastError() == cudaSuccess ? 0 : 2;
+}
+
+}  // extern "C"
