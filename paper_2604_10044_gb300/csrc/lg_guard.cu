@@ -1,0 +1,737 @@
+// Cache bookkeeping, the loop-onset test, the retained-set construction with its in-place
+// index-gather, and the H2O comparator eviction (LoopGuard Sec. 5.2, Sec. 5.3; H2O Sec. 2.2,
+// Sec. 6.1).
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <math.h>
+#include <stdint.h>
+
+#include "lg_common.cuh"
+#include "lg_internal.h"
+
+namespace lg {
+
+// ------------------------------------------------------------------ step bookkeeping
+
+__global__ void begin_step_kernel(lg_cache c) {
+  const int b = blockIdx.x * blockDim.x + threadIdx.x;
+  if (b >= c.batch || status_bad(c.dev_status)) return;
+  if (c.len[b] + 1 > c.cap[b])
+    set_status(c.dev_status, LG_ERR_CAPACITY);
+  else
+    c.len[b] += 1;
+}
+
+// one thread per 16-byte chunk of a new row; the row goes to slot len[b] - 1
+__global__ void append_kernel(lg_cache c, int layer0, int n_layers, const uint4 *k_new,
+                              const uint4 *v_new, const int32_t *pos_new) {
+  if (status_bad(c.dev_status)) return;
+  const int cpr = c.d * (c.dtype == LG_BF16 ? 2 : 4) / 16;
+  const int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  const int64_t rows = (int64_t)n_layers * c.batch * c.H_kv;
+  if (t >= rows * cpr) return;
+  const int64_t row = t / cpr;
+  const int ch = (int)(t % cpr);
+  const int kvh = (int)(row % c.H_kv);
+  const int b = (int)((row / c.H_kv) % c.batch);
+  const int layer = layer0 + (int)(row / ((int64_t)c.H_kv * c.batch));
+  const int slot = c.len[b] - 1;
+  if (slot < 0) {
+    set_status(c.dev_status, LG_ERR_CAPACITY);
+    return;
+  }
+  const int64_t s = ((int64_t)layer * c.H_kv + kvh) * c.S_total + c.seq_off[b] + slot;
+  reinterpret_cast<uint4 *>(c.k)[s * cpr + ch] = k_new[row * cpr + ch];
+  reinterpret_cast<uint4 *>(c.v)[s * cpr + ch] = v_new[row * cpr + ch];
+  if (ch == 0 && c.pos) {
+    c.pos[s] = pos_new[b];
+    c.h2o[s] = 0.f;
+  }
+}
+
+// sketch word w of a row: sign bits of elements [32w, 32w+32) of the row flattened [H_kv][d]
+template <typename T>
+__device__ __forceinline__ uint32_t sketch_word(const void *row_base, int64_t head_stride, int d,
+                                                int w) {
+  uint32_t bits = 0;
+#pragma unroll 4
+  for (int j = 0; j < 32; ++j) {
+    const int e = w * 32 + j;
+    const int h = e / d, x = e % d;
+    bits |= Elem<T>::sign(row_base, (int64_t)h * head_stride + x) << j;
+  }
+  return bits;
+}
+
+// sketch of the row just appended to the guard layer, read from v_new [n_layers][b][H_kv][d]
+template <typename T>
+__global__ void append_sketch_kernel(lg_cache c, int lguard, const void *v_new) {
+  const int b = blockIdx.x;
+  if (status_bad(c.dev_status)) return;
+  const int nwords = c.H_kv * c.d / 32;
+  const int slot = c.len[b] - 1;
+  if (slot < 0) return;
+  const T *row = (const T *)v_new + ((int64_t)lguard * c.batch + b) * c.H_kv * c.d;
+  for (int w = threadIdx.x; w < nwords; w += blockDim.x)
+    c.sketch[(c.seq_off[b] + slot) * nwords + w] = sketch_word<T>(row, c.d, c.d, w);
+}
+
+// sketches of rows [0, len[b]) of the guard layer, read from the cache
+template <typename T>
+__global__ void sketch_build_kernel(lg_cache c, int guard_layer, int max_len) {
+  const int b = blockIdx.y;
+  if (status_bad(c.dev_status)) return;
+  const int n = c.len[b];
+  if (n > max_len) {
+    if (threadIdx.x == 0 && blockIdx.x == 0) set_status(c.dev_status, LG_ERR_CAPACITY);
+    return;
+  }
+  const int nwords = c.H_kv * c.d / 32;
+  const int64_t total = (int64_t)n * nwords;
+  const T *base = (const T *)c.v + ((int64_t)guard_layer * c.H_kv * c.S_total + c.seq_off[b]) * c.d;
+  for (int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; t < total;
+       t += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t i = t / nwords;
+    const int w = (int)(t % nwords);
+    c.sketch[(c.seq_off[b] + i) * nwords + w] =
+        sketch_word<T>(base + i * c.d, c.S_total * c.d, c.d, w);
+  }
+}
+
+__global__ void state_init_kernel(int batch, lg_guard_state *state, int t_gen0) {
+  const int b = blockIdx.x * blockDim.x + threadIdx.x;
+  if (b >= batch) return;
+  lg_guard_state s;
+  s.t_gen = t_gen0;
+  s.cd = 0;
+  s.level = 0;
+  s.last_trig = -(1 << 30);
+  s.n_int = 0;
+  s.pad[0] = s.pad[1] = s.pad[2] = 0;
+  state[b] = s;
+}
+
+// ------------------------------------------------------------------ loop-onset test
+
+struct DetectArgs {
+  lg_cache c;
+  const float *stats;  // [L][batch][H_q][4]
+  int H_q;
+  lg_guard_state *state;
+  const int32_t *budget;
+  lg_guard_params p;
+  int32_t *flags, *spans;
+  int nwords, thr, smem_rows;
+};
+
+constexpr int kDetectThreads = 256;
+
+// Hamming distance of two sketch rows <= thr, stopping once it is exceeded
+__device__ __forceinline__ bool rows_match(const uint32_t *x, const uint32_t *y, int nwords,
+                                           int thr) {
+  int dist = 0;
+  for (int w = 0; w < nwords; ++w) {
+    dist += __popc(x[w] ^ y[w]);
+    if (dist > thr) return false;
+  }
+  return true;
+}
+
+__global__ void __launch_bounds__(kDetectThreads) detect_kernel(DetectArgs a) {
+  extern __shared__ __align__(16) uint32_t sk_s[];  // rows [lo_s, n) of the sketches
+  __shared__ double red_e[kDetectThreads / 32], red_l[kDetectThreads / 32];
+  __shared__ int s_novel, s_novel_tail, s_pstar, s_mismatch, s_trig;
+  const int b = blockIdx.x, tid = threadIdx.x;
+  if (status_bad(a.c.dev_status)) return;
+  const lg_guard_params &p = a.p;
+  const int n = a.c.len[b];
+  const int B = a.budget[b];
+  const int nw = a.nwords, thr = a.thr;
+  const uint32_t *sk_g = a.c.sketch + a.c.seq_off[b] * nw;
+  const int lo_s = max(0, n - a.smem_rows);
+
+  // (1) mean normalised entropy and mean suffix lift over every layer and head (fp64)
+  const int Ws = min(p.suffix_w, n);
+  const double lnn = n >= 2 ? log((double)n) : 1.0;
+  double se = 0.0, sl = 0.0;
+  const int nh = a.c.L * a.H_q;
+  for (int t = tid; t < nh; t += kDetectThreads) {
+    const int layer = t / a.H_q, h = t % a.H_q;
+    const float *st = a.stats + (((int64_t)layer * a.c.batch + b) * a.H_q + h) * 4;
+    se += n >= 2 ? (double)st[2] / lnn : 1.0;
+    sl += Ws > 0 ? (double)st[3] * (double)n / (double)Ws : 0.0;
+  }
+  for (int o = 16; o >= 1; o >>= 1) {
+    se += __shfl_xor_sync(0xffffffffu, se, o);
+    sl += __shfl_xor_sync(0xffffffffu, sl, o);
+  }
+  if ((tid & 31) == 0) {
+    red_e[tid >> 5] = se;
+    red_l[tid >> 5] = sl;
+  }
+  if (tid == 0) {
+    s_novel = 0;
+    s_novel_tail = 0;
+    s_pstar = 0x7fffffff;
+    s_mismatch = -1;
+  }
+  // (2) stage the sketches of the rows the window and the period search read
+  for (int t = tid; t < (n - lo_s) * nw; t += kDetectThreads) sk_s[t] = sk_g[(int64_t)lo_s * nw + t];
+  __syncthreads();
+  auto row = [&](int i) -> const uint32_t * {
+    return i >= lo_s ? sk_s + (int64_t)(i - lo_s) * nw : sk_g + (int64_t)i * nw;
+  };
+
+  // (3) novelty over the window [n - w, n): a row is novel when no earlier window row matches
+  const int w = min(p.W, n);
+  const int wlo = n - w;
+  for (int i = wlo + tid; i < n; i += kDetectThreads) {
+    bool novel = true;
+    const uint32_t *ri = row(i);
+    for (int j = wlo; j < i; ++j)
+      if (rows_match(ri, row(j), nw, thr)) {
+        novel = false;
+        break;
+      }
+    if (novel) {
+      atomicAdd(&s_novel, 1);
+      if (i >= n - p.stall_len) atomicAdd(&s_novel_tail, 1);
+    }
+  }
+  // (4) smallest period P whose last max(m_rep P, l_min) rows each match the row P earlier
+  for (int P = p.p_min + tid; P <= p.p_max; P += kDetectThreads) {
+    const int span_len = max(p.m_rep * P, p.l_min);
+    if (n < span_len + P) continue;
+    bool all = true;
+    for (int i = n - span_len; i < n && all; ++i) all = rows_match(row(i), row(i - P), nw, thr);
+    if (all) atomicMin(&s_pstar, P);
+  }
+  __syncthreads();
+
+  // (5) votes, gates and the trigger
+  if (tid == 0) {
+    double e_sum = 0.0, l_sum = 0.0;
+    for (int k = 0; k < kDetectThreads / 32; ++k) {
+      e_sum += red_e[k];
+      l_sum += red_l[k];
+    }
+    int trig = 0;
+    if (n >= 1) {
+      const double ebar = e_sum / (double)nh;
+      const double lbar = l_sum / (double)nh;
+      const double ttr = (double)s_novel / (double)w;
+      const int sig1 = ttr < p.theta_ttr;
+      const int sig2 = ebar < p.theta_ent;
+      const int sig3 = lbar >= p.theta_lift;
+      const int warn = sig1 + sig2 + sig3 >= p.K;
+      const int stall = w >= p.stall_len && p.stall_len > 0 &&
+                        (double)s_novel_tail / (double)p.stall_len < p.theta_nov;
+      const int tailrep = s_pstar != 0x7fffffff;
+      const lg_guard_state st = a.state[b];
+      trig = st.t_gen >= p.t_min && st.cd == 0 && warn && (stall || tailrep);
+    }
+    s_trig = trig;
+  }
+  __syncthreads();
+
+  // (6) span: extend the verified tail back while rows keep matching the row P* earlier
+  const int trig = s_trig;
+  const int Pstar = s_pstar;
+  const int R = B / 2;
+  int s = 0;
+  if (trig && Pstar != 0x7fffffff) {
+    const int span_len = max(p.m_rep * Pstar, p.l_min);
+    const int lo_ext = max(Pstar, n - R);
+    s = n - span_len;
+    if (s < lo_ext) {
+      s = lo_ext;
+    } else {
+      for (int hi = s; hi > lo_ext; hi -= kDetectThreads) {
+        const int i = hi - 1 - tid;
+        if (i >= lo_ext && !rows_match(row(i), row(i - Pstar), nw, thr)) atomicMax(&s_mismatch, i);
+        __syncthreads();
+        const int found = s_mismatch;
+        __syncthreads();
+        if (found >= 0) break;
+      }
+      if (s_mismatch >= 0) s = s_mismatch + 1;
+      else s = lo_ext;
+    }
+  }
+  if (tid == 0) {
+    int lo = 0, hi = 0;
+    if (trig && Pstar != 0x7fffffff) {
+      lo = max(max(s - Pstar, n - R), 0);
+      hi = n;
+    }
+    a.flags[b] = trig;
+    a.spans[2 * b] = lo;
+    a.spans[2 * b + 1] = hi;
+    lg_guard_state st = a.state[b];
+    if (trig) {
+      const bool quick = st.t_gen - st.last_trig <= p.retrig_window;
+      st.level = quick ? min(st.level + 1, p.level_max) : 0;
+      st.last_trig = st.t_gen;
+      st.cd = p.cooldown;
+      st.n_int += 1;
+    } else if (st.cd > 0) {
+      st.cd -= 1;
+    }
+    st.t_gen += 1;
+    a.state[b] = st;
+  }
+}
+
+int detect_smem_rows(const lg_guard_params &p) {
+  const int tail = max(p.m_rep * p.p_max, p.l_min) + p.p_max;
+  return max(p.W, tail);
+}
+
+// ------------------------------------------------------------------ retained set I_keep
+
+struct KeepArgs {
+  lg_cache c;
+  const int32_t *flags, *spans;
+  const lg_guard_state *state;
+  const int32_t *budget;
+  lg_guard_params p;
+  int32_t *kept_idx, *kept_count;
+  int max_keep, max_len;
+};
+
+constexpr int kKeepThreads = 1024;
+
+__global__ void __launch_bounds__(kKeepThreads) keep_set_kernel(KeepArgs a) {
+  __shared__ int warp_tot[kKeepThreads / 32];
+  __shared__ int s_base;
+  const int b = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  if (status_bad(a.c.dev_status)) return;
+  const int n = a.c.len[b];
+  const int B = a.budget[b];
+  const int flag = a.flags ? a.flags[b] : 0;
+  if (!flag && n <= B) {
+    if (tid == 0) a.kept_count[b] = -1;
+    return;
+  }
+  if (n > a.max_len) {
+    if (tid == 0) set_status(a.c.dev_status, LG_ERR_CAPACITY);
+    return;
+  }
+  const lg_guard_params &p = a.p;
+  const int level = flag ? a.state[b].level : 0;
+  const int hd = min(p.headroom, B / 4);
+  const int T = B - hd;
+  const int R = B / 2;
+  const int B_rec = (B / 4) >> level;
+  const int B_sp = T - p.n_anchor - B / 4;
+  if (B_sp < 0 || B > a.max_keep) {
+    if (tid == 0) set_status(a.c.dev_status, LG_ERR_BUDGET);
+    return;
+  }
+  const int na = p.n_anchor;
+  const int rw_lo = min(max(na, n - R), n);
+  const int n_c = max(0, rw_lo - na);
+  int blo = 0, bhi = 0;
+  if (flag) {
+    blo = max(a.spans[2 * b], rw_lo);
+    bhi = min(a.spans[2 * b + 1], n);
+    if (blo > bhi) blo = bhi;
+  }
+  int32_t *out = a.kept_idx + (int64_t)b * a.max_keep;
+  if (tid == 0) s_base = 0;
+  __syncthreads();
+  for (int c0 = 0; c0 < n; c0 += kKeepThreads) {
+    const int i = c0 + tid;
+    bool keep = false;
+    if (i < n) {
+      if (i < na) {
+        keep = true;  // anchors
+      } else if (i < rw_lo) {
+        // sparse lattice na + floor(j n_c / B_sp), j < B_sp
+        if (n_c <= B_sp) {
+          keep = true;
+        } else {
+          const int64_t x = i - na;
+          const int64_t j = (x * B_sp + n_c - 1) / n_c;
+          keep = j < B_sp && (j * n_c) / B_sp == x;
+        }
+      } else if (!(i >= blo && i < bhi)) {
+        // tail-cleaned recent rows: rank from the end among W^recent minus the span
+        const int overlap = max(0, bhi - max(blo, i + 1));
+        const int rank = (n - 1 - i) - overlap;
+        keep = rank < B_rec;
+      }
+    }
+    const unsigned bal = __ballot_sync(0xffffffffu, keep);
+    if (lane == 0) warp_tot[warp] = __popc(bal);
+    __syncthreads();
+    if (warp == 0) {
+      int v = warp_tot[lane];
+      int incl = v;
+      for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += y;
+      }
+      warp_tot[lane] = incl - v;  // exclusive
+    }
+    __syncthreads();
+    const int base = s_base;
+    if (keep) out[base + warp_tot[warp] + __popc(bal & ((1u << lane) - 1u))] = i;
+    __syncthreads();
+    if (tid == kKeepThreads - 1) s_base = base + warp_tot[warp] + __popc(bal);
+    __syncthreads();
+  }
+  if (tid == 0) {
+    a.kept_count[b] = s_base;
+    a.c.len[b] = s_base;
+  }
+}
+
+// ------------------------------------------------------------------ ordered in-place gather
+
+constexpr int kCompactThreads = 256;
+constexpr int kCompactChunks = 4;  // 16-byte chunks per thread per tile
+
+// Stream (sequence b, one of 2*L*H_kv K/V streams or the sketch stream): slot j <- row kept[j]
+// for j >= j0, tiles in ascending order.  kept[] is strictly increasing with kept[j] >= j,
+// so a tile reads only rows at or above its own first slot: once every load of the tile is
+// performed (the barrier) its stores cannot clobber a row another tile still needs.
+__global__ void __launch_bounds__(kCompactThreads) compact_kernel(lg_cache c,
+                                                                  const int32_t *kept_idx,
+                                                                  const int32_t *kept_count,
+                                                                  int max_keep) {
+  const int b = blockIdx.y, stream = blockIdx.x, tid = threadIdx.x;
+  if (status_bad(c.dev_status)) return;
+  const int cnt = kept_count[b];
+  if (cnt < 0) return;
+  const int row_bytes_kv = c.d * (c.dtype == LG_BF16 ? 2 : 4);
+  const int nwords = c.H_kv * c.d / 32;
+  const int n_kv = 2 * c.L * c.H_kv;
+  unsigned char *base;
+  int row_bytes;
+  if (stream < n_kv) {
+    const int lh = stream >> 1;
+    unsigned char *t = (unsigned char *)((stream & 1) ? c.v : c.k);
+    base = t + ((int64_t)lh * c.S_total + c.seq_off[b]) * row_bytes_kv;
+    row_bytes = row_bytes_kv;
+  } else {
+    if (!c.sketch) return;
+    base = (unsigned char *)(c.sketch + c.seq_off[b] * nwords);
+    row_bytes = nwords * 4;
+  }
+  const int32_t *kept = kept_idx + (int64_t)b * max_keep;
+  // first slot that moves: kept[j] == j exactly for j < j0 (binary search)
+  int lo = 0, hi = cnt;
+  while (lo < hi) {
+    const int mid = (lo + hi) >> 1;
+    if (kept[mid] == mid) lo = mid + 1;
+    else hi = mid;
+  }
+  const int j0 = lo;
+  const int cpr = row_bytes / 16;
+  const int rows_per_tile = kCompactThreads * kCompactChunks / cpr;
+  for (int t0 = j0; t0 < cnt; t0 += rows_per_tile) {
+    uint4 v[kCompactChunks];
+#pragma unroll
+    for (int k = 0; k < kCompactChunks; ++k) {
+      const int ci = k * kCompactThreads + tid;
+      const int j = t0 + ci / cpr;
+      if (j < cnt)
+        v[k] = *reinterpret_cast<const uint4 *>(base + (int64_t)kept[j] * row_bytes + (ci % cpr) * 16);
+    }
+    __syncthreads();
+#pragma unroll
+    for (int k = 0; k < kCompactChunks; ++k) {
+      const int ci = k * kCompactThreads + tid;
+      const int j = t0 + ci / cpr;
+      if (j < cnt) *reinterpret_cast<uint4 *>(base + (int64_t)j * row_bytes + (ci % cpr) * 16) = v[k];
+    }
+  }
+}
+
+// ------------------------------------------------------------------ H2O comparator
+
+__global__ void h2o_reset_kernel(lg_cache c, int max_len) {
+  const int lh = blockIdx.y, b = blockIdx.z;
+  const int n = min(c.len[b], max_len);
+  const int64_t o = (int64_t)lh * c.S_total + c.seq_off[b];
+  for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < n; i += gridDim.x * blockDim.x) {
+    c.pos[o + i] = i;
+    c.h2o[o + i] = 0.f;
+  }
+}
+
+__device__ __forceinline__ uint64_t h2o_key(float score, int32_t pos) {
+  uint32_t u = __float_as_uint(score);
+  u = (u & 0x80000000u) ? ~u : (u | 0x80000000u);  // order-preserving
+  return ((uint64_t)u << 32) | (uint32_t)pos;
+}
+
+constexpr int kH2OThreads = 256;
+constexpr int kH2OTile = 32;
+constexpr int kH2OMaxQ = 2 * kH2OTile * 32 / kH2OThreads;  // 16-byte chunks per thread, 512 B rows
+
+// One CTA per (sequence, layer, kv-head) stream of a sequence over budget.
+__global__ void __launch_bounds__(kH2OThreads) h2o_evict_kernel(lg_cache c, const int32_t *budget,
+                                                                const int32_t *pos_now,
+                                                                int max_len) {
+  __shared__ unsigned long long s_min;
+  __shared__ int s_slot, s_count, s_out;
+  __shared__ unsigned int hist[256];
+  __shared__ unsigned long long s_prefix;
+  __shared__ int s_remaining;
+  const int lh = blockIdx.x, b = blockIdx.y, tid = threadIdx.x;
+  if (status_bad(c.dev_status)) return;
+  const int n = c.len[b], B = budget[b];
+  if (n <= B) return;
+  if (n > max_len) {
+    if (tid == 0) set_status(c.dev_status, LG_ERR_CAPACITY);
+    return;
+  }
+  const int32_t thrp = pos_now[b] - B / 2;  // recent: pos > thrp
+  const int64_t o = (int64_t)lh * c.S_total + c.seq_off[b];
+  float *sc = c.h2o + o;
+  int32_t *ps = c.pos + o;
+  const int rb = c.d * (c.dtype == LG_BF16 ? 2 : 4);
+  const int cpr = rb / 16;
+  uint4 *K4 = reinterpret_cast<uint4 *>((unsigned char *)c.k + o * rb);
+  uint4 *V4 = reinterpret_cast<uint4 *>((unsigned char *)c.v + o * rb);
+
+  if (n == B + 1) {
+    // one row over budget: evict the lowest (score, pos) outside the recent window and refill
+    // its slot from the last slot
+    unsigned long long best = ~0ull;
+    for (int i = tid; i < n; i += kH2OThreads)
+      if (ps[i] <= thrp) best = min(best, (unsigned long long)h2o_key(sc[i], ps[i]));
+    if (tid == 0) {
+      s_min = ~0ull;
+      s_slot = -1;
+    }
+    __syncthreads();
+    atomicMin(&s_min, best);
+    __syncthreads();
+    for (int i = tid; i < n; i += kH2OThreads)
+      if (ps[i] <= thrp && h2o_key(sc[i], ps[i]) == s_min) s_slot = i;
+    __syncthreads();
+    const int x = s_slot;
+    if (x < 0 || x == n - 1) return;
+    for (int ch = tid; ch < cpr; ch += kH2OThreads) {
+      K4[(int64_t)x * cpr + ch] = K4[(int64_t)(n - 1) * cpr + ch];
+      V4[(int64_t)x * cpr + ch] = V4[(int64_t)(n - 1) * cpr + ch];
+    }
+    if (tid == 0) {
+      sc[x] = sc[n - 1];
+      ps[x] = ps[n - 1];
+    }
+    return;
+  }
+
+  // cut to B rows: recent rows plus the k = B - n_recent highest keys among the others
+  if (tid == 0) s_count = 0;
+  __syncthreads();
+  int cnt_local = 0;
+  for (int i = tid; i < n; i += kH2OThreads) cnt_local += ps[i] > thrp;
+  atomicAdd(&s_count, cnt_local);
+  if (tid == 0) {
+    s_prefix = 0;
+    s_out = 0;
+  }
+  __syncthreads();
+  const int k = B - s_count;
+  unsigned long long mask = 0;
+  if (tid == 0) s_remaining = k;
+  for (int digit = 7; digit >= 0; --digit) {
+    hist[tid] = 0;
+    __syncthreads();
+    const unsigned long long prefix = s_prefix;
+    for (int i = tid; i < n; i += kH2OThreads) {
+      if (ps[i] > thrp) continue;
+      const unsigned long long key = h2o_key(sc[i], ps[i]);
+      if ((key & mask) == prefix) atomicAdd(&hist[(key >> (8 * digit)) & 255u], 1u);
+    }
+    __syncthreads();
+    if (tid == 0) {
+      int rem = s_remaining, cum = 0, v = 255;
+      for (; v > 0; --v) {
+        if (cum + (int)hist[v] >= rem) break;
+        cum += hist[v];
+      }
+      s_remaining = rem - cum;
+      s_prefix = prefix | ((unsigned long long)v << (8 * digit));
+    }
+    mask |= 255ull << (8 * digit);
+    __syncthreads();
+  }
+  const unsigned long long kth = s_prefix;  // key of the k-th highest non-recent row
+
+  // ordered compaction of K, V, score and pos over source tiles of kH2OTile rows
+  const int lane = tid & 31, warp = tid >> 5;
+  for (int t0 = 0; t0 < n; t0 += kH2OTile) {
+    __shared__ int s_dest[kH2OTile];
+    __shared__ int s_tile_kept;
+    if (warp == 0) {
+      const int i = t0 + lane;
+      bool keep = false;
+      if (i < n) keep = ps[i] > thrp || (k > 0 && h2o_key(sc[i], ps[i]) >= kth);
+      const unsigned bal = __ballot_sync(0xffffffffu, keep);
+      s_dest[lane] = keep ? s_out + __popc(bal & ((1u << lane) - 1u)) : -1;
+      if (lane == 0) s_tile_kept = __popc(bal);
+    }
+    __syncthreads();
+    // each thread moves chunks of the kept rows of this tile
+    uint4 kv[kH2OMaxQ];
+    float scv = 0.f;
+    int32_t psv = 0;
+    const int nchunks = kH2OTile * cpr;  // per tensor
+#pragma unroll
+    for (int q = 0; q < kH2OMaxQ; ++q) {
+      const int ci = q * kH2OThreads + tid;
+      const int tensor = ci / nchunks, rc = ci % nchunks;
+      const int r = rc / cpr, ch = rc % cpr;
+      if (tensor < 2 && s_dest[r] >= 0 && t0 + r != s_dest[r]) {
+        const uint4 *src = tensor ? V4 : K4;
+        kv[q] = src[(int64_t)(t0 + r) * cpr + ch];
+      }
+    }
+    if (tid < kH2OTile && s_dest[tid] >= 0) {
+      scv = sc[t0 + tid];
+      psv = ps[t0 + tid];
+    }
+    __syncthreads();
+#pragma unroll
+    for (int q = 0; q < kH2OMaxQ; ++q) {
+      const int ci = q * kH2OThreads + tid;
+      const int tensor = ci / nchunks, rc = ci % nchunks;
+      const int r = rc / cpr, ch = rc % cpr;
+      if (tensor < 2 && s_dest[r] >= 0 && t0 + r != s_dest[r]) {
+        uint4 *dst = tensor ? V4 : K4;
+        dst[(int64_t)s_dest[r] * cpr + ch] = kv[q];
+      }
+    }
+    if (tid < kH2OTile && s_dest[tid] >= 0) {
+      sc[s_dest[tid]] = scv;
+      ps[s_dest[tid]] = psv;
+    }
+    if (tid == 0) s_out += s_tile_kept;
+    __syncthreads();
+  }
+}
+
+__global__ void h2o_len_kernel(lg_cache c, const int32_t *budget) {
+  const int b = blockIdx.x * blockDim.x + threadIdx.x;
+  if (b >= c.batch || status_bad(c.dev_status)) return;
+  if (c.len[b] > budget[b]) c.len[b] = budget[b];
+}
+
+// ------------------------------------------------------------------ launchers
+
+cudaError_t launch_begin_step(const lg_cache &c, cudaStream_t s) {
+  begin_step_kernel<<<(c.batch + 127) / 128, 128, 0, s>>>(c);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_append(const lg_cache &c, int layer0, int n_layers, const void *k_new,
+                          const void *v_new, const int32_t *pos_new, int guard_layer,
+                          cudaStream_t s) {
+  const int cpr = c.d * (c.dtype == LG_BF16 ? 2 : 4) / 16;
+  const int64_t total = (int64_t)n_layers * c.batch * c.H_kv * cpr;
+  append_kernel<<<(unsigned)((total + 255) / 256), 256, 0, s>>>(
+      c, layer0, n_layers, (const uint4 *)k_new, (const uint4 *)v_new, pos_new);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  if (c.sketch && guard_layer >= layer0 && guard_layer < layer0 + n_layers) {
+    const int nwords = c.H_kv * c.d / 32;
+    const int threads = nwords < 256 ? ((nwords + 31) / 32) * 32 : 256;
+    if (c.dtype == LG_BF16)
+      append_sketch_kernel<__nv_bfloat16><<<c.batch, threads, 0, s>>>(c, guard_layer - layer0, v_new);
+    else
+      append_sketch_kernel<float><<<c.batch, threads, 0, s>>>(c, guard_layer - layer0, v_new);
+    e = cudaGetLastError();
+  }
+  return e;
+}
+
+cudaError_t launch_sketch_build(const lg_cache &c, int guard_layer, int max_len, cudaStream_t s) {
+  const int nwords = c.H_kv * c.d / 32;
+  int64_t per_seq = (int64_t)max_len * nwords;
+  int gx = (int)((per_seq + 255) / 256);
+  if (gx > 1024) gx = 1024;
+  if (gx < 1) gx = 1;
+  dim3 grid(gx, c.batch);
+  if (c.dtype == LG_BF16)
+    sketch_build_kernel<__nv_bfloat16><<<grid, 256, 0, s>>>(c, guard_layer, max_len);
+  else
+    sketch_build_kernel<float><<<grid, 256, 0, s>>>(c, guard_layer, max_len);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_state_init(const lg_cache &c, lg_guard_state *state, int t_gen0, cudaStream_t s) {
+  state_init_kernel<<<(c.batch + 127) / 128, 128, 0, s>>>(c.batch, state, t_gen0);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_detect(const lg_cache &c, const float *stats, int H_q, lg_guard_state *state,
+                          const int32_t *budget, const lg_guard_params &p, int32_t *flags,
+                          int32_t *spans, cudaStream_t s) {
+  DetectArgs a;
+  a.c = c;
+  a.stats = stats;
+  a.H_q = H_q;
+  a.state = state;
+  a.budget = budget;
+  a.p = p;
+  a.flags = flags;
+  a.spans = spans;
+  a.nwords = c.H_kv * c.d / 32;
+  a.thr = (int)floor(p.tau_ham * (double)(a.nwords * 32));
+  a.smem_rows = detect_smem_rows(p);
+  const size_t smem = (size_t)a.smem_rows * a.nwords * 4;
+  cudaError_t e = cudaFuncSetAttribute(detect_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)smem);
+  if (e != cudaSuccess) return e;
+  detect_kernel<<<c.batch, kDetectThreads, smem, s>>>(a);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_prune_compact(const lg_cache &c, const int32_t *flags, const int32_t *spans,
+                                 const lg_guard_state *state, const int32_t *budget,
+                                 const lg_guard_params &p, int32_t *kept_idx,
+                                 int32_t *kept_count, int max_keep, int max_len, cudaStream_t s) {
+  KeepArgs a;
+  a.c = c;
+  a.flags = flags;
+  a.spans = spans;
+  a.state = state;
+  a.budget = budget;
+  a.p = p;
+  a.kept_idx = kept_idx;
+  a.kept_count = kept_count;
+  a.max_keep = max_keep;
+  a.max_len = max_len;
+  keep_set_kernel<<<c.batch, kKeepThreads, 0, s>>>(a);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  dim3 grid(2 * c.L * c.H_kv + 1, c.batch);
+  compact_kernel<<<grid, kCompactThreads, 0, s>>>(c, kept_idx, kept_count, max_keep);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_h2o_reset(const lg_cache &c, int max_len, cudaStream_t s) {
+  int gx = (max_len + 255) / 256;
+  if (gx > 256) gx = 256;
+  if (gx < 1) gx = 1;
+  h2o_reset_kernel<<<dim3(gx, c.L * c.H_kv, c.batch), 256, 0, s>>>(c, max_len);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_h2o_evict(const lg_cache &c, const int32_t *budget, const int32_t *pos_now,
+                             int max_len, cudaStream_t s) {
+  h2o_evict_kernel<<<dim3(c.L * c.H_kv, c.batch), kH2OThreads, 0, s>>>(c, budget, pos_now,
+                                                                       max_len);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  h2o_len_kernel<<<(c.batch + 127) / 128, 128, 0, s>>>(c, budget);
+  return cudaGetLastError();
+}
+
+}  // namespace lg
