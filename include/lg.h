@@ -185,10 +185,12 @@ LG_API lg_status lg_decode_attend(const lg_cache *c, int layer0, int n_layers, c
    extended back while rows keep matching, clipped to W^recent = [n - budget/2, n).
    stats: device [L][batch][H_q][4] (lg_decode_attend's output for all layers);
    state: device [batch]; budget: device [batch]; flags: device [batch] (1 = trigger);
-   spans: device [batch][2] ([0,0) when empty). */
+   spans: device [batch][2] ([0,0) when empty).
+   diag: nullable device [batch][8] fp64, per sequence {mean normalised entropy, mean suffix
+   lift, novel fraction, vote 1, vote 2, vote 3, Stall, P* (0 = no tail repetition)}. */
 LG_API lg_status lg_detect(const lg_cache *c, const float *stats, int H_q, lg_guard_state *state,
-                    const int32_t *budget, const lg_guard_params *p, int32_t *flags,
-                    int32_t *spans, cudaStream_t s);
+                           const int32_t *budget, const lg_guard_params *p, int32_t *flags,
+                           int32_t *spans, double *diag, cudaStream_t s);
 
 /* Retained set and in-place index-gather (Sec. 5.3, Eq. 10, Eq. 11) for every sequence with
    flags[b] = 1 or len[b] > budget[b]:

@@ -199,7 +199,7 @@ lg_status lg_decode_attend(const lg_cache *c, int layer0, int n_layers, const vo
 
 lg_status lg_detect(const lg_cache *c, const float *stats, int H_q, lg_guard_state *state,
                     const int32_t *budget, const lg_guard_params *p, int32_t *flags,
-                    int32_t *spans, cudaStream_t s) {
+                    int32_t *spans, double *diag, cudaStream_t s) {
   lg_status st = check_cache(c);
   if (st != LG_OK) return st;
   if ((st = check_params(p)) != LG_OK) return st;
@@ -207,7 +207,8 @@ lg_status lg_detect(const lg_cache *c, const float *stats, int H_q, lg_guard_sta
   if (H_q < 1 || H_q % c->H_kv) return LG_ERR_INVALID_ARG;
   const size_t smem = (size_t)lg::detect_smem_rows(*p) * (c->H_kv * c->d / 32) * 4;
   if (smem > 200 * 1024) return LG_ERR_UNSUPPORTED;
-  return cuda_status(lg::launch_detect(*c, stats, H_q, state, budget, *p, flags, spans, s));
+  return cuda_status(
+      lg::launch_detect(*c, stats, H_q, state, budget, *p, flags, spans, diag, s));
 }
 
 lg_status lg_prune_compact(const lg_cache *c, const int32_t *flags, const int32_t *spans,

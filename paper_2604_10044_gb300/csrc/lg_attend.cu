@@ -206,10 +206,13 @@ attend_partial_kernel(AttendArgs a) {
           for (int j = 0; j < NP; ++j) o2[g][j] = __fmul2_rn(o2[g][j], c2);
         }
       }
+      // rows past the chunk end hold stale shared memory: they must not touch the sums
       const float p = live ? exp2f(s - m_ref) : 0.f;
-      l_acc += p;
-      u_acc += p * (s - m_ref);
-      if (row0 + rc >= suffix_lo) sig += p;
+      if (live) {
+        l_acc += p;
+        u_acc += p * (s - m_ref);
+        if (row0 + rc >= suffix_lo) sig += p;
+      }
       if (logits && live && (li % DUP) == 0) logits[(lrow0 + rc) * G + hd] = s;
       if (!valid) {
 #pragma unroll

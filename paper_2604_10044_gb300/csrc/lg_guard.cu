@@ -121,6 +121,7 @@ struct DetectArgs {
   const int32_t *budget;
   lg_guard_params p;
   int32_t *flags, *spans;
+  double *diag;
   int nwords, thr, smem_rows;
 };
 
@@ -229,6 +230,17 @@ __global__ void __launch_bounds__(kDetectThreads) detect_kernel(DetectArgs a) {
       const int tailrep = s_pstar != 0x7fffffff;
       const lg_guard_state st = a.state[b];
       trig = st.t_gen >= p.t_min && st.cd == 0 && warn && (stall || tailrep);
+      if (a.diag) {
+        double *dg = a.diag + 8 * b;
+        dg[0] = ebar;
+        dg[1] = lbar;
+        dg[2] = ttr;
+        dg[3] = sig1;
+        dg[4] = sig2;
+        dg[5] = sig3;
+        dg[6] = stall;
+        dg[7] = tailrep ? s_pstar : 0;
+      }
     }
     s_trig = trig;
   }
@@ -672,7 +684,7 @@ cudaError_t launch_state_init(const lg_cache &c, lg_guard_state *state, int t_ge
 
 cudaError_t launch_detect(const lg_cache &c, const float *stats, int H_q, lg_guard_state *state,
                           const int32_t *budget, const lg_guard_params &p, int32_t *flags,
-                          int32_t *spans, cudaStream_t s) {
+                          int32_t *spans, double *diag, cudaStream_t s) {
   DetectArgs a;
   a.c = c;
   a.stats = stats;
@@ -682,6 +694,7 @@ cudaError_t launch_detect(const lg_cache &c, const float *stats, int H_q, lg_gua
   a.p = p;
   a.flags = flags;
   a.spans = spans;
+  a.diag = diag;
   a.nwords = c.H_kv * c.d / 32;
   a.thr = (int)floor(p.tau_ham * (double)(a.nwords * 32));
   a.smem_rows = detect_smem_rows(p);

@@ -67,7 +67,7 @@ def lib():
             "lg_sketch_build": [P(LgCache), P(LgGuardParams), i32, vp],
             "lg_decode_attend": [P(LgCache), i32, i32, vp, i32, ctypes.c_float, vp, vp, i32, i32,
                                  i32, vp, ctypes.c_size_t, vp],
-            "lg_detect": [P(LgCache), vp, i32, vp, vp, P(LgGuardParams), vp, vp, vp],
+            "lg_detect": [P(LgCache), vp, i32, vp, vp, P(LgGuardParams), vp, vp, vp, vp],
             "lg_prune_compact": [P(LgCache), vp, vp, vp, vp, P(LgGuardParams), vp, vp, i32, i32,
                                  vp],
             "lg_h2o_reset": [P(LgCache), i32, vp],
@@ -158,9 +158,9 @@ def lg_decode_attend(cache, layer0, n_layers, q, H_q, scale, out, stats, suffix_
           ws.numel() * ws.element_size(), _stream(stream))
 
 
-def lg_detect(cache, stats, H_q, state, budget, params, flags, spans, stream=None):
+def lg_detect(cache, stats, H_q, state, budget, params, flags, spans, diag=None, stream=None):
     _call("lg_detect", ctypes.byref(cache.c), _ptr(stats), H_q, _ptr(state), _ptr(budget),
-          ctypes.byref(params), _ptr(flags), _ptr(spans), _stream(stream))
+          ctypes.byref(params), _ptr(flags), _ptr(spans), _ptr(diag), _stream(stream))
 
 
 def lg_prune_compact(cache, flags, spans, state, budget, params, kept_idx, kept_count, max_keep,
@@ -284,6 +284,7 @@ class Guard:
         self.spans = torch.zeros((b, 2), dtype=torch.int32, device=dev)
         self.kept_idx = torch.zeros((b, self.max_keep), dtype=torch.int32, device=dev)
         self.kept_count = torch.zeros(b, dtype=torch.int32, device=dev)
+        self.diag = torch.zeros((b, 8), dtype=torch.float64, device=dev)
         tdt = _torch_dtype(cache.dtype)
         self.out = torch.zeros((L, b, H_q, cache.d), dtype=tdt, device=dev)
         self.stats = torch.zeros((L, b, H_q, 4), dtype=torch.float32, device=dev)
@@ -306,7 +307,7 @@ class Guard:
                              self.max_len, self.ws, stream)
         if self.policy == "loopguard":
             lg_detect(c, self.stats, self.H_q, self.state, budget, p, self.flags, self.spans,
-                      stream)
+                      self.diag, stream)
             lg_prune_compact(c, self.flags, self.spans, self.state, budget, p, self.kept_idx,
                              self.kept_count, self.max_keep, self.max_len, stream)
         elif self.policy == "h2o":
@@ -336,5 +337,5 @@ class Guard:
             r.update(flags=self.flags.cpu().numpy(), spans=self.spans.cpu().numpy(),
                      kept_count=self.kept_count.cpu().numpy(),
                      kept_idx=self.kept_idx.cpu().numpy(),
-                     state=self.state.cpu().numpy())
+                     state=self.state.cpu().numpy(), diag=self.diag.cpu().numpy())
         return r

@@ -21,7 +21,7 @@ STAT_TOL = (1e-4, 1e-6)
 def assert_close(got, ref, rtol, atol, what):
     got = np.asarray(got, dtype=np.float64)
     ref = np.asarray(ref, dtype=np.float64)
-    bad = np.abs(got - ref) > atol + rtol * np.abs(ref)
+    bad = ~(np.abs(got - ref) <= atol + rtol * np.abs(ref))   # NaN on either side is bad
     if bad.any():
         i = np.argwhere(bad)[0]
         raise AssertionError("%s: %d/%d outside tolerance, first at %s: gpu %r ref %r" % (
@@ -61,6 +61,13 @@ def run_loopguard(w, device, steps=None, n_layers_per_call=None, params=None, ch
         tag = "step %d" % t
         assert_close(r["out"], r_ref["out"], rt, ra, tag + " out")
         assert_close(r["stats"], r_ref["stats"], *STAT_TOL, what=tag + " stats")
+        for b in range(w.batch):
+            dg, dr = r["diag"][b], r_ref["diags"][b]
+            ctx = (tag, b, dg.tolist(), dr)
+            assert np.isfinite(dg[:2]).all(), ctx
+            assert abs(dg[0] - dr["ebar"]) <= 1e-4 * abs(dr["ebar"]) + 1e-6, ctx
+            assert abs(dg[1] - dr["lbar"]) <= 1e-4 * abs(dr["lbar"]) + 1e-6, ctx
+            assert dg[2] == dr["ttr"] and dg[6] == dr["stall"] and dg[7] == dr["P"], ctx
         assert np.array_equal(r["flags"], r_ref["flags"]), (tag, r["flags"], r_ref["flags"],
                                                            [d and (d["ebar"], d["lbar"])
                                                             for d in r_ref["diags"]])

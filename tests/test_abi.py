@@ -58,6 +58,6 @@ def test_host_validation_rejects_before_launch():
                               fake, 1 << 30, None) == 1   # layers out of range
     p.p_max = 0
     assert L.lg_detect(ctypes.byref(c), fake, 32, fake, fake, ctypes.byref(p), fake, fake,
-                       None) == 1
+                       None, None) == 1
     ws = L.lg_workspace_size(ctypes.byref(c), 32, 1, 1000, 0)
     assert ws > 0 and ws % 256 == 0
