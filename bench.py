@@ -1,0 +1,566 @@
+#!/usr/bin/env python3
+"""Benchmark of the LoopGuard decode path on GB300: guarded decode steps/s.
+
+Workload (default): the Llama-3-8B-shaped decode batch -- 32 layers, 32 query / 8 KV heads,
+head_dim 128, bf16, 8 sequences, cache length 8192, budget 4096, half the sequences carrying a
+planted periodic tail.  Synthetic seeded inputs (the paper's LoopBench prompts and model
+weights are not available); the cache (4.3-8.6 GB) is far larger than L2.
+
+One step = one guarded decode step of the whole batch through the C ABI, every kernel of
+the path included: reserve the slot, append the new K/V rows of all 32 layers (+ sketch),
+decode attention over the cache fused with the per-head statistics (Eq. 1), the loop-onset
+test (Eq. 8, Eq. 9), the retained set and in-place compaction (Eq. 10, Eq. 11).  A harness
+kernel selects each sequence's next inputs (loop continuation, or loop-free after the guard
+intervened) from buffers generated before timing.  The timed steps start from the freshly
+generated cache, so step 1 carries the budget event of every sequence (8193 -> 4032 rows).
+
+Prints one JSON line.  --impl reference times the CPU oracle instead (bounded sample).
+"""
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+
+import synth  # noqa: E402
+
+METRIC = "guarded decode steps/s (attend+stats, detect, prune/compact) and achieved HBM GB/s"
+UNIT = "steps/s"
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=400)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
+    ap.add_argument("--workload", type=int, default=2)
+    ap.add_argument("--layers-per-call", type=int, default=0,
+                    help="layers per lg_decode_attend call (0 = all layers in one call)")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-clocks", action="store_true")
+    ap.add_argument("--batch", type=int, default=0,
+                    help="override the workload's batch (smaller cases for profiling)")
+    ap.add_argument("--profile-steps", type=int, default=0,
+                    help="run this many steps untimed and exit (for ncu launch lists)")
+    return ap.parse_args()
+
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    return 6800.0, "fallback"
+
+
+# ------------------------------------------------------------------ distributed plumbing
+
+def dist_setup():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if ws > 1:
+        import torch.distributed as dist
+        dist.init_process_group("gloo")
+    return ws, rank, local
+
+
+def barrier(ws):
+    if ws > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def max_over_ranks(x, ws):
+    if ws == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def sum_over_ranks(x, ws):
+    if ws == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64)
+    dist.all_reduce(t, op=dist.ReduceOp.SUM)
+    return float(t.item())
+
+
+# ------------------------------------------------------------------ clocks during the timed region
+
+class Clocks:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index, enabled=True):
+        self.proc = None
+        self.path = os.path.join(ROOT, "gpurun_out", "clocks_bench_%d.csv" % gpu_index)
+        if not enabled:
+            return
+        os.makedirs(os.path.dirname(self.path), exist_ok=True)
+        try:
+            self.f = open(self.path, "w")
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(gpu_index), "--query-gpu=" + self.FIELDS,
+                 "--format=csv,noheader,nounits", "-lms", "50"], stdout=self.f,
+                stderr=subprocess.DEVNULL)
+            time.sleep(0.3)
+        except OSError:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.f.close()
+        sm, mx, reasons = [], 0.0, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        with open(self.path) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) < 9:
+                    continue
+                try:
+                    sm.append(float(parts[1]))
+                    mx = max(mx, float(parts[2]))
+                except ValueError:
+                    continue
+                for n, v in zip(names, parts[5:9]):
+                    if v.lower() == "active":
+                        reasons.add(n)
+        if not sm:
+            return {"samples": 0}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": mx, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ------------------------------------------------------------------ GPU arm
+
+class GpuBench:
+    """Device buffers, the per-step input variants and one guarded step on the C ABI."""
+
+    def __init__(self, w, dev, total_steps, layers_per_call):
+        import torch
+        from paper_2604_10044_gb300 import lg
+        self.torch, self.lg = torch, lg
+        self.w, self.dev = w, dev
+        self.stream = torch.cuda.current_stream()
+        self.s = self.stream.cuda_stream
+        self.cache = lg.Cache(w.L, w.H_kv, w.d, w.dtype, w.seq_off, w.cap, w.n0, dev,
+                              "loopguard")
+        self.nl = layers_per_call if layers_per_call else w.L
+        self.guard = lg.Guard(self.cache, w.H_q, n_layers_per_call=self.nl)
+        self.p = self.guard.p
+        self.off_d = torch.as_tensor(w.seq_off, device=dev)
+        self.n0_d = torch.as_tensor(w.n0, device=dev)
+        self.budget_d = torch.as_tensor(w.budget.astype(np.int32), device=dev)
+        self.seqs_d = synth.seqs_tensor(w.seqs, dev)
+        self.pos_d = torch.as_tensor(w.n0.astype(np.int64), device=dev)
+        bf = torch.bfloat16 if w.dtype == "bf16" else torch.float32
+        S, L, b = total_steps, w.L, w.batch
+        # both input variants of every step: A = loop continues, B = loop-free
+        self.qA = torch.empty((S, L, b, w.H_q, w.d), dtype=bf, device=dev)
+        self.qB = torch.empty_like(self.qA)
+        self.kA = torch.empty((S, L, b, w.H_kv, w.d), dtype=bf, device=dev)
+        self.kB, self.vA, self.vB = (torch.empty_like(self.kA) for _ in range(3))
+        pos = torch.empty(b, dtype=torch.int64, device=dev)
+        for t in range(S):
+            pos.copy_(self.n0_d.to(torch.int64) + t)
+            synth.dev_step(w, self.seqs_d, pos, self.qA[t], self.kA[t], self.vA[t], self.s, mode=2)
+            synth.dev_step(w, self.seqs_d, pos, self.qB[t], self.kB[t], self.vB[t], self.s, mode=1)
+        self.q = torch.empty((L, b, w.H_q, w.d), dtype=bf, device=dev)
+        self.kn = torch.empty((L, b, w.H_kv, w.d), dtype=bf, device=dev)
+        self.vn = torch.empty_like(self.kn)
+        self.esz = 2 if w.dtype == "bf16" else 4
+        torch.cuda.synchronize()
+
+    def reset(self):
+        """fresh cache of the workload, guard state and sequence modes (untimed)"""
+        torch, w, lg = self.torch, self.w, self.lg
+        self.cache.len.copy_(self.n0_d)
+        synth.dev_fill_cache(w, self.cache.k, self.cache.v, self.seqs_d.copy_(
+            synth.seqs_tensor(w.seqs, self.dev)), self.off_d, self.n0_d, int(w.n0.max()), self.s)
+        lg.lg_sketch_build(self.cache, self.p, int(w.n0.max()))
+        lg.lg_state_init(self.cache, self.guard.state, 64)
+        self.pos_d.copy_(self.n0_d.to(torch.int64))
+        self.cache.status.zero_()
+        torch.cuda.synchronize()
+
+    def select_inputs(self, t):
+        w = self.w
+        e = self.esz
+        synth.dev_select(w, self.seqs_d, self.pos_d, w.H_q * w.d * e, self.qA[t], self.qB[t],
+                         self.q, self.s)
+        synth.dev_select(w, self.seqs_d, self.pos_d, w.H_kv * w.d * e, self.kA[t], self.kB[t],
+                         self.kn, self.s)
+        synth.dev_select(w, self.seqs_d, self.pos_d, w.H_kv * w.d * e, self.vA[t], self.vB[t],
+                         self.vn, self.s)
+
+    def step(self, t, ev=None):
+        """one guarded decode step; ev = (a0, a1, p0, p1) events around attend and prune"""
+        lg, c, g, p, w = self.lg, self.cache, self.guard, self.p, self.w
+        self.select_inputs(t)
+        lg.lg_begin_step(c, self.s)
+        lg.lg_append(c, 0, w.L, self.kn, self.vn, None, p, self.s)
+        if ev:
+            ev[0].record(self.stream)
+        for l0 in range(0, w.L, self.nl):
+            lg.lg_decode_attend(c, l0, self.nl, self.q[l0:l0 + self.nl], w.H_q, g.scale,
+                                g.out[l0:l0 + self.nl], g.stats[l0:l0 + self.nl], p.suffix_w, 0,
+                                g.max_len, g.ws, self.s)
+        if ev:
+            ev[1].record(self.stream)
+        lg.lg_detect(c, g.stats, w.H_q, g.state, self.budget_d, p, g.flags, g.spans, None,
+                     self.s)
+        if ev:
+            ev[2].record(self.stream)
+        lg.lg_prune_compact(c, g.flags, g.spans, g.state, self.budget_d, p, g.kept_idx,
+                            g.kept_count, g.max_keep, g.max_len, self.s)
+        if ev:
+            ev[3].record(self.stream)
+        synth.dev_advance(w, self.seqs_d, g.flags, self.pos_d, self.s)
+
+    # launches of this repository's kernels per step (harness + path)
+    def launches_per_step(self):
+        n_attend = math.ceil(self.w.L / self.nl) * 2       # partial + combine per call
+        path = 1 + 2 + n_attend + 1 + 2                     # begin, append(+sketch), attend,
+        harness = 3 + 1                                     # detect, keep+compact; select x3,
+        return path, harness                                # advance
+
+    def replay_log(self, K):
+        """replay the timed trajectory untimed, recording per-step lengths and kept lists
+        (the decisions are deterministic, so they are the timed run's)"""
+        torch = self.torch
+        self.reset()
+        lens, kept = [], []
+        for t in range(K):
+            lens.append(self.cache.len.clone())
+            self.step(t)
+            kc = self.guard.kept_count.clone()
+            kept.append((kc, self.guard.kept_idx.clone() if int((kc >= 0).sum()) else None))
+        torch.cuda.synchronize()
+        return lens, kept
+
+
+def attend_bytes(w, n_rows):
+    """algorithmic bytes of attend+stats for one step: K and V rows once per kv-head and
+    layer, queries, outputs and statistics"""
+    esz = 2 if w.dtype == "bf16" else 4
+    kv = 2 * w.L * w.H_kv * w.d * esz * int(np.sum(n_rows))
+    qo = 2 * w.L * w.batch * w.H_q * w.d * esz + w.L * w.batch * w.H_q * 16
+    return kv + qo
+
+
+def compact_bytes(w, kept_count, kept_idx):
+    """algorithmic bytes of one prune: every moved row of K and V (all layers and kv-heads) and
+    of the sketches read once and written once"""
+    esz = 2 if w.dtype == "bf16" else 4
+    total = 0
+    for b in range(w.batch):
+        c = int(kept_count[b])
+        if c < 0:
+            continue
+        k = kept_idx[b, :c]
+        moved = int(np.sum(k != np.arange(c)))
+        total += 2 * moved * (2 * w.L * w.H_kv * w.d * esz + w.H_kv * w.d // 8)
+    return total
+
+
+def traffic_from_profile(kernel_src_hash):
+    """DRAM bytes per attend launch from the committed ncu summary, if it was taken on the
+    current kernel source; else None"""
+    path = os.path.join(ROOT, "profiles", "attend_traffic.json")
+    if not os.path.exists(path):
+        return None
+    with open(path) as f:
+        d = json.load(f)
+    if d.get("source_sha256") != kernel_src_hash:
+        return None
+    return d
+
+
+def source_hash():
+    import hashlib
+    h = hashlib.sha256()
+    for f in ("lg_attend.cu", "lg_common.cuh"):
+        with open(os.path.join(ROOT, "paper_2604_10044_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()
+
+
+def run_gpu(args, ws, rank, local):
+    import torch
+    assert torch.cuda.is_available(), "the gb300 arm needs a CUDA device"
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    over = {} if rank == 0 else {"seed": 1000 + rank}
+    if args.batch:
+        over["batch"] = args.batch
+    w = synth.make_workload(args.workload, **over)
+    K, W = args.steps, args.warmup
+    if args.profile_steps:
+        # untimed steps inside an NVTX range "steps" (ncu --nvtx-include "steps/")
+        bench = GpuBench(w, dev, args.profile_steps, args.layers_per_call)
+        bench.reset()
+        torch.cuda.nvtx.range_push("steps")
+        for t in range(args.profile_steps):
+            bench.step(t)
+        torch.cuda.synchronize()
+        torch.cuda.nvtx.range_pop()
+        return None
+    bench = GpuBench(w, dev, max(K, W, 1), args.layers_per_call)
+
+    # warm-up on the trajectory's first W steps, then a fresh cache for the timed run
+    bench.reset()
+    for t in range(W):
+        bench.step(t)
+    torch.cuda.synchronize()
+    bench.reset()
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(K)]
+    start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    clocks = Clocks(local, enabled=not args.no_clocks)
+    barrier(ws)
+    torch.cuda.synchronize()
+    start.record(bench.stream)
+    for t in range(K):
+        bench.step(t, evs[t])
+    stop.record(bench.stream)
+    torch.cuda.synchronize()
+    barrier(ws)
+    clk = clocks.stop()
+    status = bench.lg.lg_read_device_status(bench.cache)
+    if status != 0:
+        raise RuntimeError("device status %d after the timed run" % status)
+    ms_local = start.elapsed_time(stop)
+    ms = max_over_ranks(ms_local, ws)
+    attend_ms = [e[0].elapsed_time(e[1]) for e in evs]
+    prune_ms = [e[2].elapsed_time(e[3]) for e in evs]
+
+    # algorithmic bytes of the same trajectory (untimed, deterministic replay)
+    lens, kept = bench.replay_log(K)
+    a_bytes, c_bytes, c_ms = [], [], []
+    triggers = 0
+    for t in range(K):
+        n_rows = lens[t].cpu().numpy() + 1
+        a_bytes.append(attend_bytes(w, n_rows))
+        kc, ki = kept[t]
+        kc = kc.cpu().numpy()
+        if ki is not None:
+            c_bytes.append(compact_bytes(w, kc, ki.cpu().numpy()))
+            c_ms.append(prune_ms[t])
+    hbm_peak, peak_kind = peaks()
+    attend_gbs = sum(a_bytes) / (sum(attend_ms) * 1e-3) / 1e9
+    compact_gbs = (sum(c_bytes) / (sum(c_ms) * 1e-3) / 1e9) if c_ms else None
+
+    e2e = None
+    if not args.no_e2e:
+        e2e = run_e2e(bench, K, ws)
+
+    value = sum_over_ranks(K, ws) / (ms * 1e-3)
+    path_l, harness_l = bench.launches_per_step()
+    prof = traffic_from_profile(source_hash())
+    traffic = None
+    if prof:
+        # per-launch DRAM bytes scaled from the captured launch to this run's mean launch
+        traffic = prof["dram_bytes_per_row"] * (sum(a_bytes) / K) / attend_bytes(w, [1]) \
+            if "dram_bytes_per_row" in prof else None
+    line = {
+        "metric": METRIC, "value": round(value, 3), "unit": UNIT, "n_gpus": ws, "steps": K,
+        "warmup": W, "ms_per_step": round(ms / K, 4), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": w.dtype, "data": "synthetic",
+        "config": dict(w.describe(), l2="inputs larger than L2 (K/V cache 4.3-8.6 GB per GPU)",
+                       layers_per_attend_call=bench.nl, parallelism="dp%d (independent batches, "
+                       "no collective)" % ws, tokens_per_step=w.batch * ws),
+        "roofline": {"bound": "hbm", "achieved": round(attend_gbs, 1), "peak": hbm_peak,
+                     "unit": "GB/s", "frac": round(attend_gbs / hbm_peak, 4),
+                     "traffic": traffic,
+                     "kernel": "lg_decode_attend (split-K partial + combine), all %d layers per "
+                               "call" % w.L if bench.nl == w.L else "lg_decode_attend",
+                     "peak_kind": peak_kind + " copy bandwidth"},
+        "kernels": {
+            "attend_stats": {"GB_per_s": round(attend_gbs, 1),
+                             "frac_of_%s_peak" % peak_kind: round(attend_gbs / hbm_peak, 4),
+                             "frac_of_8TBs_nominal": round(attend_gbs / 8000.0, 4),
+                             "ms_per_step": round(sum(attend_ms) / K, 4)},
+            "prune_compact": {"GB_per_s": round(compact_gbs, 1) if compact_gbs else None,
+                              "frac_of_%s_peak" % peak_kind:
+                                  round(compact_gbs / hbm_peak, 4) if compact_gbs else None,
+                              "events": len(c_ms),
+                              "ms_per_event": round(sum(c_ms) / len(c_ms), 4) if c_ms else None,
+                              "moved_bytes_per_event": int(sum(c_bytes) / len(c_bytes))
+                              if c_bytes else 0},
+            "other_ms_per_step": round((ms_local - sum(attend_ms) - sum(prune_ms)) / K, 4)},
+        "gpu_launches": (path_l + harness_l) * K,
+        "gpu_launches_detail": {"path_per_step": path_l, "harness_per_step": harness_l},
+        "clocks": clk,
+    }
+    if e2e:
+        line["e2e"] = e2e
+    return line, w
+
+
+def run_e2e(bench, K, ws):
+    """the same steps through the C ABI with host buffers: every step copies its inputs from
+    pinned host memory and reads the outputs back (attention output, flags, spans, lengths)"""
+    torch = bench.torch
+    w = bench.w
+    # both input variants of every step in pinned host memory (filled before timing)
+    hq = [bench.qA[:K].cpu().pin_memory(), bench.qB[:K].cpu().pin_memory()]
+    hk = [bench.kA[:K].cpu().pin_memory(), bench.kB[:K].cpu().pin_memory()]
+    hv = [bench.vA[:K].cpu().pin_memory(), bench.vB[:K].cpu().pin_memory()]
+    g = bench.guard
+    out_h = torch.empty(g.out.shape, dtype=g.out.dtype).pin_memory()
+    small_h = torch.empty(4 * w.batch, dtype=torch.int32).pin_memory()
+    small_d = torch.empty(4 * w.batch, dtype=torch.int32, device=bench.dev)
+    bench.reset()
+    barrier(ws)
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    for t in range(K):
+        # H2D: this step's input variants into the device staging slots the harness reads
+        for dst, src in ((bench.qA, hq[0]), (bench.qB, hq[1]), (bench.kA, hk[0]),
+                         (bench.kB, hk[1]), (bench.vA, hv[0]), (bench.vB, hv[1])):
+            dst[t].copy_(src[t], non_blocking=True)
+        bench.step(t)
+        out_h.copy_(g.out, non_blocking=True)
+        small_d[:w.batch].copy_(g.flags)
+        small_d[w.batch:3 * w.batch].copy_(g.spans.view(-1))
+        small_d[3 * w.batch:].copy_(bench.cache.len)
+        small_h.copy_(small_d, non_blocking=True)
+        bench.stream.synchronize()
+    dt = max_over_ranks(time.perf_counter() - t0, ws)
+    h2d = 2 * (hq[0][0].numel() + hk[0][0].numel() + hv[0][0].numel()) * hq[0].element_size()
+    d2h = out_h.numel() * out_h.element_size() + small_h.numel() * 4
+    return {"value": round(sum_over_ranks(K, ws) / dt, 3), "unit": UNIT,
+            "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
+            "note": "inputs of both sequence modes (loop continues / loop-free) copied every "
+                    "step; outputs, flags, spans and lengths read back every step"}
+
+
+# ------------------------------------------------------------------ CPU oracle arm
+
+def oracle_sample_workload(w, n_seq):
+    """the first n_seq sequences of workload w (same rows: the generator keys on the index)"""
+    sub = synth.Workload(name=w.name, L=w.L, H_q=w.H_q, H_kv=w.H_kv, d=w.d, dtype=w.dtype,
+                         batch=n_seq, n0=w.n0[:n_seq], budget=w.budget[:n_seq], steps=w.steps,
+                         seed=w.seed, seqs=w.seqs[:n_seq].copy(), head_scale=w.head_scale,
+                         n_sink=w.n_sink, sink_factor=w.sink_factor, sigma=w.sigma,
+                         query_mode=w.query_mode, zstar=w.zstar, q_noise=w.q_noise)
+    return sub
+
+
+def time_oracle(w, n_seq, n_layers, steps, warm=0):
+    """the oracle (as it stands) running `steps` guarded decode steps of the first n_seq
+    sequences restricted to the first n_layers layers; returns (seconds per step, threads)"""
+    import oracle
+    sub = oracle_sample_workload(w, n_seq)
+    sub.L = n_layers
+    K, V = synth.host_cache(sub)
+
+    def run(n):
+        g = oracle.OracleGuard(sub, K.copy(), V.copy())
+        seqs = sub.seqs.copy()
+        pos = sub.n0.astype(np.int64)
+        times = []
+        for t in range(n):
+            q, kn, vn = synth.host_step(sub, pos, seqs)
+            t0 = time.perf_counter()
+            r = g.step(q, kn, vn, pos)
+            times.append(time.perf_counter() - t0)
+            synth.note_interventions(seqs, pos, r["flags"])
+            pos = pos + 1
+        return times, g.threads
+
+    if warm:
+        run(warm)          # warm-up steps; the timed steps start again from the fresh cache
+    return run(steps)
+
+
+def cpu_baseline(w, target_s=15.0):
+    """oracle time for one guarded step of a bounded sample: all layers of the first
+    sequences, scaled to batch steps/s"""
+    n_seq = 1
+    times, threads = time_oracle(w, n_seq, w.L, 1)
+    while sum(times) < target_s / 4 and n_seq < w.batch:
+        n_seq *= 2
+        times, threads = time_oracle(w, min(n_seq, w.batch), w.L, 1)
+    n_seq = min(n_seq, w.batch)
+    frac = n_seq / w.batch
+    sec = sum(times)
+    return {"value": round(frac / sec, 6), "unit": UNIT, "cores": threads, "kind": "oracle",
+            "sample": "1 guarded decode step (step 1: attention over 8193 rows, detect, budget "
+                      "prune) of %d of the %d sequences, all %d layers; value = %d/%d batch "
+                      "steps / %.2f s" % (n_seq, w.batch, w.L, n_seq, w.batch, sec)}
+
+
+def run_reference(args, ws, rank):
+    """--impl reference: the CPU oracle on the host cores, K timed steps after W warm-up steps,
+    each step a bounded sample of the workload (the first sequence, the first layers)"""
+    if rank != 0:
+        return
+    w = synth.make_workload(args.workload)
+    K, W = args.steps, args.warmup
+    # size the sample so that the whole run stays within about two minutes
+    per_step_budget = 120.0 / max(1, K + W)
+    t1, _ = time_oracle(w, 1, 1, 1)
+    n_layers = int(max(1, min(w.L, per_step_budget / max(t1[0], 1e-6))))
+    times, threads = time_oracle(w, 1, n_layers, K, warm=W)
+    sec = sum(times)
+    frac = (1.0 / w.batch) * (n_layers / w.L)
+    value = K * frac / sec
+    line = {"impl": "reference", "metric": METRIC, "value": round(value, 6), "unit": UNIT,
+            "n_gpus": ws, "steps": K, "warmup": W, "ms_per_step": round(1e3 / value, 3),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "config": w.describe(),
+            "cpu_baseline": {"value": round(value, 6), "unit": UNIT, "cores": threads,
+                             "kind": "oracle",
+                             "sample": "each step: the oracle's guarded decode step of sequence "
+                                       "0 of %d, layers 0..%d of %d; value scaled by %.5f "
+                                       "batch steps per sample step" % (
+                                           w.batch, n_layers - 1, w.L, frac)},
+            "e2e": {"value": round(value, 6), "unit": UNIT, "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    args = parse()
+    ws, rank, local = dist_setup()
+    if ws != args.gpus:
+        raise SystemExit("--gpus %d but WORLD_SIZE=%d" % (args.gpus, ws))
+    if args.impl == "reference":
+        run_reference(args, ws, rank)
+        return
+    res = run_gpu(args, ws, rank, local)
+    if res is None:
+        return
+    line, w = res
+    if rank == 0:
+        if ws == 1 and not args.no_cpu_baseline:
+            line["cpu_baseline"] = cpu_baseline(w)
+        print(json.dumps(line), flush=True)
+
+
+if __name__ == "__main__":
+    main()

@@ -35,16 +35,19 @@ lg_status check_params(const lg_guard_params *p) {
 
 lg_status cuda_status(cudaError_t e) { return e == cudaSuccess ? LG_OK : LG_ERR_CUDA; }
 
-// rows per attend CTA: a multiple of the staging tile sized so that a launch has about four
-// waves of 152 SMs x 3 CTAs, between 2 tiles and 2048 rows
+// rows per chunk (one work item: one CTA of the fp32 path, one loop trip of a persistent CTA
+// of the bf16 path): a multiple of the staging tile, about eight chunks per SM of a 152-SM
+// GB300 for the bf16 path and twelve CTAs per SM for the fp32 path, at most 4096 rows
 int attend_chunk_rows(const lg_cache *c, int n_layers, int max_len) {
   const int tile = lg::attend_tile_rows(c->dtype, c->d);
   const int64_t rows = (int64_t)max_len * c->batch * c->H_kv * n_layers;
-  const int64_t target_ctas = 152 * 3 * 4;
-  int64_t ch = (rows + target_ctas - 1) / target_ctas;
+  const int64_t target = c->dtype == LG_BF16 ? 152 * 8 : 152 * 3 * 4;
+  int64_t ch = (rows + target - 1) / target;
   ch = (ch + tile - 1) / tile * tile;
-  if (ch < 2 * tile) ch = 2 * tile;
-  if (ch > 2048) ch = 2048 / tile * tile;
+  const int64_t lo = c->dtype == LG_BF16 ? tile : 2 * tile;
+  const int64_t hi = c->dtype == LG_BF16 ? 4096 : 2048 / tile * tile;
+  if (ch < lo) ch = lo;
+  if (ch > hi) ch = hi;
   return (int)ch;
 }
 
@@ -193,7 +196,9 @@ lg_status lg_decode_attend(const lg_cache *c, int layer0, int n_layers, const vo
   a.max_len = max_len;
   a.suffix_w = suffix_w;
   a.qscale = scale * 1.4426950408889634f;
-  return cuda_status(lg::launch_attend(a, c->dtype, c->d, g, out, stats, final_ml,
+  const int64_t rows_total = (int64_t)c->L * c->H_kv * c->S_total;
+  if (c->dtype == LG_BF16 && rows_total >= ((int64_t)1 << 31)) return LG_ERR_UNSUPPORTED;
+  return cuda_status(lg::launch_attend(a, c->dtype, c->d, g, rows_total, out, stats, final_ml,
                                        accumulate_h2o ? c->h2o : nullptr, s));
 }
 
@@ -205,8 +210,7 @@ lg_status lg_detect(const lg_cache *c, const float *stats, int H_q, lg_guard_sta
   if ((st = check_params(p)) != LG_OK) return st;
   if (!c->sketch || !stats || !state || !budget || !flags || !spans) return LG_ERR_INVALID_ARG;
   if (H_q < 1 || H_q % c->H_kv) return LG_ERR_INVALID_ARG;
-  const size_t smem = (size_t)lg::detect_smem_rows(*p) * (c->H_kv * c->d / 32) * 4;
-  if (smem > 200 * 1024) return LG_ERR_UNSUPPORTED;
+  if (lg::detect_smem_bytes(*p, c->H_kv * c->d / 32) > 200 * 1024) return LG_ERR_UNSUPPORTED;
   return cuda_status(
       lg::launch_detect(*c, stats, H_q, state, budget, *p, flags, spans, diag, s));
 }

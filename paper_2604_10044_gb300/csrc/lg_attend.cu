@@ -361,15 +361,22 @@ __global__ void h2o_accumulate_kernel(AttendArgs a, float *h2o, const float *fin
 // ------------------------------------------------------------------ launch
 
 template <typename T, int D, int G>
-static cudaError_t launch_typed(const AttendArgs &a, void *out, float *stats, float *final_ml,
-                                float *h2o, cudaStream_t s) {
+static cudaError_t launch_typed(const AttendArgs &a, int64_t rows_total, void *out, float *stats,
+                                float *final_ml, float *h2o, cudaStream_t s) {
   using C = AttendCfg<T, D, G>;
-  auto kp = attend_partial_kernel<T, D, G>;
-  cudaError_t e = cudaFuncSetAttribute(kp, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmem);
-  if (e != cudaSuccess) return e;
-  dim3 grid(a.max_chunks, a.H_kv, a.n_layers * a.batch);
-  kp<<<grid, C::kThreads, C::kSmem, s>>>(a);
-  if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  cudaError_t e;
+  if (Elem<T>::kDtype == LG_BF16) {
+    // tensor-core partial pass (lg_attend_mma.cu)
+    e = launch_attend_mma_partial(a, D, G, rows_total, s);
+    if (e != cudaSuccess) return e;
+  } else {
+    auto kp = attend_partial_kernel<T, D, G>;
+    e = cudaFuncSetAttribute(kp, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmem);
+    if (e != cudaSuccess) return e;
+    dim3 grid(a.max_chunks, a.H_kv, a.n_layers * a.batch);
+    kp<<<grid, C::kThreads, C::kSmem, s>>>(a);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  }
   attend_combine_kernel<T, D><<<dim3(a.H_q, a.batch, a.n_layers), D, 0, s>>>(a, out, stats,
                                                                             final_ml);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
@@ -384,32 +391,37 @@ static cudaError_t launch_typed(const AttendArgs &a, void *out, float *stats, fl
 }
 
 template <typename T, int D>
-static cudaError_t launch_d(const AttendArgs &a, int g, void *out, float *stats, float *fm,
-                            float *h2o, cudaStream_t s) {
+static cudaError_t launch_d(const AttendArgs &a, int64_t rt, int g, void *out, float *stats,
+                            float *fm, float *h2o, cudaStream_t s) {
   switch (g) {
-    case 1: return launch_typed<T, D, 1>(a, out, stats, fm, h2o, s);
-    case 2: return launch_typed<T, D, 2>(a, out, stats, fm, h2o, s);
-    case 3: return launch_typed<T, D, 3>(a, out, stats, fm, h2o, s);
-    case 4: return launch_typed<T, D, 4>(a, out, stats, fm, h2o, s);
-    case 5: return launch_typed<T, D, 5>(a, out, stats, fm, h2o, s);
-    case 6: return launch_typed<T, D, 6>(a, out, stats, fm, h2o, s);
-    case 7: return launch_typed<T, D, 7>(a, out, stats, fm, h2o, s);
-    case 8: return launch_typed<T, D, 8>(a, out, stats, fm, h2o, s);
+    case 1: return launch_typed<T, D, 1>(a, rt, out, stats, fm, h2o, s);
+    case 2: return launch_typed<T, D, 2>(a, rt, out, stats, fm, h2o, s);
+    case 3: return launch_typed<T, D, 3>(a, rt, out, stats, fm, h2o, s);
+    case 4: return launch_typed<T, D, 4>(a, rt, out, stats, fm, h2o, s);
+    case 5: return launch_typed<T, D, 5>(a, rt, out, stats, fm, h2o, s);
+    case 6: return launch_typed<T, D, 6>(a, rt, out, stats, fm, h2o, s);
+    case 7: return launch_typed<T, D, 7>(a, rt, out, stats, fm, h2o, s);
+    case 8: return launch_typed<T, D, 8>(a, rt, out, stats, fm, h2o, s);
   }
   return cudaErrorInvalidValue;
 }
 
+// rows per staging tile: the tensor-core path streams 128-row tiles; the fp32 path 8 KB tiles
 int attend_tile_rows(int dtype, int d) {
-  const int rb = d * (dtype == LG_BF16 ? 2 : 4);
-  return 8192 / rb;
+  if (dtype == LG_BF16) return mma_tile_rows();
+  return 8192 / (d * 4);
 }
 
-cudaError_t launch_attend(const AttendArgs &a, int dtype, int d, int g, void *out, float *stats,
-                          float *final_ml, float *h2o, cudaStream_t s) {
-  if (dtype == LG_BF16 && d == 128) return launch_d<__nv_bfloat16, 128>(a, g, out, stats, final_ml, h2o, s);
-  if (dtype == LG_BF16 && d == 64) return launch_d<__nv_bfloat16, 64>(a, g, out, stats, final_ml, h2o, s);
-  if (dtype == LG_F32 && d == 128) return launch_d<float, 128>(a, g, out, stats, final_ml, h2o, s);
-  if (dtype == LG_F32 && d == 64) return launch_d<float, 64>(a, g, out, stats, final_ml, h2o, s);
+cudaError_t launch_attend(const AttendArgs &a, int dtype, int d, int g, int64_t rows_total,
+                          void *out, float *stats, float *final_ml, float *h2o, cudaStream_t s) {
+  if (dtype == LG_BF16 && d == 128)
+    return launch_d<__nv_bfloat16, 128>(a, rows_total, g, out, stats, final_ml, h2o, s);
+  if (dtype == LG_BF16 && d == 64)
+    return launch_d<__nv_bfloat16, 64>(a, rows_total, g, out, stats, final_ml, h2o, s);
+  if (dtype == LG_F32 && d == 128)
+    return launch_d<float, 128>(a, rows_total, g, out, stats, final_ml, h2o, s);
+  if (dtype == LG_F32 && d == 64)
+    return launch_d<float, 64>(a, rows_total, g, out, stats, final_ml, h2o, s);
   return cudaErrorInvalidValue;
 }
 

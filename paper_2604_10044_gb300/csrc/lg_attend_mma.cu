@@ -1,0 +1,480 @@
+// Decode attention over a bf16 KV cache fused with the guard's per-head statistics (LoopGuard
+// Sec. 3.1, Eq. 1; statistics read by Sec. 5.2), on tensor cores.
+//
+// Persistent CTAs (one per SM) walk a list of chunks, each CHUNK consecutive rows of one
+// (layer, sequence, kv-head).  A producer warp streams 128-row K and V tiles into a 3-stage
+// shared-memory ring with 2-D tensor copies (cp.async.bulk.tensor, 128-byte swizzle, one box
+// per 64 columns) completing on mbarriers.  Each of four consumer warps owns 32 rows of a tile
+// and all g query heads of the kv-head (padded to 8):
+//   S^T[16 rows x 8 heads] = K[16 x d] q^T      mma.sync m16n8k16 bf16 -> fp32, A by ldmatrix
+//   online softmax in log2 units on the accumulator fragments (exact running max per head)
+//   o^T[d x 8 heads] += V^T[d x 16 rows] P^T    A by ldmatrix.trans, B = P^T by movmatrix,
+//                                               P split into bf16 hi + lo (two MMAs)
+// The suffix mass, the entropy term and the normaliser accumulate beside the softmax.  At the
+// end of a chunk the four warps merge through shared memory into one partial per head
+// {M, l, u, sigma, o[d]}; lg_attend.cu merges the chunk partials and emits out and the
+// statistics.  Rows past the end of a sequence (ragged last tile) are masked to zero weight,
+// and their stale V rows are zeroed in shared memory before the P.V product.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <math.h>
+#include <stdint.h>
+
+#include "lg_common.cuh"
+#include "lg_internal.h"
+
+namespace lg {
+
+namespace {
+
+constexpr int kTile = 128;          // rows per tile (TMA box height)
+constexpr int kBoxBytes = kTile * 128;  // one box: 128 rows x 64 bf16
+constexpr int kConsumerWarps = 4;
+constexpr int kThreads = (kConsumerWarps + 1) * 32;
+
+template <int D>
+struct MmaCfg {
+  static constexpr int kHalves = D / 64;                      // boxes per row
+  static constexpr int kStageBytes = 2 * kHalves * kBoxBytes;  // K and V
+  static constexpr int kStages = D == 128 ? 3 : 6;
+  static constexpr int kRingBytes = kStages * kStageBytes;
+  static constexpr int kMergeBytes = kConsumerWarps * 8 * D * 4 + kConsumerWarps * 8 * 4 * 4;
+  static constexpr int kSmem = kRingBytes + kMergeBytes + 1024;  // + alignment slack
+  static constexpr int kKSteps = D / 16;
+};
+
+__device__ __forceinline__ void tma_load_2d(void *smem_dst, const CUtensorMap *map, int x, int y,
+                                            uint64_t *bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes "
+      "[%0], [%1, {%2, %3}], [%4];" ::"r"(smem_addr(smem_dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(smem_addr(bar))
+      : "memory");
+}
+
+__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t &r0, uint32_t &r1, uint32_t &r2,
+                                        uint32_t &r3) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
+               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+               : "r"(addr));
+}
+
+__device__ __forceinline__ void ldsm_x4_trans(uint32_t addr, uint32_t &r0, uint32_t &r1,
+                                              uint32_t &r2, uint32_t &r3) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
+               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+               : "r"(addr));
+}
+
+__device__ __forceinline__ void mma_bf16(float *d, uint32_t a0, uint32_t a1, uint32_t a2,
+                                         uint32_t a3, uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, "
+      "{%4, %5, %6, %7}, {%8, %9}, {%0, %1, %2, %3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+
+__device__ __forceinline__ uint32_t movmatrix_trans(uint32_t a) {
+  uint32_t d;
+  asm volatile("movmatrix.sync.aligned.m8n8.trans.b16 %0, %1;" : "=r"(d) : "r"(a));
+  return d;
+}
+
+__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
+  __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<uint32_t *>(&v);
+}
+
+// byte offset of 16-byte chunk c8 (0..7) of row r in a 128-byte-swizzled box
+__device__ __forceinline__ uint32_t swz(int r, int c8) {
+  return (uint32_t)(r * 128 + ((c8 ^ (r & 7)) << 4));
+}
+
+struct ChunkId {
+  int lloc, b, kvh, ch;
+};
+
+__device__ __forceinline__ ChunkId decode_chunk(const AttendArgs &a, int c) {
+  ChunkId id;
+  id.ch = c % a.max_chunks;
+  int r = c / a.max_chunks;
+  id.kvh = r % a.H_kv;
+  r /= a.H_kv;
+  id.b = r % a.batch;
+  id.lloc = r / a.batch;
+  return id;
+}
+
+}  // namespace
+
+template <int D, int G>
+__global__ void __launch_bounds__(kThreads, 1)
+attend_mma_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
+                  AttendArgs a, int total_chunks) {
+  using C = MmaCfg<D>;
+  extern __shared__ unsigned char smem_raw[];
+  __shared__ __align__(8) uint64_t full_bar[C::kStages];
+  __shared__ __align__(8) uint64_t empty_bar[C::kStages];
+  unsigned char *smem = reinterpret_cast<unsigned char *>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  float *merge_o = reinterpret_cast<float *>(smem + C::kRingBytes);  // [warps][8][D]
+  float *merge_s = merge_o + kConsumerWarps * 8 * D;                  // [warps][8][4]
+
+  if (status_bad(a.status)) return;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < C::kStages; ++s) {
+      mbar_init(&full_bar[s], 1);
+      mbar_init(&empty_bar[s], kConsumerWarps);
+    }
+    mbar_fence_init();
+  }
+  __syncthreads();
+
+  if (warp == kConsumerWarps) {
+    // ------------------------------------------------------------ producer
+    if (lane == 0) {
+      asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmK)) : "memory");
+      asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmV)) : "memory");
+      uint32_t it = 0;
+      for (int c = blockIdx.x; c < total_chunks; c += gridDim.x) {
+        const ChunkId id = decode_chunk(a, c);
+        const int n = a.len[id.b];
+        const int row0 = id.ch * a.chunk_rows;
+        if (n > a.max_len || row0 >= n) continue;
+        const int rows = min(a.chunk_rows, n - row0);
+        const int ntiles = (rows + kTile - 1) / kTile;
+        const int grow =
+            (int)(((int64_t)(a.layer0 + id.lloc) * a.H_kv + id.kvh) * a.S_total + a.seq_off[id.b] +
+                  row0);
+        for (int t = 0; t < ntiles; ++t, ++it) {
+          const int st = it % C::kStages;
+          if (it >= (uint32_t)C::kStages &&
+              !mbar_wait(&empty_bar[st], ((it / C::kStages) - 1) & 1)) {
+            set_status(a.status, LG_ERR_TIMEOUT);
+            return;
+          }
+          unsigned char *stage = smem + (size_t)st * C::kStageBytes;
+          mbar_arrive_expect_tx(&full_bar[st], C::kStageBytes);
+#pragma unroll
+          for (int h = 0; h < C::kHalves; ++h) {
+            tma_load_2d(stage + h * kBoxBytes, &tmK, h * 64, grow + t * kTile, &full_bar[st]);
+            tma_load_2d(stage + (C::kHalves + h) * kBoxBytes, &tmV, h * 64, grow + t * kTile,
+                        &full_bar[st]);
+          }
+        }
+      }
+    }
+    return;
+  }
+
+  // -------------------------------------------------------------- consumers
+  const int g = lane >> 2, t4 = lane & 3;
+  const int mrow = lane & 7, msel = lane >> 3;  // ldmatrix: row within 8x8, matrix index
+  uint32_t it = 0;
+  bool ok = true;
+  for (int c = blockIdx.x; c < total_chunks && ok; c += gridDim.x) {
+    const ChunkId id = decode_chunk(a, c);
+    const int n = a.len[id.b];
+    const int row0 = id.ch * a.chunk_rows;
+    if (n > a.max_len) {
+      if (lane == 0 && warp == 0) set_status(a.status, LG_ERR_CAPACITY);
+      continue;
+    }
+    if (row0 >= n) continue;
+    const int rows = min(a.chunk_rows, n - row0);
+    const int ntiles = (rows + kTile - 1) / kTile;
+    const int suffix_lo = n - min(a.suffix_w, n);
+
+    // B fragments of q^T: head g (zero for padded heads), d = 16 ks + 2 t4 (+1, +8, +9)
+    uint32_t qf[C::kKSteps][2];
+    {
+      const int64_t qh = ((int64_t)id.lloc * a.batch + id.b) * a.H_q + (int64_t)id.kvh * G + g;
+      const uint32_t *qp = reinterpret_cast<const uint32_t *>(
+          reinterpret_cast<const __nv_bfloat16 *>(a.q) + qh * D);
+#pragma unroll
+      for (int ks = 0; ks < C::kKSteps; ++ks) {
+        qf[ks][0] = g < G ? qp[ks * 8 + t4] : 0u;
+        qf[ks][1] = g < G ? qp[ks * 8 + 4 + t4] : 0u;
+      }
+    }
+    float o[C::kKSteps][4];
+#pragma unroll
+    for (int eb = 0; eb < C::kKSteps; ++eb) o[eb][0] = o[eb][1] = o[eb][2] = o[eb][3] = 0.f;
+    float m2[2] = {-INFINITY, -INFINITY}, l2[2] = {0.f, 0.f}, u2[2] = {0.f, 0.f},
+          sg2[2] = {0.f, 0.f};
+    float *logits = a.logits;
+    const int64_t lrow0 =
+        ((int64_t)id.lloc * a.H_kv + id.kvh) * a.S_total + a.seq_off[id.b] + row0;
+
+    for (int t = 0; t < ntiles; ++t, ++it) {
+      const int st = it % C::kStages;
+      if (!mbar_wait(&full_bar[st], (it / C::kStages) & 1)) {
+        set_status(a.status, LG_ERR_TIMEOUT);
+        ok = false;
+        break;
+      }
+      unsigned char *stage = smem + (size_t)st * C::kStageBytes;
+      const uint32_t kbase = smem_addr(stage);
+      const uint32_t vbase = kbase + C::kHalves * kBoxBytes;
+      const int tile_rows = min(kTile, rows - t * kTile);
+      const int r_w = warp * 32;  // this warp's first row in the tile
+      if (tile_rows < r_w + 32) {
+        // ragged tail: zero the V rows past the end so that 0 * stale stays 0
+        for (int idx = lane; idx < 32 * C::kHalves * 8; idx += 32) {
+          const int rr = r_w + idx / (C::kHalves * 8);
+          const int hc = idx % (C::kHalves * 8);
+          if (rr >= tile_rows)
+            *reinterpret_cast<uint4 *>(stage + (C::kHalves + hc / 8) * kBoxBytes + rr * 128 +
+                                       (hc % 8) * 16) = make_uint4(0u, 0u, 0u, 0u);
+        }
+        __syncwarp();
+      }
+
+      // S^T for the warp's two 16-row blocks
+      float s[2][4];
+#pragma unroll
+      for (int mb = 0; mb < 2; ++mb) {
+        s[mb][0] = s[mb][1] = s[mb][2] = s[mb][3] = 0.f;
+        const int r = r_w + mb * 16 + (msel & 1) * 8 + mrow;
+#pragma unroll
+        for (int ks = 0; ks < C::kKSteps; ++ks) {
+          const int c8 = (ks & 3) * 2 + (msel >> 1);
+          uint32_t a0, a1, a2, a3;
+          ldsm_x4(kbase + (ks >> 2) * kBoxBytes + swz(r, c8), a0, a1, a2, a3);
+          mma_bf16(s[mb], a0, a1, a2, a3, qf[ks][0], qf[ks][1]);
+        }
+      }
+      // scale to log2 units, mask rows past the end; tile max per head (heads 2 t4, 2 t4 + 1)
+      float mx[2] = {-INFINITY, -INFINITY};
+#pragma unroll
+      for (int mb = 0; mb < 2; ++mb)
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          const int rl = r_w + mb * 16 + g + (j >> 1) * 8;  // row within the tile
+          const bool valid = rl < tile_rows;
+          s[mb][j] = valid ? s[mb][j] * a.qscale : -INFINITY;
+          mx[j & 1] = fmaxf(mx[j & 1], s[mb][j]);
+        }
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        mx[h] = fmaxf(mx[h], __shfl_xor_sync(0xffffffffu, mx[h], 4));
+        mx[h] = fmaxf(mx[h], __shfl_xor_sync(0xffffffffu, mx[h], 8));
+        mx[h] = fmaxf(mx[h], __shfl_xor_sync(0xffffffffu, mx[h], 16));
+      }
+      const bool raise = mx[0] > m2[0] || mx[1] > m2[1];
+      if (__any_sync(0xffffffffu, raise)) {
+        float corr[2];
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+          const float mn = fmaxf(m2[h], mx[h]);
+          corr[h] = mn == m2[h] ? 1.f : exp2f(m2[h] - mn);
+          u2[h] = l2[h] > 0.f ? corr[h] * (u2[h] + (m2[h] - mn) * l2[h]) : 0.f;
+          l2[h] *= corr[h];
+          sg2[h] *= corr[h];
+          m2[h] = mn;
+        }
+#pragma unroll
+        for (int eb = 0; eb < C::kKSteps; ++eb) {
+          o[eb][0] *= corr[0];
+          o[eb][1] *= corr[1];
+          o[eb][2] *= corr[0];
+          o[eb][3] *= corr[1];
+        }
+      }
+      // probabilities, sums, and P^T fragments
+      uint32_t pb[2][2], pl[2][2];
+#pragma unroll
+      for (int mb = 0; mb < 2; ++mb) {
+        float p[4];
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          const int h = j & 1;
+          const int rl = r_w + mb * 16 + g + (j >> 1) * 8;
+          const bool valid = rl < tile_rows;
+          p[j] = valid ? exp2f(s[mb][j] - m2[h]) : 0.f;
+          if (valid) {
+            l2[h] += p[j];
+            u2[h] += p[j] * (s[mb][j] - m2[h]);
+            if (row0 + t * kTile + rl >= suffix_lo) sg2[h] += p[j];
+          }
+        }
+        if (logits) {
+#pragma unroll
+          for (int half = 0; half < 2; ++half) {
+            const int rl = r_w + mb * 16 + g + half * 8;
+            if (rl < tile_rows) {
+              float *dst = logits + (lrow0 + t * kTile + rl) * G;
+              if (2 * t4 < G) dst[2 * t4] = s[mb][half * 2];
+              if (2 * t4 + 1 < G) dst[2 * t4 + 1] = s[mb][half * 2 + 1];
+            }
+          }
+        }
+        // P = hi + lo, both bf16: the P.V product keeps ~16 mantissa bits of P
+        const uint32_t h01 = pack_bf16(p[0], p[1]), h23 = pack_bf16(p[2], p[3]);
+        const float2 f01 = bf16x2_to_float2(h01), f23 = bf16x2_to_float2(h23);
+        pb[mb][0] = movmatrix_trans(h01);  // rows 0-7 of the block
+        pb[mb][1] = movmatrix_trans(h23);  // rows 8-15
+        pl[mb][0] = movmatrix_trans(pack_bf16(p[0] - f01.x, p[1] - f01.y));
+        pl[mb][1] = movmatrix_trans(pack_bf16(p[2] - f23.x, p[3] - f23.y));
+      }
+      // o^T += V^T P^T
+#pragma unroll
+      for (int mb = 0; mb < 2; ++mb) {
+        const int r = r_w + mb * 16 + (msel >> 1) * 8 + mrow;
+#pragma unroll
+        for (int eb = 0; eb < C::kKSteps; ++eb) {
+          const int c8 = (eb & 3) * 2 + (msel & 1);
+          uint32_t a0, a1, a2, a3;
+          ldsm_x4_trans(vbase + (eb >> 2) * kBoxBytes + swz(r, c8), a0, a1, a2, a3);
+          mma_bf16(o[eb], a0, a1, a2, a3, pb[mb][0], pb[mb][1]);
+          mma_bf16(o[eb], a0, a1, a2, a3, pl[mb][0], pl[mb][1]);
+        }
+      }
+      __syncwarp();
+      if (tile_rows < r_w + 32) asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+      if (lane == 0) mbar_arrive(&empty_bar[st]);
+    }
+    if (!ok) break;
+
+    // ---------------------------------------------------------- merge the four warps
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+#pragma unroll
+      for (int off = 4; off <= 16; off <<= 1) {
+        l2[h] += __shfl_xor_sync(0xffffffffu, l2[h], off);
+        u2[h] += __shfl_xor_sync(0xffffffffu, u2[h], off);
+        sg2[h] += __shfl_xor_sync(0xffffffffu, sg2[h], off);
+      }
+    }
+    float *mo = merge_o + (size_t)warp * 8 * D;
+#pragma unroll
+    for (int eb = 0; eb < C::kKSteps; ++eb) {
+      const int e = eb * 16 + g;
+      mo[(2 * t4) * D + e] = o[eb][0];
+      mo[(2 * t4 + 1) * D + e] = o[eb][1];
+      mo[(2 * t4) * D + e + 8] = o[eb][2];
+      mo[(2 * t4 + 1) * D + e + 8] = o[eb][3];
+    }
+    if (g == 0) {
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        float *ms = merge_s + ((size_t)warp * 8 + 2 * t4 + h) * 4;
+        ms[0] = m2[h];
+        ms[1] = l2[h];
+        ms[2] = u2[h];
+        ms[3] = sg2[h];
+      }
+    }
+    asm volatile("bar.sync 1, %0;" ::"n"(kConsumerWarps * 32) : "memory");
+    const int64_t pbase = ((int64_t)id.lloc * a.batch + id.b) * a.H_q + (int64_t)id.kvh * G;
+    for (int idx = threadIdx.x; idx < G * D; idx += kConsumerWarps * 32) {
+      const int h = idx / D, e = idx % D;
+      float M = -INFINITY;
+#pragma unroll
+      for (int w = 0; w < kConsumerWarps; ++w) M = fmaxf(M, merge_s[(w * 8 + h) * 4]);
+      float ov = 0.f, l = 0.f, u = 0.f, sg = 0.f;
+#pragma unroll
+      for (int w = 0; w < kConsumerWarps; ++w) {
+        const float *ms = merge_s + (w * 8 + h) * 4;
+        if (!(ms[1] > 0.f)) continue;  // warp saw no row of this chunk
+        const float f = exp2f(ms[0] - M);
+        ov += f * merge_o[((size_t)w * 8 + h) * D + e];
+        l += f * ms[1];
+        u += f * (ms[2] + (ms[0] - M) * ms[1]);
+        sg += f * ms[3];
+      }
+      float *pp = a.partial + ((pbase + h) * a.max_chunks + id.ch) * (D + 8);
+      pp[8 + e] = ov;
+      if (e == 0) {
+        pp[0] = M;
+        pp[1] = l;
+        pp[2] = u;
+        pp[3] = sg;
+      }
+    }
+    asm volatile("bar.sync 1, %0;" ::"n"(kConsumerWarps * 32) : "memory");
+  }
+}
+
+// ------------------------------------------------------------------ host side
+
+namespace {
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = [] {
+    void *p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &q) != cudaSuccess ||
+        q != cudaDriverEntryPointSuccess)
+      p = nullptr;
+    return reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  }();
+  return fn;
+}
+
+// 2-D view [L * H_kv * S_total rows][d] of one cache tensor, boxes of 128 rows x 64 columns
+bool make_map(CUtensorMap *m, const void *base, int d, int64_t rows) {
+  auto fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[2] = {(cuuint64_t)d, (cuuint64_t)rows};
+  cuuint64_t strides[1] = {(cuuint64_t)d * 2};
+  cuuint32_t box[2] = {64, (cuuint32_t)kTile};
+  cuuint32_t estr[2] = {1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(base), dims, strides, box,
+            estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+template <int D, int G>
+cudaError_t launch_mma_typed(const CUtensorMap &mk, const CUtensorMap &mv, const AttendArgs &a,
+                             int total, int grid, cudaStream_t s) {
+  auto kern = attend_mma_kernel<D, G>;
+  cudaError_t e =
+      cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, MmaCfg<D>::kSmem);
+  if (e != cudaSuccess) return e;
+  kern<<<grid, kThreads, MmaCfg<D>::kSmem, s>>>(mk, mv, a, total);
+  return cudaGetLastError();
+}
+
+template <int D>
+cudaError_t launch_mma_d(const CUtensorMap &mk, const CUtensorMap &mv, const AttendArgs &a, int g,
+                         int total, int grid, cudaStream_t s) {
+  switch (g) {
+    case 1: return launch_mma_typed<D, 1>(mk, mv, a, total, grid, s);
+    case 2: return launch_mma_typed<D, 2>(mk, mv, a, total, grid, s);
+    case 3: return launch_mma_typed<D, 3>(mk, mv, a, total, grid, s);
+    case 4: return launch_mma_typed<D, 4>(mk, mv, a, total, grid, s);
+    case 5: return launch_mma_typed<D, 5>(mk, mv, a, total, grid, s);
+    case 6: return launch_mma_typed<D, 6>(mk, mv, a, total, grid, s);
+    case 7: return launch_mma_typed<D, 7>(mk, mv, a, total, grid, s);
+    case 8: return launch_mma_typed<D, 8>(mk, mv, a, total, grid, s);
+  }
+  return cudaErrorInvalidValue;
+}
+
+}  // namespace
+
+int mma_tile_rows() { return kTile; }
+
+cudaError_t launch_attend_mma_partial(const AttendArgs &a, int d, int g, int64_t rows_total,
+                                      cudaStream_t s) {
+  CUtensorMap mk, mv;
+  if (!make_map(&mk, a.K, d, rows_total) || !make_map(&mv, a.V, d, rows_total))
+    return cudaErrorInvalidValue;
+  int dev = 0, sms = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  if (e != cudaSuccess) return e;
+  const int total = a.n_layers * a.batch * a.H_kv * a.max_chunks;
+  const int grid = total < sms ? total : sms;
+  if (d == 128) return launch_mma_d<128>(mk, mv, a, g, total, grid, s);
+  if (d == 64) return launch_mma_d<64>(mk, mv, a, g, total, grid, s);
+  return cudaErrorInvalidValue;
+}
+
+}  // namespace lg

@@ -125,21 +125,28 @@ struct DetectArgs {
   int nwords, thr, smem_rows;
 };
 
-constexpr int kDetectThreads = 256;
+constexpr int kDetectThreads = 1024;
 
 // Hamming distance of two sketch rows <= thr, stopping once it is exceeded
 __device__ __forceinline__ bool rows_match(const uint32_t *x, const uint32_t *y, int nwords,
                                            int thr) {
   int dist = 0;
-  for (int w = 0; w < nwords; ++w) {
-    dist += __popc(x[w] ^ y[w]);
+  int w = 0;
+  for (; w + 4 <= nwords; w += 4) {
+    dist += __popc(x[w] ^ y[w]) + __popc(x[w + 1] ^ y[w + 1]) + __popc(x[w + 2] ^ y[w + 2]) +
+            __popc(x[w + 3] ^ y[w + 3]);
     if (dist > thr) return false;
   }
-  return true;
+  for (; w < nwords; ++w) dist += __popc(x[w] ^ y[w]);
+  return dist <= thr;
 }
 
+// One CTA per sequence.  The sketches of the last smem_rows rows are staged in shared memory
+// with a row stride of nwords + 1 words (rows that different lanes read fall in different
+// banks); the novelty test runs over all (i, j) row pairs of the window and the period test
+// over all (P, i) pairs, spread over the CTA's threads.
 __global__ void __launch_bounds__(kDetectThreads) detect_kernel(DetectArgs a) {
-  extern __shared__ __align__(16) uint32_t sk_s[];  // rows [lo_s, n) of the sketches
+  extern __shared__ __align__(16) uint32_t sk_s[];
   __shared__ double red_e[kDetectThreads / 32], red_l[kDetectThreads / 32];
   __shared__ int s_novel, s_novel_tail, s_pstar, s_mismatch, s_trig;
   const int b = blockIdx.x, tid = threadIdx.x;
@@ -147,9 +154,15 @@ __global__ void __launch_bounds__(kDetectThreads) detect_kernel(DetectArgs a) {
   const lg_guard_params &p = a.p;
   const int n = a.c.len[b];
   const int B = a.budget[b];
-  const int nw = a.nwords, thr = a.thr;
+  const int nw = a.nwords, thr = a.thr, stride = nw + 1;
   const uint32_t *sk_g = a.c.sketch + a.c.seq_off[b] * nw;
   const int lo_s = max(0, n - a.smem_rows);
+  const int w = min(p.W, n);
+  const int wlo = n - w;
+  const int np = p.p_max - p.p_min + 1;
+  const int span_max = max(p.m_rep * p.p_max, p.l_min);
+  unsigned char *s_match = reinterpret_cast<unsigned char *>(sk_s + (size_t)a.smem_rows * stride);
+  unsigned char *s_fail = s_match + p.W;
 
   // (1) mean normalised entropy and mean suffix lift over every layer and head (fp64)
   const int Ws = min(p.suffix_w, n);
@@ -177,35 +190,47 @@ __global__ void __launch_bounds__(kDetectThreads) detect_kernel(DetectArgs a) {
     s_mismatch = -1;
   }
   // (2) stage the sketches of the rows the window and the period search read
-  for (int t = tid; t < (n - lo_s) * nw; t += kDetectThreads) sk_s[t] = sk_g[(int64_t)lo_s * nw + t];
+  for (int t = tid; t < (n - lo_s) * nw; t += kDetectThreads)
+    sk_s[(t / nw) * stride + t % nw] = sk_g[(int64_t)lo_s * nw + t];
+  for (int t = tid; t < w; t += kDetectThreads) s_match[t] = 0;
+  for (int t = tid; t < np; t += kDetectThreads) s_fail[t] = 0;
   __syncthreads();
   auto row = [&](int i) -> const uint32_t * {
-    return i >= lo_s ? sk_s + (int64_t)(i - lo_s) * nw : sk_g + (int64_t)i * nw;
+    return i >= lo_s ? sk_s + (int64_t)(i - lo_s) * stride : sk_g + (int64_t)i * nw;
   };
 
-  // (3) novelty over the window [n - w, n): a row is novel when no earlier window row matches
-  const int w = min(p.W, n);
-  const int wlo = n - w;
-  for (int i = wlo + tid; i < n; i += kDetectThreads) {
-    bool novel = true;
-    const uint32_t *ri = row(i);
-    for (int j = wlo; j < i; ++j)
-      if (rows_match(ri, row(j), nw, thr)) {
-        novel = false;
-        break;
-      }
-    if (novel) {
-      atomicAdd(&s_novel, 1);
-      if (i >= n - p.stall_len) atomicAdd(&s_novel_tail, 1);
-    }
+  // (3) novelty: row i of the window is novel when no earlier window row matches it
+  for (int cell = tid; cell < w * w; cell += kDetectThreads) {
+    const int ii = cell / w, jj = cell % w;
+    if (jj >= ii || s_match[ii]) continue;
+    if (rows_match(row(wlo + ii), row(wlo + jj), nw, thr)) s_match[ii] = 1;
   }
-  // (4) smallest period P whose last max(m_rep P, l_min) rows each match the row P earlier
-  for (int P = p.p_min + tid; P <= p.p_max; P += kDetectThreads) {
+  // (4) period test: P fails when one of its last max(m_rep P, l_min) rows does not match the
+  // row P earlier, or when the sequence is too short for the test
+  for (int cell = tid; cell < np * span_max; cell += kDetectThreads) {
+    const int pi = cell / span_max, k = cell % span_max;
+    const int P = p.p_min + pi;
     const int span_len = max(p.m_rep * P, p.l_min);
-    if (n < span_len + P) continue;
-    bool all = true;
-    for (int i = n - span_len; i < n && all; ++i) all = rows_match(row(i), row(i - P), nw, thr);
-    if (all) atomicMin(&s_pstar, P);
+    if (k >= span_len || s_fail[pi]) continue;
+    if (n < span_len + P) {
+      s_fail[pi] = 1;
+      continue;
+    }
+    const int i = n - span_len + k;
+    if (!rows_match(row(i), row(i - P), nw, thr)) s_fail[pi] = 1;
+  }
+  __syncthreads();
+  {
+    int nov = 0, nov_tail = 0;
+    for (int t = tid; t < w; t += kDetectThreads) {
+      const int novel = !s_match[t];
+      nov += novel;
+      if (wlo + t >= n - p.stall_len) nov_tail += novel;
+    }
+    if (nov) atomicAdd(&s_novel, nov);
+    if (nov_tail) atomicAdd(&s_novel_tail, nov_tail);
+    for (int t = tid; t < np; t += kDetectThreads)
+      if (!s_fail[t]) atomicMin(&s_pstar, p.p_min + t);
   }
   __syncthreads();
 
@@ -297,6 +322,11 @@ __global__ void __launch_bounds__(kDetectThreads) detect_kernel(DetectArgs a) {
 int detect_smem_rows(const lg_guard_params &p) {
   const int tail = max(p.m_rep * p.p_max, p.l_min) + p.p_max;
   return max(p.W, tail);
+}
+
+size_t detect_smem_bytes(const lg_guard_params &p, int nwords) {
+  const size_t rows = (size_t)detect_smem_rows(p) * (nwords + 1) * 4;
+  return rows + (size_t)p.W + (size_t)(p.p_max - p.p_min + 1) + 16;
 }
 
 // ------------------------------------------------------------------ retained set I_keep
@@ -698,7 +728,7 @@ cudaError_t launch_detect(const lg_cache &c, const float *stats, int H_q, lg_gua
   a.nwords = c.H_kv * c.d / 32;
   a.thr = (int)floor(p.tau_ham * (double)(a.nwords * 32));
   a.smem_rows = detect_smem_rows(p);
-  const size_t smem = (size_t)a.smem_rows * a.nwords * 4;
+  const size_t smem = detect_smem_bytes(p, a.nwords);
   cudaError_t e = cudaFuncSetAttribute(detect_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)smem);
   if (e != cudaSuccess) return e;

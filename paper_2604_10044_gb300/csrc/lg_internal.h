@@ -25,8 +25,12 @@ struct AttendArgs {
 };
 
 int attend_tile_rows(int dtype, int d);
-cudaError_t launch_attend(const AttendArgs &a, int dtype, int d, int g, void *out, float *stats,
-                          float *final_ml, float *h2o, cudaStream_t s);
+cudaError_t launch_attend(const AttendArgs &a, int dtype, int d, int g, int64_t rows_total,
+                          void *out, float *stats, float *final_ml, float *h2o, cudaStream_t s);
+// tensor-core partial pass for bf16 caches (lg_attend_mma.cu)
+int mma_tile_rows();
+cudaError_t launch_attend_mma_partial(const AttendArgs &a, int d, int g, int64_t rows_total,
+                                      cudaStream_t s);
 
 // guard kernels (lg_guard.cu)
 cudaError_t launch_begin_step(const lg_cache &c, cudaStream_t s);
@@ -40,6 +44,7 @@ cudaError_t launch_detect(const lg_cache &c, const float *stats, int H_q, lg_gua
                           const int32_t *budget, const lg_guard_params &p, int32_t *flags,
                           int32_t *spans, double *diag, cudaStream_t s);
 int detect_smem_rows(const lg_guard_params &p);
+size_t detect_smem_bytes(const lg_guard_params &p, int nwords);
 cudaError_t launch_prune_compact(const lg_cache &c, const int32_t *flags, const int32_t *spans,
                                  const lg_guard_state *state, const int32_t *budget,
                                  const lg_guard_params &p, int32_t *kept_idx,
