@@ -221,6 +221,27 @@ LG_API lg_status lg_h2o_reset(const lg_cache *c, int max_len, cudaStream_t s);
 LG_API lg_status lg_h2o_evict(const lg_cache *c, const int32_t *budget, const int32_t *pos_now,
                        int max_len, cudaStream_t s);
 
+/* Maximum scratch of lg_decode_attend_noalloc: 32 MiB of device memory per GPU. */
+#define LG_NOALLOC_SCRATCH_BYTES (32u << 20)
+
+/* lg_decode_attend for callers that cannot allocate device memory (a plugin inside a framework
+   that owns every device allocation, or a latency-critical loop that cannot take cudaMalloc's
+   implicit synchronisation).  The paper has no counterpart; this is a deployment variant.
+   Same arguments and results as lg_decode_attend, without ws / ws_bytes: the scratch is a
+   statically sized array of this library (LG_NOALLOC_SCRATCH_BYTES per GPU that loads the
+   library, held until the process exits), and the call allocates nothing.
+   - A call whose workspace (lg_workspace_size) exceeds LG_NOALLOC_SCRATCH_BYTES returns
+     LG_ERR_WORKSPACE and launches nothing.
+   - The first call on each device looks up the array's device address (cudaGetSymbolAddress,
+     with that device current); make that first call before any stream capture.
+   - Every call on a device shares the one array, and it keeps the last call's contents (no
+     clearing is needed: every scratch byte read is written earlier in the same call).  Calls
+     that overlap on the GPU (different streams without ordering) race on it: order them. */
+LG_API lg_status lg_decode_attend_noalloc(const lg_cache *c, int layer0, int n_layers,
+                                          const void *q, int H_q, float scale, void *out,
+                                          float *stats, int suffix_w, int accumulate_h2o,
+                                          int max_len, cudaStream_t s);
+
 /* Copies *dev_status to *host_code after synchronising the stream. */
 LG_API lg_status lg_read_device_status(const lg_cache *c, int32_t *host_code, cudaStream_t s);
 

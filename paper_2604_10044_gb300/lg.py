@@ -73,6 +73,8 @@ def lib():
             "lg_h2o_reset": [P(LgCache), i32, vp],
             "lg_h2o_evict": [P(LgCache), vp, vp, i32, vp],
             "lg_read_device_status": [P(LgCache), vp, vp],
+            "lg_decode_attend_noalloc": [P(LgCache), i32, i32, vp, i32, ctypes.c_float, vp, vp,
+                                         i32, i32, i32, vp],
             "lg_status_string": [i32],
         }
         for name, args in sig.items():
@@ -89,7 +91,10 @@ def exported_symbols():
     """names of the C ABI functions declared in include/lg.h"""
     return ["lg_default_params", "lg_status_string", "lg_workspace_size", "lg_state_init",
             "lg_begin_step", "lg_append", "lg_sketch_build", "lg_decode_attend", "lg_detect",
-            "lg_prune_compact", "lg_h2o_reset", "lg_h2o_evict", "lg_read_device_status"]
+            "lg_prune_compact", "lg_h2o_reset", "lg_h2o_evict", "lg_read_device_status",
+            "lg_decode_attend_noalloc"]
+
+NOALLOC_SCRATCH_BYTES = 32 << 20  # LG_NOALLOC_SCRATCH_BYTES in include/lg.h
 
 
 def _ptr(t):
@@ -156,6 +161,14 @@ def lg_decode_attend(cache, layer0, n_layers, q, H_q, scale, out, stats, suffix_
     _call("lg_decode_attend", ctypes.byref(cache.c), layer0, n_layers, _ptr(q), H_q,
           float(scale), _ptr(out), _ptr(stats), suffix_w, accumulate_h2o, max_len, _ptr(ws),
           ws.numel() * ws.element_size(), _stream(stream))
+
+
+def lg_decode_attend_noalloc(cache, layer0, n_layers, q, H_q, scale, out, stats, suffix_w,
+                             accumulate_h2o, max_len, stream=None):
+    """lg_decode_attend with the library's own static scratch (no workspace argument)"""
+    _call("lg_decode_attend_noalloc", ctypes.byref(cache.c), layer0, n_layers, _ptr(q), H_q,
+          float(scale), _ptr(out), _ptr(stats), suffix_w, accumulate_h2o, max_len,
+          _stream(stream))
 
 
 def lg_detect(cache, stats, H_q, state, budget, params, flags, spans, diag=None, stream=None):
