@@ -193,6 +193,9 @@ class GpuBench:
         self.kn = torch.empty((L, b, w.H_kv, w.d), dtype=bf, device=dev)
         self.vn = torch.empty_like(self.kn)
         self.esz = 2 if w.dtype == "bf16" else 4
+        e = self.esz
+        self.sel = synth.Select3(w, self.seqs_d, self.pos_d, (self.q, self.kn, self.vn),
+                                 (w.H_q * w.d * e, w.H_kv * w.d * e, w.H_kv * w.d * e))
         torch.cuda.synchronize()
 
     def reset(self):
@@ -203,19 +206,14 @@ class GpuBench:
             synth.seqs_tensor(w.seqs, self.dev)), self.off_d, self.n0_d, int(w.n0.max()), self.s)
         lg.lg_sketch_build(self.cache, self.p, int(w.n0.max()))
         lg.lg_state_init(self.cache, self.guard.state, 64)
+        self.guard.dstate.zero_()
         self.pos_d.copy_(self.n0_d.to(torch.int64))
         self.cache.status.zero_()
         torch.cuda.synchronize()
 
     def select_inputs(self, t):
-        w = self.w
-        e = self.esz
-        synth.dev_select(w, self.seqs_d, self.pos_d, w.H_q * w.d * e, self.qA[t], self.qB[t],
-                         self.q, self.s)
-        synth.dev_select(w, self.seqs_d, self.pos_d, w.H_kv * w.d * e, self.kA[t], self.kB[t],
-                         self.kn, self.s)
-        synth.dev_select(w, self.seqs_d, self.pos_d, w.H_kv * w.d * e, self.vA[t], self.vB[t],
-                         self.vn, self.s)
+        self.sel((self.qA[t], self.kA[t], self.vA[t]), (self.qB[t], self.kB[t], self.vB[t]),
+                 self.s)
 
     def step(self, t, ev=None):
         """one guarded decode step; ev = (a0, a1, p0, p1) events around attend and prune"""
@@ -232,7 +230,7 @@ class GpuBench:
         if ev:
             ev[1].record(self.stream)
         lg.lg_detect(c, g.stats, w.H_q, g.state, self.budget_d, p, g.flags, g.spans, None,
-                     self.s)
+                     g.dstate, self.s)
         if ev:
             ev[2].record(self.stream)
         lg.lg_prune_compact(c, g.flags, g.spans, g.state, self.budget_d, p, g.kept_idx,
@@ -244,8 +242,8 @@ class GpuBench:
     # launches of this repository's kernels per step (harness + path)
     def launches_per_step(self):
         n_attend = math.ceil(self.w.L / self.nl) * 2       # partial + combine per call
-        path = 1 + 2 + n_attend + 1 + 2                     # begin, append(+sketch), attend,
-        harness = 3 + 1                                     # detect, keep+compact; select x3,
+        path = 1 + 1 + n_attend + 1 + 2                     # begin, append (+sketch), attend,
+        harness = 1 + 1                                     # detect, keep + compact; select,
         return path, harness                                # advance
 
     def replay_log(self, K):

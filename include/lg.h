@@ -187,10 +187,18 @@ LG_API lg_status lg_decode_attend(const lg_cache *c, int layer0, int n_layers, c
    state: device [batch]; budget: device [batch]; flags: device [batch] (1 = trigger);
    spans: device [batch][2] ([0,0) when empty).
    diag: nullable device [batch][8] fp64, per sequence {mean normalised entropy, mean suffix
-   lift, novel fraction, vote 1, vote 2, vote 3, Stall, P* (0 = no tail repetition)}. */
+   lift, novel fraction, vote 1, vote 2, vote 3, Stall, P* (0 = no tail repetition)}.
+   dstate: device, lg_detect_state_size bytes, zero-filled before the first call on a cache and
+   after any change of W or of the period range.  It carries the monitor from call to call (for
+   each slot the latest earlier matching row, for each period the trailing matching run), so a
+   step that appended one row costs O(W + p_max - p_min) row comparisons (Sec. 5.4); after a
+   prune, or any other change of a length, the call recomputes it from the sketches. */
 LG_API lg_status lg_detect(const lg_cache *c, const float *stats, int H_q, lg_guard_state *state,
                            const int32_t *budget, const lg_guard_params *p, int32_t *flags,
-                           int32_t *spans, double *diag, cudaStream_t s);
+                           int32_t *spans, double *diag, void *dstate, cudaStream_t s);
+
+/* Bytes of lg_detect's dstate: (batch * (p_max - p_min + 3) + S_total) 32-bit words. */
+LG_API size_t lg_detect_state_size(const lg_cache *c, const lg_guard_params *p);
 
 /* Retained set and in-place index-gather (Sec. 5.3, Eq. 10, Eq. 11) for every sequence with
    flags[b] = 1 or len[b] > budget[b]:

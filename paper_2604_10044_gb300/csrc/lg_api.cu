@@ -204,15 +204,22 @@ lg_status lg_decode_attend(const lg_cache *c, int layer0, int n_layers, const vo
 
 lg_status lg_detect(const lg_cache *c, const float *stats, int H_q, lg_guard_state *state,
                     const int32_t *budget, const lg_guard_params *p, int32_t *flags,
-                    int32_t *spans, double *diag, cudaStream_t s) {
+                    int32_t *spans, double *diag, void *dstate, cudaStream_t s) {
   lg_status st = check_cache(c);
   if (st != LG_OK) return st;
   if ((st = check_params(p)) != LG_OK) return st;
-  if (!c->sketch || !stats || !state || !budget || !flags || !spans) return LG_ERR_INVALID_ARG;
+  if (!c->sketch || !stats || !state || !budget || !flags || !spans || !dstate)
+    return LG_ERR_INVALID_ARG;
+  if ((uintptr_t)dstate & 3u) return LG_ERR_INVALID_ARG;
   if (H_q < 1 || H_q % c->H_kv) return LG_ERR_INVALID_ARG;
   if (lg::detect_smem_bytes(*p, c->H_kv * c->d / 32) > 200 * 1024) return LG_ERR_UNSUPPORTED;
   return cuda_status(
-      lg::launch_detect(*c, stats, H_q, state, budget, *p, flags, spans, diag, s));
+      lg::launch_detect(*c, stats, H_q, state, budget, *p, flags, spans, diag, dstate, s));
+}
+
+size_t lg_detect_state_size(const lg_cache *c, const lg_guard_params *p) {
+  if (check_cache(c) != LG_OK || check_params(p) != LG_OK) return 0;
+  return lg::detect_state_bytes(*c, *p);
 }
 
 lg_status lg_prune_compact(const lg_cache *c, const int32_t *flags, const int32_t *spans,

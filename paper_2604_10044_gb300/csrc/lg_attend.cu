@@ -283,17 +283,21 @@ attend_partial_kernel(AttendArgs a) {
 }
 
 // Merge the chunk partials of one (layer, sequence, query head): out = O / l and the
-// statistics {m, l, H, S} in natural units.
+// statistics {m, l, H, S} in natural units.  One warp per head, eight heads per block.
 template <typename T, int D>
 __global__ void attend_combine_kernel(AttendArgs a, void *out, float *stats, float *final_ml) {
-  const int h = blockIdx.x, b = blockIdx.y, lloc = blockIdx.z;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int64_t head = (int64_t)blockIdx.x * (blockDim.x >> 5) + warp;
+  if (head >= (int64_t)a.n_layers * a.batch * a.H_q) return;
   if (status_bad(a.status)) return;
+  const int b = (int)((head / a.H_q) % a.batch);
   const int n = a.len[b];
   if (n > a.max_len) return;
-  const int64_t head = ((int64_t)lloc * a.batch + b) * a.H_q + h;
+  constexpr int EPL = D / 32;
   if (n <= 0) {  // empty sequence: no attention; zero output, m = -inf
-    for (int e = threadIdx.x; e < D; e += blockDim.x) Elem<T>::store(out, head * D + e, 0.f);
-    if (threadIdx.x == 0) {
+#pragma unroll
+    for (int k = 0; k < EPL; ++k) Elem<T>::store(out, head * D + lane + 32 * k, 0.f);
+    if (lane == 0) {
       stats[head * 4] = -INFINITY;
       stats[head * 4 + 1] = stats[head * 4 + 2] = stats[head * 4 + 3] = 0.f;
     }
@@ -303,21 +307,22 @@ __global__ void attend_combine_kernel(AttendArgs a, void *out, float *stats, flo
   const float *pp = a.partial + head * a.max_chunks * (D + 8);
   float M = -INFINITY;
   for (int j = 0; j < nch; ++j) M = fmaxf(M, pp[j * (D + 8)]);
-  float l = 0.f, u = 0.f, sg = 0.f;
+  float l = 0.f, u = 0.f, sg = 0.f, o[EPL];
+#pragma unroll
+  for (int k = 0; k < EPL; ++k) o[k] = 0.f;
   for (int j = 0; j < nch; ++j) {
     const float *q = pp + j * (D + 8);
     const float f = exp2f(q[0] - M);
     l += f * q[1];
     u += f * (q[2] + (q[0] - M) * q[1]);
     sg += f * q[3];
+#pragma unroll
+    for (int k = 0; k < EPL; ++k) o[k] += f * q[8 + lane + 32 * k];
   }
   const float inv_l = 1.f / l;
-  for (int e = threadIdx.x; e < D; e += blockDim.x) {
-    float o = 0.f;
-    for (int j = 0; j < nch; ++j) o += exp2f(pp[j * (D + 8)] - M) * pp[j * (D + 8) + 8 + e];
-    Elem<T>::store(out, head * D + e, o * inv_l);
-  }
-  if (threadIdx.x == 0) {
+#pragma unroll
+  for (int k = 0; k < EPL; ++k) Elem<T>::store(out, head * D + lane + 32 * k, o[k] * inv_l);
+  if (lane == 0) {
     constexpr float kLn2 = 0.69314718055994530942f;
     float *st = stats + head * 4;
     st[0] = M * kLn2;
@@ -377,8 +382,9 @@ static cudaError_t launch_typed(const AttendArgs &a, int64_t rows_total, void *o
     kp<<<grid, C::kThreads, C::kSmem, s>>>(a);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
   }
-  attend_combine_kernel<T, D><<<dim3(a.H_q, a.batch, a.n_layers), D, 0, s>>>(a, out, stats,
-                                                                            final_ml);
+  const int64_t heads = (int64_t)a.n_layers * a.batch * a.H_q;
+  attend_combine_kernel<T, D><<<(unsigned)((heads + 7) / 8), 256, 0, s>>>(a, out, stats,
+                                                                          final_ml);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   if (h2o) {
     int gx = (a.max_len + 255) / 256;

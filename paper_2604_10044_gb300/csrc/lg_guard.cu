@@ -22,11 +22,39 @@ __global__ void begin_step_kernel(lg_cache c) {
     c.len[b] += 1;
 }
 
-// one thread per 16-byte chunk of a new row; the row goes to slot len[b] - 1
+// sketch word w of a row: sign bits of elements [32w, 32w+32) of the row flattened [H_kv][d]
+template <typename T>
+__device__ __forceinline__ uint32_t sketch_word(const void *row_base, int64_t head_stride, int d,
+                                                int w) {
+  uint32_t bits = 0;
+#pragma unroll 4
+  for (int j = 0; j < 32; ++j) {
+    const int e = w * 32 + j;
+    const int h = e / d, x = e % d;
+    bits |= Elem<T>::sign(row_base, (int64_t)h * head_stride + x) << j;
+  }
+  return bits;
+}
+
+// Blocks [0, row_blocks): one thread per 16-byte chunk of a new row, written to slot
+// len[b] - 1.  Blocks [row_blocks, row_blocks + batch) when the guard layer is in the call:
+// the sketch of that layer's new V row (read from v_new [n_layers][b][H_kv][d]).
+template <typename T>
 __global__ void append_kernel(lg_cache c, int layer0, int n_layers, const uint4 *k_new,
-                              const uint4 *v_new, const int32_t *pos_new) {
+                              const uint4 *v_new, const int32_t *pos_new, int row_blocks,
+                              int lguard) {
   if (status_bad(c.dev_status)) return;
-  const int cpr = c.d * (c.dtype == LG_BF16 ? 2 : 4) / 16;
+  if ((int)blockIdx.x >= row_blocks) {
+    const int b = blockIdx.x - row_blocks;
+    const int nwords = c.H_kv * c.d / 32;
+    const int slot = c.len[b] - 1;
+    if (slot < 0) return;
+    const T *row = (const T *)v_new + ((int64_t)lguard * c.batch + b) * c.H_kv * c.d;
+    for (int w = threadIdx.x; w < nwords; w += blockDim.x)
+      c.sketch[(c.seq_off[b] + slot) * nwords + w] = sketch_word<T>(row, c.d, c.d, w);
+    return;
+  }
+  const int cpr = c.d * (int)sizeof(T) / 16;
   const int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   const int64_t rows = (int64_t)n_layers * c.batch * c.H_kv;
   if (t >= rows * cpr) return;
@@ -47,33 +75,6 @@ __global__ void append_kernel(lg_cache c, int layer0, int n_layers, const uint4 
     c.pos[s] = pos_new[b];
     c.h2o[s] = 0.f;
   }
-}
-
-// sketch word w of a row: sign bits of elements [32w, 32w+32) of the row flattened [H_kv][d]
-template <typename T>
-__device__ __forceinline__ uint32_t sketch_word(const void *row_base, int64_t head_stride, int d,
-                                                int w) {
-  uint32_t bits = 0;
-#pragma unroll 4
-  for (int j = 0; j < 32; ++j) {
-    const int e = w * 32 + j;
-    const int h = e / d, x = e % d;
-    bits |= Elem<T>::sign(row_base, (int64_t)h * head_stride + x) << j;
-  }
-  return bits;
-}
-
-// sketch of the row just appended to the guard layer, read from v_new [n_layers][b][H_kv][d]
-template <typename T>
-__global__ void append_sketch_kernel(lg_cache c, int lguard, const void *v_new) {
-  const int b = blockIdx.x;
-  if (status_bad(c.dev_status)) return;
-  const int nwords = c.H_kv * c.d / 32;
-  const int slot = c.len[b] - 1;
-  if (slot < 0) return;
-  const T *row = (const T *)v_new + ((int64_t)lguard * c.batch + b) * c.H_kv * c.d;
-  for (int w = threadIdx.x; w < nwords; w += blockDim.x)
-    c.sketch[(c.seq_off[b] + slot) * nwords + w] = sketch_word<T>(row, c.d, c.d, w);
 }
 
 // sketches of rows [0, len[b]) of the guard layer, read from the cache
@@ -122,10 +123,11 @@ struct DetectArgs {
   lg_guard_params p;
   int32_t *flags, *spans;
   double *diag;
+  int32_t *dstate;
   int nwords, thr, smem_rows;
 };
 
-constexpr int kDetectThreads = 1024;
+constexpr int kDetectThreads = 512;
 
 // Hamming distance of two sketch rows <= thr, stopping once it is exceeded
 __device__ __forceinline__ bool rows_match(const uint32_t *x, const uint32_t *y, int nwords,
@@ -141,96 +143,145 @@ __device__ __forceinline__ bool rows_match(const uint32_t *x, const uint32_t *y,
   return dist <= thr;
 }
 
-// One CTA per sequence.  The sketches of the last smem_rows rows are staged in shared memory
+// One CTA per sequence, monitor state carried from call to call in dstate:
+//   lm[slot]  latest earlier row of the window (as it was when the row was examined) whose
+//             sketch matches the row, -1 if none.  Row i of the window [wlo, n) is novel iff
+//             lm[i] < wlo, and this stays true as the window start moves forward.
+//   run[P]    trailing rows (up to the test length) that match the row P earlier.
+//   synced    the length seen by the previous call.
+// When the length grew by exactly one row since the previous call, only the new row is
+// examined (one scan of the window, one comparison per period): O(W + P) row comparisons per
+// step.  Otherwise (first call, after a prune or any other change of the cache) the window and
+// the runs are recomputed: the sketches of the last smem_rows rows are staged in shared memory
 // with a row stride of nwords + 1 words (rows that different lanes read fall in different
-// banks); the novelty test runs over all (i, j) row pairs of the window and the period test
-// over all (P, i) pairs, spread over the CTA's threads.
+// banks), one warp scans each window row, one warp each period.
 __global__ void __launch_bounds__(kDetectThreads) detect_kernel(DetectArgs a) {
   extern __shared__ __align__(16) uint32_t sk_s[];
   __shared__ double red_e[kDetectThreads / 32], red_l[kDetectThreads / 32];
-  __shared__ int s_novel, s_novel_tail, s_pstar, s_mismatch, s_trig;
-  const int b = blockIdx.x, tid = threadIdx.x;
+  __shared__ int s_novel, s_novel_tail, s_pstar, s_mismatch, s_trig, s_latest;
+  constexpr int kWarps = kDetectThreads / 32;
+  const int b = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   if (status_bad(a.c.dev_status)) return;
   const lg_guard_params &p = a.p;
   const int n = a.c.len[b];
   const int B = a.budget[b];
   const int nw = a.nwords, thr = a.thr, stride = nw + 1;
   const uint32_t *sk_g = a.c.sketch + a.c.seq_off[b] * nw;
-  const int lo_s = max(0, n - a.smem_rows);
   const int w = min(p.W, n);
   const int wlo = n - w;
   const int np = p.p_max - p.p_min + 1;
-  const int span_max = max(p.m_rep * p.p_max, p.l_min);
-  unsigned char *s_match = reinterpret_cast<unsigned char *>(sk_s + (size_t)a.smem_rows * stride);
-  unsigned char *s_fail = s_match + p.W;
+  int32_t *ds = a.dstate + (int64_t)b * (np + 2);
+  int32_t *run = ds + 2;
+  int32_t *lm = a.dstate + (int64_t)a.c.batch * (np + 2) + a.c.seq_off[b];
+  const bool incr = n >= 1 && ds[0] + 1 == n;
+  // staged rows: the window and the period comparisons of the new row, or (recompute) every
+  // row the window and the period runs read
+  const int lo_s = max(0, n - (incr ? max(p.W, p.p_max + 1) : a.smem_rows));
 
-  // (1) mean normalised entropy and mean suffix lift over every layer and head (fp64)
-  const int Ws = min(p.suffix_w, n);
-  const double lnn = n >= 2 ? log((double)n) : 1.0;
+  // (1) sums of the entropies and suffix masses over every layer and head (fp64)
   double se = 0.0, sl = 0.0;
   const int nh = a.c.L * a.H_q;
   for (int t = tid; t < nh; t += kDetectThreads) {
-    const int layer = t / a.H_q, h = t % a.H_q;
+    const int layer = t / a.H_q, h = t - layer * a.H_q;
     const float *st = a.stats + (((int64_t)layer * a.c.batch + b) * a.H_q + h) * 4;
-    se += n >= 2 ? (double)st[2] / lnn : 1.0;
-    sl += Ws > 0 ? (double)st[3] * (double)n / (double)Ws : 0.0;
+    se += (double)st[2];
+    sl += (double)st[3];
   }
   for (int o = 16; o >= 1; o >>= 1) {
     se += __shfl_xor_sync(0xffffffffu, se, o);
     sl += __shfl_xor_sync(0xffffffffu, sl, o);
   }
-  if ((tid & 31) == 0) {
-    red_e[tid >> 5] = se;
-    red_l[tid >> 5] = sl;
+  if (lane == 0) {
+    red_e[warp] = se;
+    red_l[warp] = sl;
   }
   if (tid == 0) {
     s_novel = 0;
     s_novel_tail = 0;
     s_pstar = 0x7fffffff;
     s_mismatch = -1;
+    s_latest = -1;
   }
-  // (2) stage the sketches of the rows the window and the period search read
-  for (int t = tid; t < (n - lo_s) * nw; t += kDetectThreads)
-    sk_s[(t / nw) * stride + t % nw] = sk_g[(int64_t)lo_s * nw + t];
-  for (int t = tid; t < w; t += kDetectThreads) s_match[t] = 0;
-  for (int t = tid; t < np; t += kDetectThreads) s_fail[t] = 0;
+  for (int t = tid; t < (n - lo_s) * nw; t += kDetectThreads) {
+    const int r = t / nw;
+    sk_s[r * stride + (t - r * nw)] = sk_g[(int64_t)lo_s * nw + t];
+  }
   __syncthreads();
   auto row = [&](int i) -> const uint32_t * {
     return i >= lo_s ? sk_s + (int64_t)(i - lo_s) * stride : sk_g + (int64_t)i * nw;
   };
-
-  // (3) novelty: row i of the window is novel when no earlier window row matches it
-  for (int cell = tid; cell < w * w; cell += kDetectThreads) {
-    const int ii = cell / w, jj = cell % w;
-    if (jj >= ii || s_match[ii]) continue;
-    if (rows_match(row(wlo + ii), row(wlo + jj), nw, thr)) s_match[ii] = 1;
-  }
-  // (4) period test: P fails when one of its last max(m_rep P, l_min) rows does not match the
-  // row P earlier, or when the sequence is too short for the test
-  for (int cell = tid; cell < np * span_max; cell += kDetectThreads) {
-    const int pi = cell / span_max, k = cell % span_max;
-    const int P = p.p_min + pi;
-    const int span_len = max(p.m_rep * P, p.l_min);
-    if (k >= span_len || s_fail[pi]) continue;
-    if (n < span_len + P) {
-      s_fail[pi] = 1;
-      continue;
+  // latest j in [lo, i) whose row matches row i, or -1 (one warp, nearest rows first)
+  auto latest_match = [&](int i, int lo) -> int {
+    const uint32_t *ri = row(i);
+    for (int top = i - 1; top >= lo; top -= 32) {
+      const int j = top - lane;
+      const bool m = j >= lo && rows_match(ri, row(j), nw, thr);
+      const unsigned bal = __ballot_sync(0xffffffffu, m);
+      if (bal) return top - (__ffs(bal) - 1);
     }
-    const int i = n - span_len + k;
-    if (!rows_match(row(i), row(i - P), nw, thr)) s_fail[pi] = 1;
+    return -1;
+  };
+
+  if (incr) {
+    // (2) the new row n-1: its latest match in the window (one candidate row per thread),
+    // and every period's run
+    const int i = n - 1;
+    const uint32_t *ri = row(i);
+    for (int j = i - 1 - tid; j >= wlo; j -= kDetectThreads)
+      if (rows_match(ri, row(j), nw, thr)) {
+        atomicMax(&s_latest, j);
+        break;
+      }
+    for (int pi = tid; pi < np; pi += kDetectThreads) {
+      const int P = p.p_min + pi;
+      const int cap = max(p.m_rep * P, p.l_min);
+      const bool m = i - P >= 0 && rows_match(ri, row(i - P), nw, thr);
+      run[pi] = m ? min(run[pi] + 1, cap) : 0;
+    }
+    __syncthreads();
+    if (tid == 0) lm[i] = s_latest;
+  } else {
+    // (2') recompute: every window row's latest match, every period's trailing run
+    for (int i = wlo + warp; i < n; i += kWarps) {
+      const int j = latest_match(i, wlo);
+      if (lane == 0) lm[i] = j;
+    }
+    for (int pi = warp; pi < np; pi += kWarps) {
+      const int P = p.p_min + pi;
+      const int cap = max(p.m_rep * P, p.l_min);
+      int r = cap;
+      for (int k0 = 0; k0 < cap; k0 += 32) {
+        const int k = k0 + lane;
+        const int i = n - 1 - k;
+        const bool ok = k < cap && i - P >= 0 && rows_match(row(i), row(i - P), nw, thr);
+        const unsigned bad = __ballot_sync(0xffffffffu, !ok);
+        if (bad) {
+          r = min(cap, k0 + __ffs(bad) - 1);
+          break;
+        }
+      }
+      if (lane == 0) run[pi] = r;
+    }
   }
   __syncthreads();
+
+  // (3) novelty of the window rows, stall, and the smallest period with a full verified run
   {
     int nov = 0, nov_tail = 0;
-    for (int t = tid; t < w; t += kDetectThreads) {
-      const int novel = !s_match[t];
+    for (int i = wlo + tid; i < n; i += kDetectThreads) {
+      const int novel = lm[i] < wlo;
       nov += novel;
-      if (wlo + t >= n - p.stall_len) nov_tail += novel;
+      if (i >= n - p.stall_len) nov_tail += novel;
     }
-    if (nov) atomicAdd(&s_novel, nov);
-    if (nov_tail) atomicAdd(&s_novel_tail, nov_tail);
-    for (int t = tid; t < np; t += kDetectThreads)
-      if (!s_fail[t]) atomicMin(&s_pstar, p.p_min + t);
+    nov = __reduce_add_sync(0xffffffffu, nov);
+    nov_tail = __reduce_add_sync(0xffffffffu, nov_tail);
+    if (lane == 0 && nov) atomicAdd(&s_novel, nov);
+    if (lane == 0 && nov_tail) atomicAdd(&s_novel_tail, nov_tail);
+    for (int pi = tid; pi < np; pi += kDetectThreads) {
+      const int P = p.p_min + pi;
+      const int span_len = max(p.m_rep * P, p.l_min);
+      if (n >= span_len + P && run[pi] >= span_len) atomicMin(&s_pstar, P);
+    }
   }
   __syncthreads();
 
@@ -243,8 +294,10 @@ __global__ void __launch_bounds__(kDetectThreads) detect_kernel(DetectArgs a) {
     }
     int trig = 0;
     if (n >= 1) {
-      const double ebar = e_sum / (double)nh;
-      const double lbar = l_sum / (double)nh;
+      // mean of H / ln n and of S * n / W_s over every layer and head
+      const int Ws = min(p.suffix_w, n);
+      const double ebar = n >= 2 ? e_sum / ((double)nh * log((double)n)) : 1.0;
+      const double lbar = l_sum * (double)n / ((double)Ws * (double)nh);
       const double ttr = (double)s_novel / (double)w;
       const int sig1 = ttr < p.theta_ttr;
       const int sig2 = ebar < p.theta_ent;
@@ -316,6 +369,7 @@ __global__ void __launch_bounds__(kDetectThreads) detect_kernel(DetectArgs a) {
     }
     st.t_gen += 1;
     a.state[b] = st;
+    ds[0] = n;
   }
 }
 
@@ -325,8 +379,12 @@ int detect_smem_rows(const lg_guard_params &p) {
 }
 
 size_t detect_smem_bytes(const lg_guard_params &p, int nwords) {
-  const size_t rows = (size_t)detect_smem_rows(p) * (nwords + 1) * 4;
-  return rows + (size_t)p.W + (size_t)(p.p_max - p.p_min + 1) + 16;
+  return (size_t)detect_smem_rows(p) * (nwords + 1) * 4;
+}
+
+size_t detect_state_bytes(const lg_cache &c, const lg_guard_params &p) {
+  const int64_t np = p.p_max - p.p_min + 1;
+  return (size_t)((int64_t)c.batch * (np + 2) + c.S_total) * sizeof(int32_t);
 }
 
 // ------------------------------------------------------------------ retained set I_keep
@@ -435,58 +493,65 @@ constexpr int kCompactThreads = 256;
 constexpr int kCompactChunks = 4;  // 16-byte chunks per thread per tile
 
 // Stream (sequence b, one of 2*L*H_kv K/V streams or the sketch stream): slot j <- row kept[j]
-// for j >= j0, tiles in ascending order.  kept[] is strictly increasing with kept[j] >= j,
+// for j >= j0, tiles in ascending order; CTAs take (sequence, stream) items grid-stride.  kept[] is strictly increasing with kept[j] >= j,
 // so a tile reads only rows at or above its own first slot: once every load of the tile is
 // performed (the barrier) its stores cannot clobber a row another tile still needs.
 __global__ void __launch_bounds__(kCompactThreads) compact_kernel(lg_cache c,
                                                                   const int32_t *kept_idx,
                                                                   const int32_t *kept_count,
                                                                   int max_keep) {
-  const int b = blockIdx.y, stream = blockIdx.x, tid = threadIdx.x;
+  const int tid = threadIdx.x;
   if (status_bad(c.dev_status)) return;
-  const int cnt = kept_count[b];
-  if (cnt < 0) return;
   const int row_bytes_kv = c.d * (c.dtype == LG_BF16 ? 2 : 4);
   const int nwords = c.H_kv * c.d / 32;
   const int n_kv = 2 * c.L * c.H_kv;
-  unsigned char *base;
-  int row_bytes;
-  if (stream < n_kv) {
-    const int lh = stream >> 1;
-    unsigned char *t = (unsigned char *)((stream & 1) ? c.v : c.k);
-    base = t + ((int64_t)lh * c.S_total + c.seq_off[b]) * row_bytes_kv;
-    row_bytes = row_bytes_kv;
-  } else {
-    if (!c.sketch) return;
-    base = (unsigned char *)(c.sketch + c.seq_off[b] * nwords);
-    row_bytes = nwords * 4;
-  }
-  const int32_t *kept = kept_idx + (int64_t)b * max_keep;
-  // first slot that moves: kept[j] == j exactly for j < j0 (binary search)
-  int lo = 0, hi = cnt;
-  while (lo < hi) {
-    const int mid = (lo + hi) >> 1;
-    if (kept[mid] == mid) lo = mid + 1;
-    else hi = mid;
-  }
-  const int j0 = lo;
-  const int cpr = row_bytes / 16;
-  const int rows_per_tile = kCompactThreads * kCompactChunks / cpr;
-  for (int t0 = j0; t0 < cnt; t0 += rows_per_tile) {
-    uint4 v[kCompactChunks];
-#pragma unroll
-    for (int k = 0; k < kCompactChunks; ++k) {
-      const int ci = k * kCompactThreads + tid;
-      const int j = t0 + ci / cpr;
-      if (j < cnt)
-        v[k] = *reinterpret_cast<const uint4 *>(base + (int64_t)kept[j] * row_bytes + (ci % cpr) * 16);
+  const int per_seq = n_kv + 1;
+  // grid-stride over (sequence, stream); sequences left as they were cost one load each
+  for (int item = blockIdx.x; item < c.batch * per_seq; item += gridDim.x) {
+    const int b = item / per_seq, stream = item - b * per_seq;
+    const int cnt = kept_count[b];
+    if (cnt < 0) continue;
+    unsigned char *base;
+    int row_bytes;
+    if (stream < n_kv) {
+      const int lh = stream >> 1;
+      unsigned char *t = (unsigned char *)((stream & 1) ? c.v : c.k);
+      base = t + ((int64_t)lh * c.S_total + c.seq_off[b]) * row_bytes_kv;
+      row_bytes = row_bytes_kv;
+    } else {
+      if (!c.sketch) continue;
+      base = (unsigned char *)(c.sketch + c.seq_off[b] * nwords);
+      row_bytes = nwords * 4;
     }
-    __syncthreads();
+    const int32_t *kept = kept_idx + (int64_t)b * max_keep;
+    // first slot that moves: kept[j] == j exactly for j < j0 (binary search)
+    int lo = 0, hi = cnt;
+    while (lo < hi) {
+      const int mid = (lo + hi) >> 1;
+      if (kept[mid] == mid) lo = mid + 1;
+      else hi = mid;
+    }
+    const int j0 = lo;
+    const int cpr = row_bytes / 16;
+    const int rows_per_tile = kCompactThreads * kCompactChunks / cpr;
+    for (int t0 = j0; t0 < cnt; t0 += rows_per_tile) {
+      uint4 v[kCompactChunks];
 #pragma unroll
-    for (int k = 0; k < kCompactChunks; ++k) {
-      const int ci = k * kCompactThreads + tid;
-      const int j = t0 + ci / cpr;
-      if (j < cnt) *reinterpret_cast<uint4 *>(base + (int64_t)j * row_bytes + (ci % cpr) * 16) = v[k];
+      for (int k = 0; k < kCompactChunks; ++k) {
+        const int ci = k * kCompactThreads + tid;
+        const int j = t0 + ci / cpr;
+        if (j < cnt)
+          v[k] = *reinterpret_cast<const uint4 *>(base + (int64_t)kept[j] * row_bytes +
+                                                  (ci % cpr) * 16);
+      }
+      __syncthreads();
+#pragma unroll
+      for (int k = 0; k < kCompactChunks; ++k) {
+        const int ci = k * kCompactThreads + tid;
+        const int j = t0 + ci / cpr;
+        if (j < cnt)
+          *reinterpret_cast<uint4 *>(base + (int64_t)j * row_bytes + (ci % cpr) * 16) = v[k];
+      }
     }
   }
 }
@@ -677,20 +742,18 @@ cudaError_t launch_append(const lg_cache &c, int layer0, int n_layers, const voi
                           cudaStream_t s) {
   const int cpr = c.d * (c.dtype == LG_BF16 ? 2 : 4) / 16;
   const int64_t total = (int64_t)n_layers * c.batch * c.H_kv * cpr;
-  append_kernel<<<(unsigned)((total + 255) / 256), 256, 0, s>>>(
-      c, layer0, n_layers, (const uint4 *)k_new, (const uint4 *)v_new, pos_new);
-  cudaError_t e = cudaGetLastError();
-  if (e != cudaSuccess) return e;
-  if (c.sketch && guard_layer >= layer0 && guard_layer < layer0 + n_layers) {
-    const int nwords = c.H_kv * c.d / 32;
-    const int threads = nwords < 256 ? ((nwords + 31) / 32) * 32 : 256;
-    if (c.dtype == LG_BF16)
-      append_sketch_kernel<__nv_bfloat16><<<c.batch, threads, 0, s>>>(c, guard_layer - layer0, v_new);
-    else
-      append_sketch_kernel<float><<<c.batch, threads, 0, s>>>(c, guard_layer - layer0, v_new);
-    e = cudaGetLastError();
-  }
-  return e;
+  const int row_blocks = (int)((total + 255) / 256);
+  const bool sk = c.sketch && guard_layer >= layer0 && guard_layer < layer0 + n_layers;
+  const int grid = row_blocks + (sk ? c.batch : 0);
+  if (c.dtype == LG_BF16)
+    append_kernel<__nv_bfloat16><<<grid, 256, 0, s>>>(c, layer0, n_layers, (const uint4 *)k_new,
+                                                      (const uint4 *)v_new, pos_new, row_blocks,
+                                                      guard_layer - layer0);
+  else
+    append_kernel<float><<<grid, 256, 0, s>>>(c, layer0, n_layers, (const uint4 *)k_new,
+                                              (const uint4 *)v_new, pos_new, row_blocks,
+                                              guard_layer - layer0);
+  return cudaGetLastError();
 }
 
 cudaError_t launch_sketch_build(const lg_cache &c, int guard_layer, int max_len, cudaStream_t s) {
@@ -714,7 +777,7 @@ cudaError_t launch_state_init(const lg_cache &c, lg_guard_state *state, int t_ge
 
 cudaError_t launch_detect(const lg_cache &c, const float *stats, int H_q, lg_guard_state *state,
                           const int32_t *budget, const lg_guard_params &p, int32_t *flags,
-                          int32_t *spans, double *diag, cudaStream_t s) {
+                          int32_t *spans, double *diag, void *dstate, cudaStream_t s) {
   DetectArgs a;
   a.c = c;
   a.stats = stats;
@@ -725,6 +788,7 @@ cudaError_t launch_detect(const lg_cache &c, const float *stats, int H_q, lg_gua
   a.flags = flags;
   a.spans = spans;
   a.diag = diag;
+  a.dstate = (int32_t *)dstate;
   a.nwords = c.H_kv * c.d / 32;
   a.thr = (int)floor(p.tau_ham * (double)(a.nwords * 32));
   a.smem_rows = detect_smem_rows(p);
@@ -754,7 +818,11 @@ cudaError_t launch_prune_compact(const lg_cache &c, const int32_t *flags, const 
   keep_set_kernel<<<c.batch, kKeepThreads, 0, s>>>(a);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
-  dim3 grid(2 * c.L * c.H_kv + 1, c.batch);
+  int dev = 0, sms = 152;
+  if (cudaGetDevice(&dev) == cudaSuccess)
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  const int items = c.batch * (2 * c.L * c.H_kv + 1);
+  const int grid = items < 4 * sms ? items : 4 * sms;
   compact_kernel<<<grid, kCompactThreads, 0, s>>>(c, kept_idx, kept_count, max_keep);
   return cudaGetLastError();
 }

@@ -42,7 +42,8 @@ cudaError_t launch_state_init(const lg_cache &c, lg_guard_state *state, int t_ge
                               cudaStream_t s);
 cudaError_t launch_detect(const lg_cache &c, const float *stats, int H_q, lg_guard_state *state,
                           const int32_t *budget, const lg_guard_params &p, int32_t *flags,
-                          int32_t *spans, double *diag, cudaStream_t s);
+                          int32_t *spans, double *diag, void *dstate, cudaStream_t s);
+size_t detect_state_bytes(const lg_cache &c, const lg_guard_params &p);
 int detect_smem_rows(const lg_guard_params &p);
 size_t detect_smem_bytes(const lg_guard_params &p, int nwords);
 cudaError_t launch_prune_compact(const lg_cache &c, const int32_t *flags, const int32_t *spans,

@@ -67,7 +67,8 @@ def lib():
             "lg_sketch_build": [P(LgCache), P(LgGuardParams), i32, vp],
             "lg_decode_attend": [P(LgCache), i32, i32, vp, i32, ctypes.c_float, vp, vp, i32, i32,
                                  i32, vp, ctypes.c_size_t, vp],
-            "lg_detect": [P(LgCache), vp, i32, vp, vp, P(LgGuardParams), vp, vp, vp, vp],
+            "lg_detect": [P(LgCache), vp, i32, vp, vp, P(LgGuardParams), vp, vp, vp, vp, vp],
+            "lg_detect_state_size": [P(LgCache), P(LgGuardParams)],
             "lg_prune_compact": [P(LgCache), vp, vp, vp, vp, P(LgGuardParams), vp, vp, i32, i32,
                                  vp],
             "lg_h2o_reset": [P(LgCache), i32, vp],
@@ -82,6 +83,7 @@ def lib():
             f.argtypes = args
             f.restype = ctypes.c_int
         L.lg_workspace_size.restype = ctypes.c_size_t
+        L.lg_detect_state_size.restype = ctypes.c_size_t
         L.lg_status_string.restype = ctypes.c_char_p
         _lib = L
     return _lib
@@ -92,7 +94,7 @@ def exported_symbols():
     return ["lg_default_params", "lg_status_string", "lg_workspace_size", "lg_state_init",
             "lg_begin_step", "lg_append", "lg_sketch_build", "lg_decode_attend", "lg_detect",
             "lg_prune_compact", "lg_h2o_reset", "lg_h2o_evict", "lg_read_device_status",
-            "lg_decode_attend_noalloc"]
+            "lg_decode_attend_noalloc", "lg_detect_state_size"]
 
 NOALLOC_SCRATCH_BYTES = 32 << 20  # LG_NOALLOC_SCRATCH_BYTES in include/lg.h
 
@@ -171,9 +173,14 @@ def lg_decode_attend_noalloc(cache, layer0, n_layers, q, H_q, scale, out, stats,
           _stream(stream))
 
 
-def lg_detect(cache, stats, H_q, state, budget, params, flags, spans, diag=None, stream=None):
+def lg_detect_state_size(cache, params) -> int:
+    return int(lib().lg_detect_state_size(ctypes.byref(cache.c), ctypes.byref(params)))
+
+
+def lg_detect(cache, stats, H_q, state, budget, params, flags, spans, diag, dstate, stream=None):
     _call("lg_detect", ctypes.byref(cache.c), _ptr(stats), H_q, _ptr(state), _ptr(budget),
-          ctypes.byref(params), _ptr(flags), _ptr(spans), _ptr(diag), _stream(stream))
+          ctypes.byref(params), _ptr(flags), _ptr(spans), _ptr(diag), _ptr(dstate),
+          _stream(stream))
 
 
 def lg_prune_compact(cache, flags, spans, state, budget, params, kept_idx, kept_count, max_keep,
@@ -298,6 +305,8 @@ class Guard:
         self.kept_idx = torch.zeros((b, self.max_keep), dtype=torch.int32, device=dev)
         self.kept_count = torch.zeros(b, dtype=torch.int32, device=dev)
         self.diag = torch.zeros((b, 8), dtype=torch.float64, device=dev)
+        ds_words = lg_detect_state_size(cache, self.p) // 4 if policy != "h2o" else 1
+        self.dstate = torch.zeros(ds_words, dtype=torch.int32, device=dev)
         tdt = _torch_dtype(cache.dtype)
         self.out = torch.zeros((L, b, H_q, cache.d), dtype=tdt, device=dev)
         self.stats = torch.zeros((L, b, H_q, 4), dtype=torch.float32, device=dev)
@@ -320,7 +329,7 @@ class Guard:
                              self.max_len, self.ws, stream)
         if self.policy == "loopguard":
             lg_detect(c, self.stats, self.H_q, self.state, budget, p, self.flags, self.spans,
-                      self.diag, stream)
+                      self.diag, self.dstate, stream)
             lg_prune_compact(c, self.flags, self.spans, self.state, budget, p, self.kept_idx,
                              self.kept_count, self.max_keep, self.max_len, stream)
         elif self.policy == "h2o":

@@ -351,8 +351,9 @@ def dev_lib():
                                      vp]
         lib.syn_dev_advance.argtypes = [vp, i32, vp, vp, vp]
         lib.syn_dev_select.argtypes = [vp, i32, vp, i32, i64, vp, vp, vp, vp]
+        lib.syn_dev_select3.argtypes = [vp, i32, vp, i32, vp, vp, vp, vp, vp]
         for f in (lib.syn_dev_fill_cache, lib.syn_dev_step, lib.syn_dev_advance,
-                  lib.syn_dev_select):
+                  lib.syn_dev_select, lib.syn_dev_select3):
             f.restype = ctypes.c_int
         _dev = lib
     return _dev
@@ -395,6 +396,26 @@ def dev_select(w: Workload, seqs_dev, pos_dev, rowlen_bytes: int, loop_buf, fres
     _check(dev_lib().syn_dev_select(seqs_dev.data_ptr(), w.batch, pos_dev.data_ptr(), w.L,
                                     rowlen_bytes, loop_buf.data_ptr(), fresh_buf.data_ptr(),
                                     out.data_ptr(), stream), "syn_dev_select")
+
+
+class Select3:
+    """one launch that picks each sequence's inputs of a step (q, k_new, v_new) from the
+    loop-continuing or the loop-free variant; argument arrays marshalled once"""
+
+    def __init__(self, w, seqs_dev, pos_dev, outs, rowlens):
+        self.w, self.seqs, self.pos = w, seqs_dev, pos_dev
+        self.rowlens = (ctypes.c_int64 * 3)(*rowlens)
+        self.outs = (ctypes.c_void_p * 3)(*[o.data_ptr() for o in outs])
+        self.loop = (ctypes.c_void_p * 3)()
+        self.fresh = (ctypes.c_void_p * 3)()
+
+    def __call__(self, loop_bufs, fresh_bufs, stream):
+        for k in range(3):
+            self.loop[k] = loop_bufs[k].data_ptr()
+            self.fresh[k] = fresh_bufs[k].data_ptr()
+        _check(dev_lib().syn_dev_select3(self.seqs.data_ptr(), self.w.batch, self.pos.data_ptr(),
+                                         self.w.L, self.rowlens, self.loop, self.fresh,
+                                         self.outs, stream), "syn_dev_select3")
 
 
 def build(out_dir: str = _HERE, jobs=None):

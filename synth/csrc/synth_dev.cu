@@ -87,9 +87,49 @@ __global__ void select_kernel(const syn_seq *seqs, int batch, const int64_t *pos
   ((uint4 *)out)[t] = ((const uint4 *)src)[t];
 }
 
+// the three selections of one step (q, k_new, v_new) in one launch
+struct Sel3 {
+  const char *loop[3];
+  const char *fresh[3];
+  char *out[3];
+  int64_t chunks[3];  // 16-byte chunks per (layer, sequence) row of each tensor
+};
+
+__global__ void select3_kernel(const syn_seq *seqs, int batch, const int64_t *pos, int L, Sel3 s) {
+  int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  for (int k = 0; k < 3; ++k) {
+    const int64_t total = (int64_t)L * batch * s.chunks[k];
+    if (t < total) {
+      const int b = (int)((t / s.chunks[k]) % batch);
+      const char *src = pos[b] >= seqs[b].fresh_from ? s.fresh[k] : s.loop[k];
+      ((uint4 *)s.out[k])[t] = ((const uint4 *)src)[t];
+      return;
+    }
+    t -= total;
+  }
+}
+
 }  // namespace
 
 extern "C" {
+
+int syn_dev_select3(const syn_seq *seqs_dev, int batch, const int64_t *pos_dev, int L,
+                    const int64_t *rowlen_bytes, const void *const *loop_bufs,
+                    const void *const *fresh_bufs, void *const *outs, cudaStream_t stream) {
+  Sel3 s;
+  int64_t total = 0;
+  for (int k = 0; k < 3; ++k) {
+    if (rowlen_bytes[k] % 16) return 1;
+    s.loop[k] = (const char *)loop_bufs[k];
+    s.fresh[k] = (const char *)fresh_bufs[k];
+    s.out[k] = (char *)outs[k];
+    s.chunks[k] = rowlen_bytes[k] / 16;
+    total += (int64_t)L * batch * s.chunks[k];
+  }
+  select3_kernel<<<(unsigned)((total + 255) / 256), 256, 0, stream>>>(seqs_dev, batch, pos_dev, L,
+                                                                      s);
+  return cudaGetLastError() == cudaSuccess ? 0 : 2;
+}
 
 int syn_dev_fill_cache(const syn_workload *w, const syn_seq *seqs_dev, int batch,
                        const int64_t *seq_off_dev, const int32_t *n_rows_dev, int64_t S_total,

@@ -19,7 +19,7 @@ def declared():
 
 def test_every_declared_symbol_is_exported():
     names = declared()
-    assert len(names) == 14
+    assert len(names) == 15
     assert sorted(lg.exported_symbols()) == names
     L = lg.lib()
     for n in names:
@@ -58,6 +58,8 @@ def test_host_validation_rejects_before_launch():
                               fake, 1 << 30, None) == 1   # layers out of range
     p.p_max = 0
     assert L.lg_detect(ctypes.byref(c), fake, 32, fake, fake, ctypes.byref(p), fake, fake,
-                       None, None) == 1
+                       None, fake, None) == 1
+    p.p_max = 128
+    assert L.lg_detect_state_size(ctypes.byref(c), ctypes.byref(p)) == 4 * (130 + c.S_total)
     ws = L.lg_workspace_size(ctypes.byref(c), 32, 1, 1000, 0)
     assert ws > 0 and ws % 256 == 0
