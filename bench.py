@@ -288,7 +288,7 @@ def compact_bytes(w, kept_count, kept_idx):
 def traffic_from_profile(kernel_src_hash):
     """DRAM bytes per attend launch from the committed ncu summary, if it was taken on the
     current kernel source; else None"""
-    path = os.path.join(ROOT, "profiles", "attend_traffic.json")
+    path = os.path.join(ROOT, "profiles", "attend_mma_traffic.txt")
     if not os.path.exists(path):
         return None
     with open(path) as f:
@@ -301,7 +301,7 @@ def traffic_from_profile(kernel_src_hash):
 def source_hash():
     import hashlib
     h = hashlib.sha256()
-    for f in ("lg_attend.cu", "lg_common.cuh"):
+    for f in ("lg_attend_mma.cu", "lg_common.cuh"):
         with open(os.path.join(ROOT, "paper_2604_10044_gb300", "csrc", f), "rb") as fh:
             h.update(fh.read())
     return h.hexdigest()
@@ -379,10 +379,11 @@ def run_gpu(args, ws, rank, local):
     path_l, harness_l = bench.launches_per_step()
     prof = traffic_from_profile(source_hash())
     traffic = None
-    if prof:
-        # per-launch DRAM bytes scaled from the captured launch to this run's mean launch
-        traffic = prof["dram_bytes_per_row"] * (sum(a_bytes) / K) / attend_bytes(w, [1]) \
-            if "dram_bytes_per_row" in prof else None
+    if prof and bench.nl == w.L:
+        # DRAM bytes of one launch: per-row bytes of the captured (smaller) launch scaled by
+        # the K/V rows one launch of this run reads on average
+        rows_per_launch = sum(int(np.sum(l.cpu().numpy() + 1)) for l in lens) / K * w.L * w.H_kv
+        traffic = int(prof["dram_bytes_per_row"] * rows_per_launch)
     line = {
         "metric": METRIC, "value": round(value, 3), "unit": UNIT, "n_gpus": ws, "steps": K,
         "warmup": W, "ms_per_step": round(ms / K, 4), "higher_is_better": True,
