@@ -50,6 +50,9 @@ def parse():
     ap.add_argument("--no-clocks", action="store_true")
     ap.add_argument("--batch", type=int, default=0,
                     help="override the workload's batch (smaller cases for profiling)")
+    ap.add_argument("--fresh-each-step", action="store_true",
+                    help="time every step from a freshly generated cache (the first decode "
+                         "step: attention over the full prefill and the budget prune)")
     ap.add_argument("--profile-steps", type=int, default=0,
                     help="run this many steps untimed and exit (for ncu launch lists)")
     return ap.parse_args()
@@ -246,15 +249,17 @@ class GpuBench:
         harness = 1 + 1                                     # detect, keep + compact; select,
         return path, harness                                # advance
 
-    def replay_log(self, K):
+    def replay_log(self, K, fresh=False):
         """replay the timed trajectory untimed, recording per-step lengths and kept lists
         (the decisions are deterministic, so they are the timed run's)"""
         torch = self.torch
         self.reset()
         lens, kept = [], []
         for t in range(K):
+            if fresh:
+                self.reset()
             lens.append(self.cache.len.clone())
-            self.step(t)
+            self.step(0 if fresh else t)
             kc = self.guard.kept_count.clone()
             kept.append((kc, self.guard.kept_idx.clone() if int((kc >= 0).sum()) else None))
         torch.cuda.synchronize()
@@ -327,12 +332,15 @@ def run_gpu(args, ws, rank, local):
         torch.cuda.synchronize()
         torch.cuda.nvtx.range_pop()
         return None
-    bench = GpuBench(w, dev, max(K, W, 1), args.layers_per_call)
+    fresh = args.fresh_each_step
+    bench = GpuBench(w, dev, 1 if fresh else max(K, W, 1), args.layers_per_call)
 
     # warm-up on the trajectory's first W steps, then a fresh cache for the timed run
     bench.reset()
     for t in range(W):
-        bench.step(t)
+        if fresh:
+            bench.reset()
+        bench.step(0 if fresh else t)
     torch.cuda.synchronize()
     bench.reset()
     evs = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(K)]
@@ -340,23 +348,35 @@ def run_gpu(args, ws, rank, local):
     clocks = Clocks(local, enabled=not args.no_clocks)
     barrier(ws)
     torch.cuda.synchronize()
-    start.record(bench.stream)
-    for t in range(K):
-        bench.step(t, evs[t])
-    stop.record(bench.stream)
-    torch.cuda.synchronize()
+    if fresh:
+        # every step from a freshly generated cache; only the steps are timed
+        ms_local = 0.0
+        for t in range(K):
+            if t:
+                bench.reset()
+            start.record(bench.stream)
+            bench.step(0, evs[t])
+            stop.record(bench.stream)
+            torch.cuda.synchronize()
+            ms_local += start.elapsed_time(stop)
+    else:
+        start.record(bench.stream)
+        for t in range(K):
+            bench.step(t, evs[t])
+        stop.record(bench.stream)
+        torch.cuda.synchronize()
+        ms_local = start.elapsed_time(stop)
     barrier(ws)
     clk = clocks.stop()
     status = bench.lg.lg_read_device_status(bench.cache)
     if status != 0:
         raise RuntimeError("device status %d after the timed run" % status)
-    ms_local = start.elapsed_time(stop)
     ms = max_over_ranks(ms_local, ws)
     attend_ms = [e[0].elapsed_time(e[1]) for e in evs]
     prune_ms = [e[2].elapsed_time(e[3]) for e in evs]
 
     # algorithmic bytes of the same trajectory (untimed, deterministic replay)
-    lens, kept = bench.replay_log(K)
+    lens, kept = bench.replay_log(K, fresh)
     a_bytes, c_bytes, c_ms = [], [], []
     triggers = 0
     for t in range(K):
@@ -372,7 +392,7 @@ def run_gpu(args, ws, rank, local):
     compact_gbs = (sum(c_bytes) / (sum(c_ms) * 1e-3) / 1e9) if c_ms else None
 
     e2e = None
-    if not args.no_e2e:
+    if not args.no_e2e and not fresh:
         e2e = run_e2e(bench, K, ws)
 
     value = sum_over_ranks(K, ws) / (ms * 1e-3)
@@ -388,7 +408,9 @@ def run_gpu(args, ws, rank, local):
         "metric": METRIC, "value": round(value, 3), "unit": UNIT, "n_gpus": ws, "steps": K,
         "warmup": W, "ms_per_step": round(ms / K, 4), "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": w.dtype, "data": "synthetic",
-        "config": dict(w.describe(), l2="inputs larger than L2 (K/V cache 4.3-8.6 GB per GPU)",
+        "config": dict(w.describe(), l2="inputs larger than L2 (K/V cache %.1f GB per GPU)"
+                       % (w.kv_bytes() / 1e9), timed_steps="each from a fresh cache" if fresh
+                       else "consecutive decode steps from a fresh cache",
                        layers_per_attend_call=bench.nl, parallelism="dp%d (independent batches, "
                        "no collective)" % ws, tokens_per_step=w.batch * ws),
         "roofline": {"bound": "hbm", "achieved": round(attend_gbs, 1), "peak": hbm_peak,
