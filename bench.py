@@ -50,6 +50,9 @@ def parse():
     ap.add_argument("--no-clocks", action="store_true")
     ap.add_argument("--batch", type=int, default=0,
                     help="override the workload's batch (smaller cases for profiling)")
+    ap.add_argument("--policy", default="loopguard", choices=["loopguard", "h2o"],
+                    help="cache policy of the timed steps: LoopGuard, or the H2O comparator "
+                         "(accumulated-score eviction) on the same inputs")
     ap.add_argument("--fresh-each-step", action="store_true",
                     help="time every step from a freshly generated cache (the first decode "
                          "step: attention over the full prefill and the budget prune)")
@@ -163,17 +166,21 @@ class Clocks:
 class GpuBench:
     """Device buffers, the per-step input variants and one guarded step on the C ABI."""
 
-    def __init__(self, w, dev, total_steps, layers_per_call):
+    def __init__(self, w, dev, total_steps, layers_per_call, policy="loopguard"):
         import torch
         from paper_2604_10044_gb300 import lg
         self.torch, self.lg = torch, lg
         self.w, self.dev = w, dev
+        self.policy = policy
         self.stream = torch.cuda.current_stream()
         self.s = self.stream.cuda_stream
-        self.cache = lg.Cache(w.L, w.H_kv, w.d, w.dtype, w.seq_off, w.cap, w.n0, dev,
-                              "loopguard")
+        self.cache = lg.Cache(w.L, w.H_kv, w.d, w.dtype, w.seq_off, w.cap, w.n0, dev, policy)
         self.nl = layers_per_call if layers_per_call else w.L
-        self.guard = lg.Guard(self.cache, w.H_q, n_layers_per_call=self.nl)
+        self.guard = lg.Guard(self.cache, w.H_q, n_layers_per_call=self.nl, policy=policy)
+        # token positions of every step's new row (the same under either policy)
+        self.pos32 = torch.as_tensor(
+            (w.n0[None, :].astype(np.int64) + np.arange(max(total_steps, 1))[:, None]).astype(
+                np.int32), device=dev)
         self.p = self.guard.p
         self.off_d = torch.as_tensor(w.seq_off, device=dev)
         self.n0_d = torch.as_tensor(w.n0, device=dev)
@@ -207,7 +214,10 @@ class GpuBench:
         self.cache.len.copy_(self.n0_d)
         synth.dev_fill_cache(w, self.cache.k, self.cache.v, self.seqs_d.copy_(
             synth.seqs_tensor(w.seqs, self.dev)), self.off_d, self.n0_d, int(w.n0.max()), self.s)
-        lg.lg_sketch_build(self.cache, self.p, int(w.n0.max()))
+        if self.policy == "h2o":
+            lg.lg_h2o_reset(self.cache, int(w.n0.max()))
+        else:
+            lg.lg_sketch_build(self.cache, self.p, int(w.n0.max()))
         lg.lg_state_init(self.cache, self.guard.state, 64)
         self.guard.dstate.zero_()
         self.pos_d.copy_(self.n0_d.to(torch.int64))
@@ -221,33 +231,42 @@ class GpuBench:
     def step(self, t, ev=None):
         """one guarded decode step; ev = (a0, a1, p0, p1) events around attend and prune"""
         lg, c, g, p, w = self.lg, self.cache, self.guard, self.p, self.w
+        h2o = self.policy == "h2o"
+        pos_t = self.pos32[t] if h2o else None
         self.select_inputs(t)
         lg.lg_begin_step(c, self.s)
-        lg.lg_append(c, 0, w.L, self.kn, self.vn, None, p, self.s)
+        lg.lg_append(c, 0, w.L, self.kn, self.vn, pos_t, p, self.s)
         if ev:
             ev[0].record(self.stream)
         for l0 in range(0, w.L, self.nl):
             lg.lg_decode_attend(c, l0, self.nl, self.q[l0:l0 + self.nl], w.H_q, g.scale,
-                                g.out[l0:l0 + self.nl], g.stats[l0:l0 + self.nl], p.suffix_w, 0,
-                                g.max_len, g.ws, self.s)
+                                g.out[l0:l0 + self.nl], g.stats[l0:l0 + self.nl], p.suffix_w,
+                                1 if h2o else 0, g.max_len, g.ws, self.s)
         if ev:
             ev[1].record(self.stream)
-        lg.lg_detect(c, g.stats, w.H_q, g.state, self.budget_d, p, g.flags, g.spans, None,
-                     g.dstate, self.s)
+        if not h2o:
+            lg.lg_detect(c, g.stats, w.H_q, g.state, self.budget_d, p, g.flags, g.spans, None,
+                         g.dstate, self.s)
         if ev:
             ev[2].record(self.stream)
-        lg.lg_prune_compact(c, g.flags, g.spans, g.state, self.budget_d, p, g.kept_idx,
-                            g.kept_count, g.max_keep, g.max_len, self.s)
+        if h2o:
+            lg.lg_h2o_evict(c, self.budget_d, pos_t, g.max_len, self.s)
+        else:
+            lg.lg_prune_compact(c, g.flags, g.spans, g.state, self.budget_d, p, g.kept_idx,
+                                g.kept_count, g.max_keep, g.max_len, self.s)
         if ev:
             ev[3].record(self.stream)
-        synth.dev_advance(w, self.seqs_d, g.flags, self.pos_d, self.s)
+        synth.dev_advance(w, self.seqs_d, None if h2o else g.flags, self.pos_d, self.s)
 
     # launches of this repository's kernels per step (harness + path)
     def launches_per_step(self):
-        n_attend = math.ceil(self.w.L / self.nl) * 2       # partial + combine per call
-        path = 1 + 1 + n_attend + 1 + 2                     # begin, append (+sketch), attend,
-        harness = 1 + 1                                     # detect, keep + compact; select,
-        return path, harness                                # advance
+        calls = math.ceil(self.w.L / self.nl)
+        if self.policy == "h2o":   # begin, append, attend (partial, combine, accumulate), evict x2
+            path = 1 + 1 + 3 * calls + 2
+        else:                      # begin, append (+sketch), attend (partial, combine), detect,
+            path = 1 + 1 + 2 * calls + 1 + 2        # keep + compact
+        harness = 1 + 1                             # select, advance
+        return path, harness
 
     def replay_log(self, K, fresh=False):
         """replay the timed trajectory untimed, recording per-step lengths and kept lists
@@ -260,6 +279,9 @@ class GpuBench:
                 self.reset()
             lens.append(self.cache.len.clone())
             self.step(0 if fresh else t)
+            if self.policy == "h2o":
+                kept.append((None, None))
+                continue
             kc = self.guard.kept_count.clone()
             kept.append((kc, self.guard.kept_idx.clone() if int((kc >= 0).sum()) else None))
         torch.cuda.synchronize()
@@ -333,7 +355,7 @@ def run_gpu(args, ws, rank, local):
         torch.cuda.nvtx.range_pop()
         return None
     fresh = args.fresh_each_step
-    bench = GpuBench(w, dev, 1 if fresh else max(K, W, 1), args.layers_per_call)
+    bench = GpuBench(w, dev, 1 if fresh else max(K, W, 1), args.layers_per_call, args.policy)
 
     # warm-up on the trajectory's first W steps, then a fresh cache for the timed run
     bench.reset()
@@ -383,6 +405,8 @@ def run_gpu(args, ws, rank, local):
         n_rows = lens[t].cpu().numpy() + 1
         a_bytes.append(attend_bytes(w, n_rows))
         kc, ki = kept[t]
+        if kc is None:
+            continue
         kc = kc.cpu().numpy()
         if ki is not None:
             c_bytes.append(compact_bytes(w, kc, ki.cpu().numpy()))
@@ -392,7 +416,7 @@ def run_gpu(args, ws, rank, local):
     compact_gbs = (sum(c_bytes) / (sum(c_ms) * 1e-3) / 1e9) if c_ms else None
 
     e2e = None
-    if not args.no_e2e and not fresh:
+    if not args.no_e2e and not fresh and args.policy == "loopguard":
         e2e = run_e2e(bench, K, ws)
 
     value = sum_over_ranks(K, ws) / (ms * 1e-3)
@@ -409,7 +433,8 @@ def run_gpu(args, ws, rank, local):
         "warmup": W, "ms_per_step": round(ms / K, 4), "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": w.dtype, "data": "synthetic",
         "config": dict(w.describe(), l2="inputs larger than L2 (K/V cache %.1f GB per GPU)"
-                       % (w.kv_bytes() / 1e9), timed_steps="each from a fresh cache" if fresh
+                       % (w.kv_bytes() / 1e9), policy=args.policy,
+                       timed_steps="each from a fresh cache" if fresh
                        else "consecutive decode steps from a fresh cache",
                        layers_per_attend_call=bench.nl, parallelism="dp%d (independent batches, "
                        "no collective)" % ws, tokens_per_step=w.batch * ws),
@@ -431,6 +456,7 @@ def run_gpu(args, ws, rank, local):
                               "ms_per_event": round(sum(c_ms) / len(c_ms), 4) if c_ms else None,
                               "moved_bytes_per_event": int(sum(c_bytes) / len(c_bytes))
                               if c_bytes else 0},
+            "cache_update_ms_per_step": round(sum(prune_ms) / K, 4),
             "other_ms_per_step": round((ms_local - sum(attend_ms) - sum(prune_ms)) / K, 4)},
         "gpu_launches": (path_l + harness_l) * K,
         "gpu_launches_detail": {"path_per_step": path_l, "harness_per_step": harness_l},

@@ -53,7 +53,7 @@ int attend_chunk_rows(const lg_cache *c, int n_layers, int max_len) {
 
 struct AttendLayout {
   int chunk_rows, max_chunks;
-  size_t partial_bytes, final_bytes, logits_bytes, total;
+  size_t partial_bytes, final_bytes, logits_bytes, counter_bytes, total;
 };
 
 size_t round256(size_t x) { return (x + 255) / 256 * 256; }
@@ -69,7 +69,8 @@ AttendLayout attend_layout(const lg_cache *c, int H_q, int n_layers, int max_len
   L.logits_bytes =
       h2o ? round256((size_t)n_layers * c->H_kv * c->S_total * (H_q / c->H_kv) * sizeof(float))
           : 0;
-  L.total = L.partial_bytes + L.final_bytes + L.logits_bytes;
+  L.counter_bytes = 256;
+  L.total = L.partial_bytes + L.final_bytes + L.logits_bytes + L.counter_bytes;
   return L;
 }
 
@@ -185,6 +186,7 @@ lg_status lg_decode_attend(const lg_cache *c, int layer0, int n_layers, const vo
   a.partial = (float *)ws;
   float *final_ml = accumulate_h2o ? (float *)((char *)ws + L.partial_bytes) : nullptr;
   a.logits = accumulate_h2o ? (float *)((char *)ws + L.partial_bytes + L.final_bytes) : nullptr;
+  a.counter = (int *)((char *)ws + L.partial_bytes + L.final_bytes + L.logits_bytes);
   a.S_total = c->S_total;
   a.layer0 = layer0;
   a.n_layers = n_layers;

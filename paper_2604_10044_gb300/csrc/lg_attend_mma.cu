@@ -1,8 +1,8 @@
 // Decode attention over a bf16 KV cache fused with the guard's per-head statistics (LoopGuard
 // Sec. 3.1, Eq. 1; statistics read by Sec. 5.2), on tensor cores.
 //
-// Persistent CTAs (one per SM) walk a list of chunks, each CHUNK consecutive rows of one
-// (layer, sequence, kv-head).  A producer warp streams 128-row K and V tiles into a 3-stage
+// Persistent CTAs (one per SM) take chunks from a shared counter, each CHUNK consecutive rows
+// of one (layer, sequence, kv-head).  A producer warp streams 128-row K and V tiles into a 3-stage
 // shared-memory ring with 2-D tensor copies (cp.async.bulk.tensor, 128-byte swizzle, one box
 // per 64 columns) completing on mbarriers.  Each of four consumer warps owns 32 rows of a tile
 // and all g query heads of the kv-head (padded to 8):
@@ -113,11 +113,13 @@ __device__ __forceinline__ ChunkId decode_chunk(const AttendArgs &a, int c) {
 template <int D, int G>
 __global__ void __launch_bounds__(kThreads, 1)
 attend_mma_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
-                  AttendArgs a, int total_chunks) {
+                  AttendArgs a, int total_chunks, int *next_chunk) {
   using C = MmaCfg<D>;
   extern __shared__ unsigned char smem_raw[];
   __shared__ __align__(8) uint64_t full_bar[C::kStages];
   __shared__ __align__(8) uint64_t empty_bar[C::kStages];
+  __shared__ int stage_chunk[C::kStages];  // chunk of the tile in each stage, -1: no more work
+  __shared__ int stage_tile[C::kStages];   // tile index within that chunk
   unsigned char *smem = reinterpret_cast<unsigned char *>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   float *merge_o = reinterpret_cast<float *>(smem + C::kRingBytes);  // [warps][8][D]
@@ -136,26 +138,40 @@ attend_mma_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant
 
   if (warp == kConsumerWarps) {
     // ------------------------------------------------------------ producer
+    // Chunks are taken from a shared counter (ragged lengths balance across CTAs); each
+    // stage carries its chunk and tile index to the consumers.
     if (lane == 0) {
       asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmK)) : "memory");
       asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmV)) : "memory");
       uint32_t it = 0;
-      for (int c = blockIdx.x; c < total_chunks; c += gridDim.x) {
-        const ChunkId id = decode_chunk(a, c);
-        const int n = a.len[id.b];
-        const int row0 = id.ch * a.chunk_rows;
-        if (n > a.max_len || row0 >= n) continue;
-        const int rows = min(a.chunk_rows, n - row0);
-        const int ntiles = (rows + kTile - 1) / kTile;
-        const int grow =
-            (int)(((int64_t)(a.layer0 + id.lloc) * a.H_kv + id.kvh) * a.S_total + a.seq_off[id.b] +
-                  row0);
-        for (int t = 0; t < ntiles; ++t, ++it) {
+      bool alive = true;
+      while (alive) {
+        const int c = atomicAdd(next_chunk, 1);
+        int ntiles = 0, grow = 0;
+        if (c < total_chunks) {
+          const ChunkId id = decode_chunk(a, c);
+          const int n = a.len[id.b];
+          const int row0 = id.ch * a.chunk_rows;
+          if (n > a.max_len) set_status(a.status, LG_ERR_CAPACITY);
+          if (n > a.max_len || row0 >= n) continue;
+          ntiles = (min(a.chunk_rows, n - row0) + kTile - 1) / kTile;
+          grow = (int)(((int64_t)(a.layer0 + id.lloc) * a.H_kv + id.kvh) * a.S_total +
+                       a.seq_off[id.b] + row0);
+        } else {
+          alive = false;
+        }
+        for (int t = 0; t < (alive ? ntiles : 1); ++t, ++it) {
           const int st = it % C::kStages;
           if (it >= (uint32_t)C::kStages &&
               !mbar_wait(&empty_bar[st], ((it / C::kStages) - 1) & 1)) {
             set_status(a.status, LG_ERR_TIMEOUT);
             return;
+          }
+          stage_chunk[st] = alive ? c : -1;
+          stage_tile[st] = t;
+          if (!alive) {
+            mbar_arrive(&full_bar[st]);  // end of work: completes the phase without a copy
+            break;
           }
           unsigned char *stage = smem + (size_t)st * C::kStageBytes;
           mbar_arrive_expect_tx(&full_bar[st], C::kStageBytes);
@@ -174,24 +190,32 @@ attend_mma_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant
   // -------------------------------------------------------------- consumers
   const int g = lane >> 2, t4 = lane & 3;
   const int mrow = lane & 7, msel = lane >> 3;  // ldmatrix: row within 8x8, matrix index
-  uint32_t it = 0;
-  bool ok = true;
-  for (int c = blockIdx.x; c < total_chunks && ok; c += gridDim.x) {
-    const ChunkId id = decode_chunk(a, c);
-    const int n = a.len[id.b];
-    const int row0 = id.ch * a.chunk_rows;
-    if (n > a.max_len) {
-      if (lane == 0 && warp == 0) set_status(a.status, LG_ERR_CAPACITY);
-      continue;
+  ChunkId id;
+  int n = 0, row0 = 0, rows = 0, ntiles = 0, suffix_lo = 0;
+  int64_t lrow0 = 0;
+  uint32_t qf[C::kKSteps][2];
+  float o[C::kKSteps][4];
+  float m2[2], l2[2], u2[2], sg2[2];
+  float *logits = a.logits;
+  for (uint32_t it = 0;; ++it) {
+    const int st = it % C::kStages;
+    if (!mbar_wait(&full_bar[st], (it / C::kStages) & 1)) {
+      set_status(a.status, LG_ERR_TIMEOUT);
+      return;
     }
-    if (row0 >= n) continue;
-    const int rows = min(a.chunk_rows, n - row0);
-    const int ntiles = (rows + kTile - 1) / kTile;
-    const int suffix_lo = n - min(a.suffix_w, n);
-
-    // B fragments of q^T: head g (zero for padded heads), d = 16 ks + 2 t4 (+1, +8, +9)
-    uint32_t qf[C::kKSteps][2];
-    {
+    const int c = stage_chunk[st];
+    if (c < 0) break;
+    const int t = stage_tile[st];
+    if (t == 0) {
+      // first tile of a chunk: its geometry, the q^T fragments, fresh softmax state
+      id = decode_chunk(a, c);
+      n = a.len[id.b];
+      row0 = id.ch * a.chunk_rows;
+      rows = min(a.chunk_rows, n - row0);
+      ntiles = (rows + kTile - 1) / kTile;
+      suffix_lo = n - min(a.suffix_w, n);
+      lrow0 = ((int64_t)id.lloc * a.H_kv + id.kvh) * a.S_total + a.seq_off[id.b] + row0;
+      // B fragments of q^T: head g (zero for padded heads), d = 16 ks + 2 t4 (+1, +8, +9)
       const int64_t qh = ((int64_t)id.lloc * a.batch + id.b) * a.H_q + (int64_t)id.kvh * G + g;
       const uint32_t *qp = reinterpret_cast<const uint32_t *>(
           reinterpret_cast<const __nv_bfloat16 *>(a.q) + qh * D);
@@ -200,147 +224,137 @@ attend_mma_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant
         qf[ks][0] = g < G ? qp[ks * 8 + t4] : 0u;
         qf[ks][1] = g < G ? qp[ks * 8 + 4 + t4] : 0u;
       }
-    }
-    float o[C::kKSteps][4];
 #pragma unroll
-    for (int eb = 0; eb < C::kKSteps; ++eb) o[eb][0] = o[eb][1] = o[eb][2] = o[eb][3] = 0.f;
-    float m2[2] = {-INFINITY, -INFINITY}, l2[2] = {0.f, 0.f}, u2[2] = {0.f, 0.f},
-          sg2[2] = {0.f, 0.f};
-    float *logits = a.logits;
-    const int64_t lrow0 =
-        ((int64_t)id.lloc * a.H_kv + id.kvh) * a.S_total + a.seq_off[id.b] + row0;
-
-    for (int t = 0; t < ntiles; ++t, ++it) {
-      const int st = it % C::kStages;
-      if (!mbar_wait(&full_bar[st], (it / C::kStages) & 1)) {
-        set_status(a.status, LG_ERR_TIMEOUT);
-        ok = false;
-        break;
-      }
-      unsigned char *stage = smem + (size_t)st * C::kStageBytes;
-      const uint32_t kbase = smem_addr(stage);
-      const uint32_t vbase = kbase + C::kHalves * kBoxBytes;
-      const int tile_rows = min(kTile, rows - t * kTile);
-      const int r_w = warp * 32;  // this warp's first row in the tile
-      if (tile_rows < r_w + 32) {
-        // ragged tail: zero the V rows past the end so that 0 * stale stays 0
-        for (int idx = lane; idx < 32 * C::kHalves * 8; idx += 32) {
-          const int rr = r_w + idx / (C::kHalves * 8);
-          const int hc = idx % (C::kHalves * 8);
-          if (rr >= tile_rows)
-            *reinterpret_cast<uint4 *>(stage + (C::kHalves + hc / 8) * kBoxBytes + rr * 128 +
-                                       (hc % 8) * 16) = make_uint4(0u, 0u, 0u, 0u);
-        }
-        __syncwarp();
-      }
-
-      // S^T for the warp's two 16-row blocks
-      float s[2][4];
-#pragma unroll
-      for (int mb = 0; mb < 2; ++mb) {
-        s[mb][0] = s[mb][1] = s[mb][2] = s[mb][3] = 0.f;
-        const int r = r_w + mb * 16 + (msel & 1) * 8 + mrow;
-#pragma unroll
-        for (int ks = 0; ks < C::kKSteps; ++ks) {
-          const int c8 = (ks & 3) * 2 + (msel >> 1);
-          uint32_t a0, a1, a2, a3;
-          ldsm_x4(kbase + (ks >> 2) * kBoxBytes + swz(r, c8), a0, a1, a2, a3);
-          mma_bf16(s[mb], a0, a1, a2, a3, qf[ks][0], qf[ks][1]);
-        }
-      }
-      // scale to log2 units, mask rows past the end; tile max per head (heads 2 t4, 2 t4 + 1)
-      float mx[2] = {-INFINITY, -INFINITY};
-#pragma unroll
-      for (int mb = 0; mb < 2; ++mb)
-#pragma unroll
-        for (int j = 0; j < 4; ++j) {
-          const int rl = r_w + mb * 16 + g + (j >> 1) * 8;  // row within the tile
-          const bool valid = rl < tile_rows;
-          s[mb][j] = valid ? s[mb][j] * a.qscale : -INFINITY;
-          mx[j & 1] = fmaxf(mx[j & 1], s[mb][j]);
-        }
+      for (int eb = 0; eb < C::kKSteps; ++eb) o[eb][0] = o[eb][1] = o[eb][2] = o[eb][3] = 0.f;
 #pragma unroll
       for (int h = 0; h < 2; ++h) {
-        mx[h] = fmaxf(mx[h], __shfl_xor_sync(0xffffffffu, mx[h], 4));
-        mx[h] = fmaxf(mx[h], __shfl_xor_sync(0xffffffffu, mx[h], 8));
-        mx[h] = fmaxf(mx[h], __shfl_xor_sync(0xffffffffu, mx[h], 16));
+        m2[h] = -INFINITY;
+        l2[h] = u2[h] = sg2[h] = 0.f;
       }
-      const bool raise = mx[0] > m2[0] || mx[1] > m2[1];
-      if (__any_sync(0xffffffffu, raise)) {
-        float corr[2];
-#pragma unroll
-        for (int h = 0; h < 2; ++h) {
-          const float mn = fmaxf(m2[h], mx[h]);
-          corr[h] = mn == m2[h] ? 1.f : exp2f(m2[h] - mn);
-          u2[h] = l2[h] > 0.f ? corr[h] * (u2[h] + (m2[h] - mn) * l2[h]) : 0.f;
-          l2[h] *= corr[h];
-          sg2[h] *= corr[h];
-          m2[h] = mn;
-        }
-#pragma unroll
-        for (int eb = 0; eb < C::kKSteps; ++eb) {
-          o[eb][0] *= corr[0];
-          o[eb][1] *= corr[1];
-          o[eb][2] *= corr[0];
-          o[eb][3] *= corr[1];
-        }
-      }
-      // probabilities, sums, and P^T fragments
-      uint32_t pb[2][2], pl[2][2];
-#pragma unroll
-      for (int mb = 0; mb < 2; ++mb) {
-        float p[4];
-#pragma unroll
-        for (int j = 0; j < 4; ++j) {
-          const int h = j & 1;
-          const int rl = r_w + mb * 16 + g + (j >> 1) * 8;
-          const bool valid = rl < tile_rows;
-          p[j] = valid ? exp2f(s[mb][j] - m2[h]) : 0.f;
-          if (valid) {
-            l2[h] += p[j];
-            u2[h] += p[j] * (s[mb][j] - m2[h]);
-            if (row0 + t * kTile + rl >= suffix_lo) sg2[h] += p[j];
-          }
-        }
-        if (logits) {
-#pragma unroll
-          for (int half = 0; half < 2; ++half) {
-            const int rl = r_w + mb * 16 + g + half * 8;
-            if (rl < tile_rows) {
-              float *dst = logits + (lrow0 + t * kTile + rl) * G;
-              if (2 * t4 < G) dst[2 * t4] = s[mb][half * 2];
-              if (2 * t4 + 1 < G) dst[2 * t4 + 1] = s[mb][half * 2 + 1];
-            }
-          }
-        }
-        // P = hi + lo, both bf16: the P.V product keeps ~16 mantissa bits of P
-        const uint32_t h01 = pack_bf16(p[0], p[1]), h23 = pack_bf16(p[2], p[3]);
-        const float2 f01 = bf16x2_to_float2(h01), f23 = bf16x2_to_float2(h23);
-        pb[mb][0] = movmatrix_trans(h01);  // rows 0-7 of the block
-        pb[mb][1] = movmatrix_trans(h23);  // rows 8-15
-        pl[mb][0] = movmatrix_trans(pack_bf16(p[0] - f01.x, p[1] - f01.y));
-        pl[mb][1] = movmatrix_trans(pack_bf16(p[2] - f23.x, p[3] - f23.y));
-      }
-      // o^T += V^T P^T
-#pragma unroll
-      for (int mb = 0; mb < 2; ++mb) {
-        const int r = r_w + mb * 16 + (msel >> 1) * 8 + mrow;
-#pragma unroll
-        for (int eb = 0; eb < C::kKSteps; ++eb) {
-          const int c8 = (eb & 3) * 2 + (msel & 1);
-          uint32_t a0, a1, a2, a3;
-          ldsm_x4_trans(vbase + (eb >> 2) * kBoxBytes + swz(r, c8), a0, a1, a2, a3);
-          mma_bf16(o[eb], a0, a1, a2, a3, pb[mb][0], pb[mb][1]);
-          mma_bf16(o[eb], a0, a1, a2, a3, pl[mb][0], pl[mb][1]);
-        }
+    }
+    unsigned char *stage = smem + (size_t)st * C::kStageBytes;
+    const uint32_t kbase = smem_addr(stage);
+    const uint32_t vbase = kbase + C::kHalves * kBoxBytes;
+    const int tile_rows = min(kTile, rows - t * kTile);
+    const int r_w = warp * 32;  // this warp's first row in the tile
+    if (tile_rows < r_w + 32) {
+      // ragged tail: zero the V rows past the end so that 0 * stale stays 0
+      for (int idx = lane; idx < 32 * C::kHalves * 8; idx += 32) {
+        const int rr = r_w + idx / (C::kHalves * 8);
+        const int hc = idx % (C::kHalves * 8);
+        if (rr >= tile_rows)
+          *reinterpret_cast<uint4 *>(stage + (C::kHalves + hc / 8) * kBoxBytes + rr * 128 +
+                                     (hc % 8) * 16) = make_uint4(0u, 0u, 0u, 0u);
       }
       __syncwarp();
-      if (tile_rows < r_w + 32) asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-      if (lane == 0) mbar_arrive(&empty_bar[st]);
     }
-    if (!ok) break;
 
-    // ---------------------------------------------------------- merge the four warps
+    // S^T for the warp's two 16-row blocks
+    float s[2][4];
+#pragma unroll
+    for (int mb = 0; mb < 2; ++mb) {
+      s[mb][0] = s[mb][1] = s[mb][2] = s[mb][3] = 0.f;
+      const int r = r_w + mb * 16 + (msel & 1) * 8 + mrow;
+#pragma unroll
+      for (int ks = 0; ks < C::kKSteps; ++ks) {
+        const int c8 = (ks & 3) * 2 + (msel >> 1);
+        uint32_t a0, a1, a2, a3;
+        ldsm_x4(kbase + (ks >> 2) * kBoxBytes + swz(r, c8), a0, a1, a2, a3);
+        mma_bf16(s[mb], a0, a1, a2, a3, qf[ks][0], qf[ks][1]);
+      }
+    }
+    // scale to log2 units, mask rows past the end; tile max per head (heads 2 t4, 2 t4 + 1)
+    float mx[2] = {-INFINITY, -INFINITY};
+#pragma unroll
+    for (int mb = 0; mb < 2; ++mb)
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const int rl = r_w + mb * 16 + g + (j >> 1) * 8;  // row within the tile
+        const bool valid = rl < tile_rows;
+        s[mb][j] = valid ? s[mb][j] * a.qscale : -INFINITY;
+        mx[j & 1] = fmaxf(mx[j & 1], s[mb][j]);
+      }
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      mx[h] = fmaxf(mx[h], __shfl_xor_sync(0xffffffffu, mx[h], 4));
+      mx[h] = fmaxf(mx[h], __shfl_xor_sync(0xffffffffu, mx[h], 8));
+      mx[h] = fmaxf(mx[h], __shfl_xor_sync(0xffffffffu, mx[h], 16));
+    }
+    const bool raise = mx[0] > m2[0] || mx[1] > m2[1];
+    if (__any_sync(0xffffffffu, raise)) {
+      float corr[2];
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        const float mn = fmaxf(m2[h], mx[h]);
+        corr[h] = mn == m2[h] ? 1.f : exp2f(m2[h] - mn);
+        u2[h] = l2[h] > 0.f ? corr[h] * (u2[h] + (m2[h] - mn) * l2[h]) : 0.f;
+        l2[h] *= corr[h];
+        sg2[h] *= corr[h];
+        m2[h] = mn;
+      }
+#pragma unroll
+      for (int eb = 0; eb < C::kKSteps; ++eb) {
+        o[eb][0] *= corr[0];
+        o[eb][1] *= corr[1];
+        o[eb][2] *= corr[0];
+        o[eb][3] *= corr[1];
+      }
+    }
+    // probabilities, sums, and P^T fragments
+    uint32_t pb[2][2], pl[2][2];
+#pragma unroll
+    for (int mb = 0; mb < 2; ++mb) {
+      float p[4];
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const int h = j & 1;
+        const int rl = r_w + mb * 16 + g + (j >> 1) * 8;
+        const bool valid = rl < tile_rows;
+        p[j] = valid ? exp2f(s[mb][j] - m2[h]) : 0.f;
+        if (valid) {
+          l2[h] += p[j];
+          u2[h] += p[j] * (s[mb][j] - m2[h]);
+          if (row0 + t * kTile + rl >= suffix_lo) sg2[h] += p[j];
+        }
+      }
+      if (logits) {
+#pragma unroll
+        for (int half = 0; half < 2; ++half) {
+          const int rl = r_w + mb * 16 + g + half * 8;
+          if (rl < tile_rows) {
+            float *dst = logits + (lrow0 + t * kTile + rl) * G;
+            if (2 * t4 < G) dst[2 * t4] = s[mb][half * 2];
+            if (2 * t4 + 1 < G) dst[2 * t4 + 1] = s[mb][half * 2 + 1];
+          }
+        }
+      }
+      // P = hi + lo, both bf16: the P.V product keeps ~16 mantissa bits of P
+      const uint32_t h01 = pack_bf16(p[0], p[1]), h23 = pack_bf16(p[2], p[3]);
+      const float2 f01 = bf16x2_to_float2(h01), f23 = bf16x2_to_float2(h23);
+      pb[mb][0] = movmatrix_trans(h01);  // rows 0-7 of the block
+      pb[mb][1] = movmatrix_trans(h23);  // rows 8-15
+      pl[mb][0] = movmatrix_trans(pack_bf16(p[0] - f01.x, p[1] - f01.y));
+      pl[mb][1] = movmatrix_trans(pack_bf16(p[2] - f23.x, p[3] - f23.y));
+    }
+    // o^T += V^T P^T
+#pragma unroll
+    for (int mb = 0; mb < 2; ++mb) {
+      const int r = r_w + mb * 16 + (msel >> 1) * 8 + mrow;
+#pragma unroll
+      for (int eb = 0; eb < C::kKSteps; ++eb) {
+        const int c8 = (eb & 3) * 2 + (msel & 1);
+        uint32_t a0, a1, a2, a3;
+        ldsm_x4_trans(vbase + (eb >> 2) * kBoxBytes + swz(r, c8), a0, a1, a2, a3);
+        mma_bf16(o[eb], a0, a1, a2, a3, pb[mb][0], pb[mb][1]);
+        mma_bf16(o[eb], a0, a1, a2, a3, pl[mb][0], pl[mb][1]);
+      }
+    }
+    __syncwarp();
+    if (tile_rows < r_w + 32) asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    if (lane == 0) mbar_arrive(&empty_bar[st]);
+    if (t != ntiles - 1) continue;
+
+    // ---------------------------------------------------------- chunk done: merge the warps
 #pragma unroll
     for (int h = 0; h < 2; ++h) {
 #pragma unroll
@@ -432,27 +446,27 @@ bool make_map(CUtensorMap *m, const void *base, int d, int64_t rows) {
 
 template <int D, int G>
 cudaError_t launch_mma_typed(const CUtensorMap &mk, const CUtensorMap &mv, const AttendArgs &a,
-                             int total, int grid, cudaStream_t s) {
+                             int total, int grid, int *counter, cudaStream_t s) {
   auto kern = attend_mma_kernel<D, G>;
   cudaError_t e =
       cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, MmaCfg<D>::kSmem);
   if (e != cudaSuccess) return e;
-  kern<<<grid, kThreads, MmaCfg<D>::kSmem, s>>>(mk, mv, a, total);
+  kern<<<grid, kThreads, MmaCfg<D>::kSmem, s>>>(mk, mv, a, total, counter);
   return cudaGetLastError();
 }
 
 template <int D>
 cudaError_t launch_mma_d(const CUtensorMap &mk, const CUtensorMap &mv, const AttendArgs &a, int g,
-                         int total, int grid, cudaStream_t s) {
+                         int total, int grid, int *counter, cudaStream_t s) {
   switch (g) {
-    case 1: return launch_mma_typed<D, 1>(mk, mv, a, total, grid, s);
-    case 2: return launch_mma_typed<D, 2>(mk, mv, a, total, grid, s);
-    case 3: return launch_mma_typed<D, 3>(mk, mv, a, total, grid, s);
-    case 4: return launch_mma_typed<D, 4>(mk, mv, a, total, grid, s);
-    case 5: return launch_mma_typed<D, 5>(mk, mv, a, total, grid, s);
-    case 6: return launch_mma_typed<D, 6>(mk, mv, a, total, grid, s);
-    case 7: return launch_mma_typed<D, 7>(mk, mv, a, total, grid, s);
-    case 8: return launch_mma_typed<D, 8>(mk, mv, a, total, grid, s);
+    case 1: return launch_mma_typed<D, 1>(mk, mv, a, total, grid, counter, s);
+    case 2: return launch_mma_typed<D, 2>(mk, mv, a, total, grid, counter, s);
+    case 3: return launch_mma_typed<D, 3>(mk, mv, a, total, grid, counter, s);
+    case 4: return launch_mma_typed<D, 4>(mk, mv, a, total, grid, counter, s);
+    case 5: return launch_mma_typed<D, 5>(mk, mv, a, total, grid, counter, s);
+    case 6: return launch_mma_typed<D, 6>(mk, mv, a, total, grid, counter, s);
+    case 7: return launch_mma_typed<D, 7>(mk, mv, a, total, grid, counter, s);
+    case 8: return launch_mma_typed<D, 8>(mk, mv, a, total, grid, counter, s);
   }
   return cudaErrorInvalidValue;
 }
@@ -472,8 +486,10 @@ cudaError_t launch_attend_mma_partial(const AttendArgs &a, int d, int g, int64_t
   if (e != cudaSuccess) return e;
   const int total = a.n_layers * a.batch * a.H_kv * a.max_chunks;
   const int grid = total < sms ? total : sms;
-  if (d == 128) return launch_mma_d<128>(mk, mv, a, g, total, grid, s);
-  if (d == 64) return launch_mma_d<64>(mk, mv, a, g, total, grid, s);
+  if (!a.counter) return cudaErrorInvalidValue;
+  if ((e = cudaMemsetAsync(a.counter, 0, sizeof(int), s)) != cudaSuccess) return e;
+  if (d == 128) return launch_mma_d<128>(mk, mv, a, g, total, grid, a.counter, s);
+  if (d == 64) return launch_mma_d<64>(mk, mv, a, g, total, grid, a.counter, s);
   return cudaErrorInvalidValue;
 }
 

@@ -15,6 +15,7 @@ struct AttendArgs {
   int32_t *status;
   float *partial;          // [n_layers][batch][H_q][max_chunks][d + 8]
   float *logits;           // nullable [n_layers][H_kv][S_total][g], log2 units
+  int *counter;            // work counter of the persistent tensor-core pass (bf16)
   int64_t S_total;
   int layer0, n_layers, batch, H_kv, H_q;
   int chunk_rows;          // rows per CTA, a multiple of the tile
