@@ -288,13 +288,16 @@ class GpuBench:
         return lens, kept
 
 
-def attend_bytes(w, n_rows):
+def attend_bytes(w, n_rows, h2o=False):
     """algorithmic bytes of attend+stats for one step: K and V rows once per kv-head and
-    layer, queries, outputs and statistics"""
+    layer, queries, outputs and statistics; on the H2O path also the logits written and read
+    back (4 g bytes each) and the score read-modify-write (8 bytes) per (layer, kv-head, row)"""
     esz = 2 if w.dtype == "bf16" else 4
-    kv = 2 * w.L * w.H_kv * w.d * esz * int(np.sum(n_rows))
+    rows = w.L * w.H_kv * int(np.sum(n_rows))
+    kv = 2 * w.d * esz * rows
     qo = 2 * w.L * w.batch * w.H_q * w.d * esz + w.L * w.batch * w.H_q * 16
-    return kv + qo
+    extra = (8 * w.g + 8) * rows if h2o else 0
+    return kv + qo + extra
 
 
 def compact_bytes(w, kept_count, kept_idx):
@@ -403,7 +406,7 @@ def run_gpu(args, ws, rank, local):
     triggers = 0
     for t in range(K):
         n_rows = lens[t].cpu().numpy() + 1
-        a_bytes.append(attend_bytes(w, n_rows))
+        a_bytes.append(attend_bytes(w, n_rows, args.policy == "h2o"))
         kc, ki = kept[t]
         if kc is None:
             continue

@@ -534,8 +534,10 @@ __global__ void __launch_bounds__(kCompactThreads) compact_kernel(lg_cache c,
     const int j0 = lo;
     const int cpr = row_bytes / 16;
     const int rows_per_tile = kCompactThreads * kCompactChunks / cpr;
-    for (int t0 = j0; t0 < cnt; t0 += rows_per_tile) {
-      uint4 v[kCompactChunks];
+    // double-buffered: the next tile's loads are issued before the barrier that releases this
+    // tile's stores (the next tile reads only rows above every slot this tile writes)
+    uint4 cur[kCompactChunks], nxt[kCompactChunks];
+    auto load_tile = [&](uint4 *v, int t0) {
 #pragma unroll
       for (int k = 0; k < kCompactChunks; ++k) {
         const int ci = k * kCompactThreads + tid;
@@ -544,15 +546,23 @@ __global__ void __launch_bounds__(kCompactThreads) compact_kernel(lg_cache c,
           v[k] = *reinterpret_cast<const uint4 *>(base + (int64_t)kept[j] * row_bytes +
                                                   (ci % cpr) * 16);
       }
+    };
+    if (j0 < cnt) load_tile(cur, j0);
+    for (int t0 = j0; t0 < cnt; t0 += rows_per_tile) {
+      const int t1 = t0 + rows_per_tile;
+      if (t1 < cnt) load_tile(nxt, t1);
       __syncthreads();
 #pragma unroll
       for (int k = 0; k < kCompactChunks; ++k) {
         const int ci = k * kCompactThreads + tid;
         const int j = t0 + ci / cpr;
         if (j < cnt)
-          *reinterpret_cast<uint4 *>(base + (int64_t)j * row_bytes + (ci % cpr) * 16) = v[k];
+          *reinterpret_cast<uint4 *>(base + (int64_t)j * row_bytes + (ci % cpr) * 16) = cur[k];
       }
+#pragma unroll
+      for (int k = 0; k < kCompactChunks; ++k) cur[k] = nxt[k];
     }
+    __syncthreads();  // the next item reuses no memory, but keep the CTA in step
   }
 }
 
