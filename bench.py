@@ -50,9 +50,10 @@ def parse():
     ap.add_argument("--no-clocks", action="store_true")
     ap.add_argument("--batch", type=int, default=0,
                     help="override the workload's batch (smaller cases for profiling)")
-    ap.add_argument("--policy", default="loopguard", choices=["loopguard", "h2o"],
-                    help="cache policy of the timed steps: LoopGuard, or the H2O comparator "
-                         "(accumulated-score eviction) on the same inputs")
+    ap.add_argument("--policy", default="loopguard", choices=["loopguard", "h2o", "streaming"],
+                    help="cache policy of the timed steps: LoopGuard, or a comparator on the "
+                         "same inputs: H2O (accumulated-score eviction) or StreamingLLM "
+                         "(attention sinks + sliding window)")
     ap.add_argument("--fresh-each-step", action="store_true",
                     help="time every step from a freshly generated cache (the first decode "
                          "step: attention over the full prefill and the budget prune)")
@@ -214,7 +215,7 @@ class GpuBench:
         self.cache.len.copy_(self.n0_d)
         synth.dev_fill_cache(w, self.cache.k, self.cache.v, self.seqs_d.copy_(
             synth.seqs_tensor(w.seqs, self.dev)), self.off_d, self.n0_d, int(w.n0.max()), self.s)
-        if self.policy == "h2o":
+        if self.policy in ("h2o", "streaming"):
             lg.lg_h2o_reset(self.cache, int(w.n0.max()))
         else:
             lg.lg_sketch_build(self.cache, self.p, int(w.n0.max()))
@@ -232,7 +233,8 @@ class GpuBench:
         """one guarded decode step; ev = (a0, a1, p0, p1) events around attend and prune"""
         lg, c, g, p, w = self.lg, self.cache, self.guard, self.p, self.w
         h2o = self.policy == "h2o"
-        pos_t = self.pos32[t] if h2o else None
+        guard_path = self.policy == "loopguard"
+        pos_t = None if guard_path else self.pos32[t]
         self.select_inputs(t)
         lg.lg_begin_step(c, self.s)
         lg.lg_append(c, 0, w.L, self.kn, self.vn, pos_t, p, self.s)
@@ -244,25 +246,29 @@ class GpuBench:
                                 1 if h2o else 0, g.max_len, g.ws, self.s)
         if ev:
             ev[1].record(self.stream)
-        if not h2o:
+        if guard_path:
             lg.lg_detect(c, g.stats, w.H_q, g.state, self.budget_d, p, g.flags, g.spans, None,
                          g.dstate, self.s)
         if ev:
             ev[2].record(self.stream)
         if h2o:
             lg.lg_h2o_evict(c, self.budget_d, pos_t, g.max_len, self.s)
-        else:
+        elif guard_path:
             lg.lg_prune_compact(c, g.flags, g.spans, g.state, self.budget_d, p, g.kept_idx,
                                 g.kept_count, g.max_keep, g.max_len, self.s)
+        else:
+            lg.lg_streaming_evict(c, self.budget_d, pos_t, lg.N_SINK, g.max_len, self.s)
         if ev:
             ev[3].record(self.stream)
-        synth.dev_advance(w, self.seqs_d, None if h2o else g.flags, self.pos_d, self.s)
+        synth.dev_advance(w, self.seqs_d, g.flags if guard_path else None, self.pos_d, self.s)
 
     # launches of this repository's kernels per step (harness + path)
     def launches_per_step(self):
         calls = math.ceil(self.w.L / self.nl)
         if self.policy == "h2o":   # begin, append, attend (partial, combine, accumulate), evict x2
             path = 1 + 1 + 3 * calls + 2
+        elif self.policy == "streaming":   # begin, append, attend (partial, combine), evict x2
+            path = 1 + 1 + 2 * calls + 2
         else:                      # begin, append (+sketch), attend (partial, combine), detect,
             path = 1 + 1 + 2 * calls + 1 + 2        # keep + compact
         harness = 1 + 1                             # select, advance
@@ -279,7 +285,7 @@ class GpuBench:
                 self.reset()
             lens.append(self.cache.len.clone())
             self.step(0 if fresh else t)
-            if self.policy == "h2o":
+            if self.policy != "loopguard":
                 kept.append((None, None))
                 continue
             kc = self.guard.kept_count.clone()

@@ -250,6 +250,15 @@ LG_API lg_status lg_decode_attend_noalloc(const lg_cache *c, int layer0, int n_l
                                           float *stats, int suffix_w, int accumulate_h2o,
                                           int max_len, cudaStream_t s);
 
+/* StreamingLLM comparator eviction (attention sinks + sliding window, Sec. 2.2, Sec. 6.1) for
+   every sequence with len[b] > budget[b], per (layer, kv-head): positions < n_sink and the
+   budget[b] - n_sink newest positions stay.  len[b] = budget[b] + 1: the oldest non-sink slot
+   is refilled from slot len-1; otherwise the kept rows move to slots 0..budget-1 in order.
+   Uses c->pos (positions are written by lg_append; lg_h2o_reset initialises them). */
+LG_API lg_status lg_streaming_evict(const lg_cache *c, const int32_t *budget,
+                                    const int32_t *pos_now, int n_sink, int max_len,
+                                    cudaStream_t s);
+
 /* Copies *dev_status to *host_code after synchronising the stream. */
 LG_API lg_status lg_read_device_status(const lg_cache *c, int32_t *host_code, cudaStream_t s);
 

@@ -92,6 +92,8 @@ def lib():
         L.lgref_compact_rows.restype = None
         L.lgref_h2o_select.argtypes = [i32, vp, vp, i32, ctypes.c_int32, vp]
         L.lgref_h2o_argmin.argtypes = [i32, vp, vp, i32, ctypes.c_int32]
+        L.lgref_streaming_select.argtypes = [i32, vp, i32, i32, ctypes.c_int32, vp]
+        L.lgref_streaming_oldest.argtypes = [i32, vp, i32]
         _lib = L
     return _lib
 
@@ -191,6 +193,22 @@ def h2o_argmin(score, pos, budget, pos_now) -> int:
     return int(lib().lgref_h2o_argmin(score.size, _p(score), _p(pos), int(budget), int(pos_now)))
 
 
+def streaming_select(pos, budget, n_sink, pos_now) -> np.ndarray:
+    pos = np.ascontiguousarray(pos, dtype=np.int32)
+    kept = np.zeros(max(pos.size, 1), dtype=np.int32)
+    c = lib().lgref_streaming_select(pos.size, _p(pos), int(budget), int(n_sink), int(pos_now),
+                                     _p(kept))
+    return kept[:c].copy()
+
+
+def streaming_oldest(pos, n_sink) -> int:
+    pos = np.ascontiguousarray(pos, dtype=np.int32)
+    return int(lib().lgref_streaming_oldest(pos.size, _p(pos), int(n_sink)))
+
+
+N_SINK = 4   # StreamingLLM attention sinks (the paper does not state the count)
+
+
 # ------------------------------------------------------------------ full decode step
 
 class OracleGuard:
@@ -198,8 +216,8 @@ class OracleGuard:
     K, V [L][H_kv][S_total][d]; sketches [S_total][H_kv*d/32] of the guard layer's V rows;
     per-sequence lengths, guard state; H2O scores and positions [L][H_kv][S_total].
 
-    policy: 'loopguard' (detect + I_keep), 'h2o' (accumulated-score eviction) or 'full'
-    (no eviction)."""
+    policy: 'loopguard' (detect + I_keep), 'h2o' (accumulated-score eviction), 'streaming'
+    (attention sinks + sliding window) or 'full' (no eviction)."""
 
     def __init__(self, w, K, V, prm: Params | None = None, policy="loopguard", t_gen0=64,
                  threads=None):
@@ -220,7 +238,7 @@ class OracleGuard:
         self.state = [new_state(t_gen0) for _ in range(w.batch)]
         self.h2o = None
         self.pos = None
-        if policy == "h2o":
+        if policy in ("h2o", "streaming"):
             self.h2o = np.zeros((w.L, w.H_kv, w.S_total))
             self.pos = np.zeros((w.L, w.H_kv, w.S_total), dtype=np.int32)
             for b in range(w.batch):
@@ -331,6 +349,32 @@ class OracleGuard:
             self.len[b] = B
         return events
 
+    def streaming_evict(self, pos_now, budget=None, n_sink=N_SINK):
+        """StreamingLLM comparator after a step: sinks + the most recent positions; one
+        swap-remove per (layer, kv-head) when one row over budget, else an ordered cut"""
+        w = self.w
+        budget = w.budget if budget is None else budget
+        for b in range(w.batch):
+            n, B, o = int(self.len[b]), int(budget[b]), self.off[b]
+            if n <= B:
+                continue
+            for layer in range(w.L):
+                for kvh in range(w.H_kv):
+                    ps = self.pos[layer, kvh, o:o + n]
+                    if n == B + 1:
+                        x = streaming_oldest(ps, n_sink)
+                        if x != n - 1:
+                            for arr in (self.K, self.V):
+                                arr[layer, kvh, o + x] = arr[layer, kvh, o + n - 1]
+                            ps[x] = ps[n - 1]
+                    else:
+                        kept = streaming_select(ps, B, n_sink, pos_now[b])
+                        compact_rows(self.K[layer, kvh, o:o + n], kept)
+                        compact_rows(self.V[layer, kvh, o:o + n], kept)
+                        ps[:len(kept)] = ps[kept].copy()
+            self.len[b] = B
+        return None
+
     def step(self, q, kn, vn, pos_new, budget=None):
         """one decode step: append, attend (Eq. 1), then the policy's cache update"""
         self.append(kn, vn, pos_new)
@@ -342,5 +386,7 @@ class OracleGuard:
                        kept=self.prune(flags, spans, budget))
         elif self.policy == "h2o":
             res.update(events=self.h2o_evict(pos_new, budget))
+        elif self.policy == "streaming":
+            res.update(events=self.streaming_evict(pos_new, budget))
         res["len"] = self.len.copy()
         return res

@@ -15,6 +15,7 @@
  *   retained set I_keep, tail-cleaned recent . Sec. 5.3, Eq. 10, Eq. 11
  *   progressive aggressiveness, gather ....... Sec. 5.3
  *   H2O comparator (cited, not defined) ...... Sec. 2.2, Sec. 6.1
+ *   StreamingLLM comparator (cited) .......... Sec. 2.2, Sec. 6.1
  *
  * The paper's detector reads generated token ids and top-1 probabilities; the
  * decode path carries only K/V caches and attention, so each signal is
@@ -394,6 +395,30 @@ int lgref_h2o_argmin(int n, const double *score, const int32_t *pos, int budget,
     if (pos[i] > pos_now - R) continue;
     if (best < 0 || score[i] < score[best] || (score[i] == score[best] && pos[i] < pos[best]))
       best = i;
+  }
+  return best;
+}
+
+/* ---------------------------------------------------------------- StreamingLLM comparator */
+
+int lgref_streaming_select(int n, const int32_t *pos, int budget, int n_sink, int32_t pos_now,
+                           int32_t *kept) {
+  if (n <= budget) {
+    for (int i = 0; i < n; ++i) kept[i] = i;
+    return n;
+  }
+  int window = budget - n_sink;
+  int count = 0;
+  for (int i = 0; i < n; ++i)
+    if (pos[i] < n_sink || pos[i] > pos_now - window) kept[count++] = i;
+  return count;
+}
+
+int lgref_streaming_oldest(int n, const int32_t *pos, int n_sink) {
+  int best = -1;
+  for (int i = 0; i < n; ++i) {
+    if (pos[i] < n_sink) continue;
+    if (best < 0 || pos[i] < pos[best]) best = i;
   }
   return best;
 }

@@ -106,6 +106,15 @@ int lgref_h2o_select(int n, const double *score, const int32_t *pos, int budget,
    window, older position first on ties), or -1 when nothing is evictable. */
 int lgref_h2o_argmin(int n, const double *score, const int32_t *pos, int budget, int32_t pos_now);
 
+/* StreamingLLM comparator (attention sinks + sliding window, Sec. 2.2, Sec. 6.1): rows kept when a
+   (layer, kv-head) stream of n > budget rows is cut to `budget`: positions < n_sink and the
+   budget - n_sink most recent positions.  kept[] ascending slots; returns the count. */
+int lgref_streaming_select(int n, const int32_t *pos, int budget, int n_sink, int32_t pos_now,
+                           int32_t *kept);
+
+/* StreamingLLM comparator, one row over budget: the slot of the oldest position >= n_sink. */
+int lgref_streaming_oldest(int n, const int32_t *pos, int n_sink);
+
 #ifdef __cplusplus
 }
 #endif

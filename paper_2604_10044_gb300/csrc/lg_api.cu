@@ -252,6 +252,14 @@ lg_status lg_h2o_evict(const lg_cache *c, const int32_t *budget, const int32_t *
   return cuda_status(lg::launch_h2o_evict(*c, budget, pos_now, max_len, s));
 }
 
+lg_status lg_streaming_evict(const lg_cache *c, const int32_t *budget, const int32_t *pos_now,
+                             int n_sink, int max_len, cudaStream_t s) {
+  lg_status st = check_cache(c);
+  if (st != LG_OK) return st;
+  if (!c->pos || !budget || !pos_now || max_len < 0 || n_sink < 0) return LG_ERR_INVALID_ARG;
+  return cuda_status(lg::launch_streaming_evict(*c, budget, pos_now, n_sink, max_len, s));
+}
+
 lg_status lg_read_device_status(const lg_cache *c, int32_t *host_code, cudaStream_t s) {
   if (!c || !c->dev_status || !host_code) return LG_ERR_INVALID_ARG;
   if (cudaMemcpyAsync(host_code, c->dev_status, sizeof(int32_t), cudaMemcpyDeviceToHost, s) !=

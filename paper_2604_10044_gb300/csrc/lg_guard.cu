@@ -589,9 +589,14 @@ constexpr int kH2OTile = 32;
 constexpr int kH2OMaxQ = 2 * kH2OTile * 32 / kH2OThreads;  // 16-byte chunks per thread, 512 B rows
 
 // One CTA per (sequence, layer, kv-head) stream of a sequence over budget.
-__global__ void __launch_bounds__(kH2OThreads) h2o_evict_kernel(lg_cache c, const int32_t *budget,
-                                                                const int32_t *pos_now,
-                                                                int max_len) {
+// kMode kEvictH2O: keep the recent half of the budget and the highest (score, pos) rows.
+// kMode kEvictStreaming: keep positions < n_sink and the budget - n_sink most recent ones.
+enum { kEvictH2O = 0, kEvictStreaming = 1 };
+
+template <int kMode>
+__global__ void __launch_bounds__(kH2OThreads) evict_kernel(lg_cache c, const int32_t *budget,
+                                                            const int32_t *pos_now, int max_len,
+                                                            int n_sink) {
   __shared__ unsigned long long s_min;
   __shared__ int s_slot, s_count, s_out;
   __shared__ unsigned int hist[256];
@@ -605,7 +610,8 @@ __global__ void __launch_bounds__(kH2OThreads) h2o_evict_kernel(lg_cache c, cons
     if (tid == 0) set_status(c.dev_status, LG_ERR_CAPACITY);
     return;
   }
-  const int32_t thrp = pos_now[b] - B / 2;  // recent: pos > thrp
+  // recent: pos > thrp (H2O: the newest B/2 positions; streaming: the newest B - n_sink)
+  const int32_t thrp = pos_now[b] - (kMode == kEvictH2O ? B / 2 : B - n_sink);
   const int64_t o = (int64_t)lh * c.S_total + c.seq_off[b];
   float *sc = c.h2o + o;
   int32_t *ps = c.pos + o;
@@ -614,12 +620,20 @@ __global__ void __launch_bounds__(kH2OThreads) h2o_evict_kernel(lg_cache c, cons
   uint4 *K4 = reinterpret_cast<uint4 *>((unsigned char *)c.k + o * rb);
   uint4 *V4 = reinterpret_cast<uint4 *>((unsigned char *)c.v + o * rb);
 
+  // eviction order among the rows outside the protected set: lowest key first
+  auto evict_key = [&](int i) -> unsigned long long {
+    return kMode == kEvictH2O ? (unsigned long long)h2o_key(sc[i], ps[i])
+                              : (unsigned long long)(uint32_t)ps[i];
+  };
+  auto protected_row = [&](int i) -> bool {
+    return ps[i] > thrp || (kMode == kEvictStreaming && ps[i] < n_sink);
+  };
   if (n == B + 1) {
-    // one row over budget: evict the lowest (score, pos) outside the recent window and refill
-    // its slot from the last slot
+    // one row over budget: evict the lowest key outside the protected rows and refill its
+    // slot from the last slot
     unsigned long long best = ~0ull;
     for (int i = tid; i < n; i += kH2OThreads)
-      if (ps[i] <= thrp) best = min(best, (unsigned long long)h2o_key(sc[i], ps[i]));
+      if (!protected_row(i)) best = min(best, evict_key(i));
     if (tid == 0) {
       s_min = ~0ull;
       s_slot = -1;
@@ -628,7 +642,7 @@ __global__ void __launch_bounds__(kH2OThreads) h2o_evict_kernel(lg_cache c, cons
     atomicMin(&s_min, best);
     __syncthreads();
     for (int i = tid; i < n; i += kH2OThreads)
-      if (ps[i] <= thrp && h2o_key(sc[i], ps[i]) == s_min) s_slot = i;
+      if (!protected_row(i) && evict_key(i) == s_min) s_slot = i;
     __syncthreads();
     const int x = s_slot;
     if (x < 0 || x == n - 1) return;
@@ -642,8 +656,16 @@ __global__ void __launch_bounds__(kH2OThreads) h2o_evict_kernel(lg_cache c, cons
     }
     return;
   }
+  if (kMode == kEvictStreaming) {
+    // closed form: sinks and the newest B - n_sink positions
+    if (tid == 0) s_out = 0;
+    __syncthreads();
+  }
 
   // cut to B rows: recent rows plus the k = B - n_recent highest keys among the others
+  int k = 0;
+  unsigned long long kth = 0;
+  if (kMode == kEvictH2O) {
   if (tid == 0) s_count = 0;
   __syncthreads();
   int cnt_local = 0;
@@ -654,7 +676,7 @@ __global__ void __launch_bounds__(kH2OThreads) h2o_evict_kernel(lg_cache c, cons
     s_out = 0;
   }
   __syncthreads();
-  const int k = B - s_count;
+  k = B - s_count;
   unsigned long long mask = 0;
   if (tid == 0) s_remaining = k;
   for (int digit = 7; digit >= 0; --digit) {
@@ -679,7 +701,8 @@ __global__ void __launch_bounds__(kH2OThreads) h2o_evict_kernel(lg_cache c, cons
     mask |= 255ull << (8 * digit);
     __syncthreads();
   }
-  const unsigned long long kth = s_prefix;  // key of the k-th highest non-recent row
+  kth = s_prefix;  // key of the k-th highest non-recent row
+  }
 
   // ordered compaction of K, V, score and pos over source tiles of kH2OTile rows
   const int lane = tid & 31, warp = tid >> 5;
@@ -689,7 +712,8 @@ __global__ void __launch_bounds__(kH2OThreads) h2o_evict_kernel(lg_cache c, cons
     if (warp == 0) {
       const int i = t0 + lane;
       bool keep = false;
-      if (i < n) keep = ps[i] > thrp || (k > 0 && h2o_key(sc[i], ps[i]) >= kth);
+      if (i < n)
+        keep = protected_row(i) || (kMode == kEvictH2O && k > 0 && h2o_key(sc[i], ps[i]) >= kth);
       const unsigned bal = __ballot_sync(0xffffffffu, keep);
       s_dest[lane] = keep ? s_out + __popc(bal & ((1u << lane) - 1u)) : -1;
       if (lane == 0) s_tile_kept = __popc(bal);
@@ -847,8 +871,23 @@ cudaError_t launch_h2o_reset(const lg_cache &c, int max_len, cudaStream_t s) {
 
 cudaError_t launch_h2o_evict(const lg_cache &c, const int32_t *budget, const int32_t *pos_now,
                              int max_len, cudaStream_t s) {
-  h2o_evict_kernel<<<dim3(c.L * c.H_kv, c.batch), kH2OThreads, 0, s>>>(c, budget, pos_now,
-                                                                       max_len);
+  evict_kernel<kEvictH2O><<<dim3(c.L * c.H_kv, c.batch), kH2OThreads, 0, s>>>(c, budget, pos_now,
+                                                                             max_len, 0);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  h2o_len_kernel<<<(c.batch + 127) / 128, 128, 0, s>>>(c, budget);
+  return cudaGetLastError();
+}
+
+}  // namespace lg
+
+namespace lg {
+
+cudaError_t launch_streaming_evict(const lg_cache &c, const int32_t *budget,
+                                   const int32_t *pos_now, int n_sink, int max_len,
+                                   cudaStream_t s) {
+  evict_kernel<kEvictStreaming><<<dim3(c.L * c.H_kv, c.batch), kH2OThreads, 0, s>>>(
+      c, budget, pos_now, max_len, n_sink);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   h2o_len_kernel<<<(c.batch + 127) / 128, 128, 0, s>>>(c, budget);

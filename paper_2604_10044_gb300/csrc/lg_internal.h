@@ -54,5 +54,8 @@ cudaError_t launch_prune_compact(const lg_cache &c, const int32_t *flags, const 
 cudaError_t launch_h2o_reset(const lg_cache &c, int max_len, cudaStream_t s);
 cudaError_t launch_h2o_evict(const lg_cache &c, const int32_t *budget, const int32_t *pos_now,
                              int max_len, cudaStream_t s);
+cudaError_t launch_streaming_evict(const lg_cache &c, const int32_t *budget,
+                                   const int32_t *pos_now, int n_sink, int max_len,
+                                   cudaStream_t s);
 
 }  // namespace lg

@@ -73,6 +73,7 @@ def lib():
                                  vp],
             "lg_h2o_reset": [P(LgCache), i32, vp],
             "lg_h2o_evict": [P(LgCache), vp, vp, i32, vp],
+            "lg_streaming_evict": [P(LgCache), vp, vp, i32, i32, vp],
             "lg_read_device_status": [P(LgCache), vp, vp],
             "lg_decode_attend_noalloc": [P(LgCache), i32, i32, vp, i32, ctypes.c_float, vp, vp,
                                          i32, i32, i32, vp],
@@ -94,7 +95,7 @@ def exported_symbols():
     return ["lg_default_params", "lg_status_string", "lg_workspace_size", "lg_state_init",
             "lg_begin_step", "lg_append", "lg_sketch_build", "lg_decode_attend", "lg_detect",
             "lg_prune_compact", "lg_h2o_reset", "lg_h2o_evict", "lg_read_device_status",
-            "lg_decode_attend_noalloc", "lg_detect_state_size"]
+            "lg_decode_attend_noalloc", "lg_detect_state_size", "lg_streaming_evict"]
 
 NOALLOC_SCRATCH_BYTES = 32 << 20  # LG_NOALLOC_SCRATCH_BYTES in include/lg.h
 
@@ -199,6 +200,14 @@ def lg_h2o_evict(cache, budget, pos_now, max_len, stream=None):
           _stream(stream))
 
 
+def lg_streaming_evict(cache, budget, pos_now, n_sink, max_len, stream=None):
+    _call("lg_streaming_evict", ctypes.byref(cache.c), _ptr(budget), _ptr(pos_now), n_sink,
+          max_len, _stream(stream))
+
+
+N_SINK = 4  # StreamingLLM attention sinks (count not stated by the paper)
+
+
 def lg_read_device_status(cache, stream=None) -> int:
     code = ctypes.c_int32(0)
     _call("lg_read_device_status", ctypes.byref(cache.c), ctypes.byref(code), _stream(stream))
@@ -249,7 +258,7 @@ class Cache:
         if policy in ("loopguard", "full"):
             self.sketch = torch.zeros((self.S_total, self.nwords), dtype=torch.int32,
                                       device=self.device)
-        if policy == "h2o":
+        if policy in ("h2o", "streaming"):
             self.h2o = torch.zeros((L, H_kv, self.S_total), dtype=torch.float32,
                                    device=self.device)
             self.pos = torch.zeros((L, H_kv, self.S_total), dtype=torch.int32,
@@ -305,7 +314,7 @@ class Guard:
         self.kept_idx = torch.zeros((b, self.max_keep), dtype=torch.int32, device=dev)
         self.kept_count = torch.zeros(b, dtype=torch.int32, device=dev)
         self.diag = torch.zeros((b, 8), dtype=torch.float64, device=dev)
-        ds_words = lg_detect_state_size(cache, self.p) // 4 if policy != "h2o" else 1
+        ds_words = lg_detect_state_size(cache, self.p) // 4 if policy == "loopguard" else 1
         self.dstate = torch.zeros(ds_words, dtype=torch.int32, device=dev)
         tdt = _torch_dtype(cache.dtype)
         self.out = torch.zeros((L, b, H_q, cache.d), dtype=tdt, device=dev)
@@ -334,6 +343,8 @@ class Guard:
                              self.kept_count, self.max_keep, self.max_len, stream)
         elif self.policy == "h2o":
             lg_h2o_evict(c, budget, pos_new, self.max_len, stream)
+        elif self.policy == "streaming":
+            lg_streaming_evict(c, budget, pos_new, N_SINK, self.max_len, stream)
 
     def step_host(self, q, k_new, v_new, budget, pos_new=None):
         """same step from host numpy arrays; returns host copies of every output"""

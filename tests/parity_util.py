@@ -171,3 +171,31 @@ def run_h2o(w, device, steps=None, n_layers_per_call=None):
         assert np.array_equal(cache.lengths(), ref.len)
         pos = pos + 1
     return events
+
+
+def run_streaming(w, device, steps=None):
+    """The StreamingLLM comparator (sinks + sliding window) on the GPU and in the oracle:
+    outputs and statistics within tolerance, rows and positions bit-exact every step."""
+    steps = w.steps if steps is None else steps
+    K, V = synth.host_cache(w)
+    ref = oracle.OracleGuard(w, K.copy(), V.copy(), policy="streaming")
+    cache = lg.Cache.from_host(w, K, V, device, policy="streaming")
+    guard = lg.Guard(cache, w.H_q, policy="streaming")
+    pos = w.n0.astype(np.int64)
+    rt, ra = OUT_TOL[w.dtype]
+    for t in range(steps):
+        q, kn, vn = synth.host_step(w, pos)
+        r_ref = ref.step(q, kn, vn, pos)
+        r = guard.step_host(q, kn, vn, w.budget, pos.astype(np.int32))
+        tag = "streaming step %d" % t
+        assert_close(r["out"], r_ref["out"], rt, ra, tag + " out")
+        assert_close(r["stats"], r_ref["stats"], *STAT_TOL, what=tag + " stats")
+        assert np.array_equal(r["len"], r_ref["len"]), tag
+        Kg, Vg = cache.to_host()
+        ps = cache.pos.cpu().numpy()
+        for b in range(w.batch):
+            o, n = int(w.seq_off[b]), int(r_ref["len"][b])
+            assert np.array_equal(ps[:, :, o:o + n], ref.pos[:, :, o:o + n]), (tag, b)
+            assert np.array_equal(Kg[:, :, o:o + n], ref.K[:, :, o:o + n]), (tag, b)
+            assert np.array_equal(Vg[:, :, o:o + n], ref.V[:, :, o:o + n]), (tag, b)
+        pos = pos + 1

@@ -9,7 +9,7 @@ import pytest
 import torch
 
 import synth
-from parity_util import run_h2o, run_loopguard
+from parity_util import run_h2o, run_loopguard, run_streaming
 
 pytestmark = pytest.mark.gpu
 
@@ -107,3 +107,11 @@ def test_device_generator_matches_host(cuda):
     torch.cuda.synchronize()
     assert np.array_equal(device_to_host(qd), q)
     assert np.array_equal(device_to_host(kd), kn) and np.array_equal(device_to_host(vd), vn)
+
+
+def test_streaming_comparator(cuda):
+    """StreamingLLM path: first cut from n > B + 1 to sinks + window, then one oldest-row
+    eviction per step, ragged lengths"""
+    w = synth.make_workload(4, L=2, batch=4, len_range=(100, 900), budget_max=384, steps=4,
+                            periods=(4, 8), onset_max=2)
+    run_streaming(w, cuda)

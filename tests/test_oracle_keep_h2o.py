@@ -137,3 +137,20 @@ def test_h2o_path_keeps_budget_and_mass():
                     assert set(range(int(pos[b]) - w.budget[b] // 2 + 1, int(pos[b]) + 1)) <= \
                         set(ps.tolist())
         pos = pos + 1
+
+
+@pytest.mark.parametrize("seed", range(6))
+def test_streaming_select_brute_force(seed):
+    """StreamingLLM: the first n_sink positions and the budget - n_sink newest stay"""
+    rng = np.random.default_rng(seed)
+    n = int(rng.integers(12, 60))
+    B = int(rng.integers(6, n))
+    pos = rng.permutation(n).astype(np.int32)
+    pos_now = int(pos.max())
+    kept = oracle.streaming_select(pos, B, 4, pos_now)
+    order = sorted(range(n), key=lambda i: -pos[i])
+    expect = sorted({i for i in range(n) if pos[i] < 4} | set(
+        [i for i in order if pos[i] >= 4][:B - 4]))
+    assert kept.tolist() == expect and len(kept) == B
+    x = oracle.streaming_oldest(pos, 4)
+    assert pos[x] == 4                       # positions 0..n-1 are all present
