@@ -50,13 +50,16 @@ def parse():
     ap.add_argument("--no-clocks", action="store_true")
     ap.add_argument("--batch", type=int, default=0,
                     help="override the workload's batch (smaller cases for profiling)")
-    ap.add_argument("--policy", default="loopguard", choices=["loopguard", "h2o", "streaming"],
+    ap.add_argument("--policy", default="loopguard",
+                    choices=["loopguard", "h2o", "streaming", "full"],
                     help="cache policy of the timed steps: LoopGuard, or a comparator on the "
-                         "same inputs: H2O (accumulated-score eviction) or StreamingLLM "
-                         "(attention sinks + sliding window)")
+                         "same inputs: H2O (accumulated-score eviction), StreamingLLM "
+                         "(attention sinks + sliding window) or the full cache (no eviction)")
     ap.add_argument("--fresh-each-step", action="store_true",
                     help="time every step from a freshly generated cache (the first decode "
                          "step: attention over the full prefill and the budget prune)")
+    ap.add_argument("--eager", action="store_true",
+                    help="time the steps as eager launches instead of one CUDA graph replay")
     ap.add_argument("--profile-steps", type=int, default=0,
                     help="run this many steps untimed and exit (for ncu launch lists)")
     return ap.parse_args()
@@ -215,7 +218,7 @@ class GpuBench:
         self.cache.len.copy_(self.n0_d)
         synth.dev_fill_cache(w, self.cache.k, self.cache.v, self.seqs_d.copy_(
             synth.seqs_tensor(w.seqs, self.dev)), self.off_d, self.n0_d, int(w.n0.max()), self.s)
-        if self.policy in ("h2o", "streaming"):
+        if self.policy in ("h2o", "streaming", "full"):
             lg.lg_h2o_reset(self.cache, int(w.n0.max()))
         else:
             lg.lg_sketch_build(self.cache, self.p, int(w.n0.max()))
@@ -256,7 +259,7 @@ class GpuBench:
         elif guard_path:
             lg.lg_prune_compact(c, g.flags, g.spans, g.state, self.budget_d, p, g.kept_idx,
                                 g.kept_count, g.max_keep, g.max_len, self.s)
-        else:
+        elif self.policy == "streaming":
             lg.lg_streaming_evict(c, self.budget_d, pos_t, lg.N_SINK, g.max_len, self.s)
         if ev:
             ev[3].record(self.stream)
@@ -269,6 +272,8 @@ class GpuBench:
             path = 1 + 1 + 3 * calls + 2
         elif self.policy == "streaming":   # begin, append, attend (partial, combine), evict x2
             path = 1 + 1 + 2 * calls + 2
+        elif self.policy == "full":        # begin, append, attend (partial, combine)
+            path = 1 + 1 + 2 * calls
         else:                      # begin, append (+sketch), attend (partial, combine), detect,
             path = 1 + 1 + 2 * calls + 1 + 2        # keep + compact
         harness = 1 + 1                             # select, advance
@@ -364,6 +369,9 @@ def run_gpu(args, ws, rank, local):
         torch.cuda.nvtx.range_pop()
         return None
     fresh = args.fresh_each_step
+    # every launch of the run goes to one side stream (stream capture needs a non-default one)
+    side = torch.cuda.Stream(device=dev)
+    torch.cuda.set_stream(side)
     bench = GpuBench(w, dev, 1 if fresh else max(K, W, 1), args.layers_per_call, args.policy)
 
     # warm-up on the trajectory's first W steps, then a fresh cache for the timed run
@@ -373,13 +381,50 @@ def run_gpu(args, ws, rank, local):
             bench.reset()
         bench.step(0 if fresh else t)
     torch.cuda.synchronize()
-    bench.reset()
-    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(K)]
     start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    graph = None
+    eager_ms = None
+    if not fresh and not args.eager:
+        # the same K steps timed eagerly first (reported beside the graph figure), then
+        # captured once as a CUDA graph whose single replay is the timed region; events
+        # recorded as graph nodes time each part of every step
+        bench.reset()
+        barrier(ws)
+        torch.cuda.synchronize()
+        start.record(bench.stream)
+        for t in range(K):
+            bench.step(t)
+        stop.record(bench.stream)
+        torch.cuda.synchronize()
+        eager_ms = max_over_ranks(start.elapsed_time(stop), ws)
+        evs = [[torch.cuda.Event(enable_timing=True, external=True) for _ in range(4)]
+               for _ in range(K)]
+        for e in evs:
+            for x in e:
+                x.record(bench.stream)
+        bench.reset()
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph, stream=bench.stream, capture_error_mode="thread_local"):
+            for t in range(K):
+                bench.step(t, evs[t])
+        graph.replay()                        # untimed: uploads the graph
+        torch.cuda.synchronize()
+        if bench.lg.lg_read_device_status(bench.cache) != 0:
+            raise RuntimeError("device status %d after the graph warm-up replay"
+                               % bench.lg.lg_read_device_status(bench.cache))
+    else:
+        evs = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(K)]
+    bench.reset()
     clocks = Clocks(local, enabled=not args.no_clocks)
     barrier(ws)
     torch.cuda.synchronize()
-    if fresh:
+    if graph is not None:
+        start.record(bench.stream)
+        graph.replay()
+        stop.record(bench.stream)
+        torch.cuda.synchronize()
+        ms_local = start.elapsed_time(stop)
+    elif fresh:
         # every step from a freshly generated cache; only the steps are timed
         ms_local = 0.0
         for t in range(K):
@@ -404,6 +449,7 @@ def run_gpu(args, ws, rank, local):
         raise RuntimeError("device status %d after the timed run" % status)
     ms = max_over_ranks(ms_local, ws)
     attend_ms = [e[0].elapsed_time(e[1]) for e in evs]
+    detect_ms = [e[1].elapsed_time(e[2]) for e in evs]
     prune_ms = [e[2].elapsed_time(e[3]) for e in evs]
 
     # algorithmic bytes of the same trajectory (untimed, deterministic replay)
@@ -445,6 +491,8 @@ def run_gpu(args, ws, rank, local):
                        % (w.kv_bytes() / 1e9), policy=args.policy,
                        timed_steps="each from a fresh cache" if fresh
                        else "consecutive decode steps from a fresh cache",
+                       launch="eager" if graph is None else
+                       "one CUDA graph replay of the K steps (captured before timing)",
                        layers_per_attend_call=bench.nl, parallelism="dp%d (independent batches, "
                        "no collective)" % ws, tokens_per_step=w.batch * ws),
         "roofline": {"bound": "hbm", "achieved": round(attend_gbs, 1), "peak": hbm_peak,
@@ -465,8 +513,11 @@ def run_gpu(args, ws, rank, local):
                               "ms_per_event": round(sum(c_ms) / len(c_ms), 4) if c_ms else None,
                               "moved_bytes_per_event": int(sum(c_bytes) / len(c_bytes))
                               if c_bytes else 0},
+            "detect_ms_per_step": round(sum(detect_ms) / K, 4),
             "cache_update_ms_per_step": round(sum(prune_ms) / K, 4),
-            "other_ms_per_step": round((ms_local - sum(attend_ms) - sum(prune_ms)) / K, 4)},
+            "other_ms_per_step": round((ms_local - sum(attend_ms) - sum(detect_ms) -
+                                        sum(prune_ms)) / K, 4)},
+        "eager_ms_per_step": round(eager_ms / K, 4) if eager_ms is not None else None,
         "gpu_launches": (path_l + harness_l) * K,
         "gpu_launches_detail": {"path_per_step": path_l, "harness_per_step": harness_l},
         "clocks": clk,

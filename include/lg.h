@@ -183,8 +183,8 @@ LG_API lg_status lg_decode_attend(const lg_cache *c, int layer0, int n_layers, c
      Trigger = t_gen >= t_min and cd = 0 and Warn and (Stall or TailRep).
    On a trigger with TailRep the span [lo, hi) of I_bad covers every copy of the period
    extended back while rows keep matching, clipped to W^recent = [n - budget/2, n).
-   stats: device [L][batch][H_q][4] (lg_decode_attend's output for all layers);
-   state: device [batch]; budget: device [batch]; flags: device [batch] (1 = trigger);
+   stats: device [L][batch][H_q][4], 16-byte aligned (lg_decode_attend's output for all
+   layers); state: device [batch]; budget: device [batch]; flags: device [batch] (1 = trigger);
    spans: device [batch][2] ([0,0) when empty).
    diag: nullable device [batch][8] fp64, per sequence {mean normalised entropy, mean suffix
    lift, novel fraction, vote 1, vote 2, vote 3, Stall, P* (0 = no tail repetition)}.

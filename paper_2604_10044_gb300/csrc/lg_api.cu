@@ -212,7 +212,7 @@ lg_status lg_detect(const lg_cache *c, const float *stats, int H_q, lg_guard_sta
   if ((st = check_params(p)) != LG_OK) return st;
   if (!c->sketch || !stats || !state || !budget || !flags || !spans || !dstate)
     return LG_ERR_INVALID_ARG;
-  if ((uintptr_t)dstate & 3u) return LG_ERR_INVALID_ARG;
+  if (((uintptr_t)dstate & 3u) || ((uintptr_t)stats & 15u)) return LG_ERR_INVALID_ARG;
   if (H_q < 1 || H_q % c->H_kv) return LG_ERR_INVALID_ARG;
   if (lg::detect_smem_bytes(*p, c->H_kv * c->d / 32) > 200 * 1024) return LG_ERR_UNSUPPORTED;
   return cuda_status(

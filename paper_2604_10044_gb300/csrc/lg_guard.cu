@@ -143,110 +143,202 @@ __device__ __forceinline__ bool rows_match(const uint32_t *x, const uint32_t *y,
   return dist <= thr;
 }
 
+// Full Hamming distance of two sketch rows of nwords words (nwords a multiple of 4, rows
+// 16-byte aligned); the loads are independent, so a thread has all of them in flight at once.
+__device__ __forceinline__ int hamming(const uint32_t *x, const uint32_t *y, int nwords) {
+  const uint4 *a = reinterpret_cast<const uint4 *>(x);
+  const uint4 *b = reinterpret_cast<const uint4 *>(y);
+  int dist = 0;
+#pragma unroll 8
+  for (int w = 0; w < nwords / 4; ++w) {
+    const uint4 u = __ldg(a + w), v = __ldg(b + w);
+    dist += __popc(u.x ^ v.x) + __popc(u.y ^ v.y) + __popc(u.z ^ v.z) + __popc(u.w ^ v.w);
+  }
+  return dist;
+}
+
+// fp32 -> fp64 by moving the bits (IEEE-754 binary32 into binary64: exponent rebiased by
+// 1023 - 127 = 896, mantissa shifted up by 29), exact; normal numbers and zeros stay on the
+// integer pipe, subnormals, infinities and NaNs take the conversion instruction.
+__device__ __forceinline__ double widen(float x) {
+  const uint32_t u = __float_as_uint(x);
+  const uint32_t e = (u >> 23) & 0xffu, m = u & 0x7fffffu, sgn = u & 0x80000000u;
+  if (e - 1u < 254u)
+    return __hiloint2double((int)(sgn | ((e + 896u) << 20) | (m >> 3)), (int)(u << 29));
+  if (e == 0u && m == 0u) return __hiloint2double((int)sgn, 0);
+  return (double)x;
+}
+
+constexpr int kDetectWarps = kDetectThreads / 32;
+constexpr int kStatWarps = 3;  // warps that sum the statistics in fp64 (one per SM sub-partition)
+
 // One CTA per sequence, monitor state carried from call to call in dstate:
 //   lm[slot]  latest earlier row of the window (as it was when the row was examined) whose
 //             sketch matches the row, -1 if none.  Row i of the window [wlo, n) is novel iff
 //             lm[i] < wlo, and this stays true as the window start moves forward.
 //   run[P]    trailing rows (up to the test length) that match the row P earlier.
 //   synced    the length seen by the previous call.
-// When the length grew by exactly one row since the previous call, only the new row is
-// examined (one scan of the window, one comparison per period): O(W + P) row comparisons per
-// step.  Otherwise (first call, after a prune or any other change of the cache) the window and
-// the runs are recomputed: the sketches of the last smem_rows rows are staged in shared memory
-// with a row stride of nwords + 1 words (rows that different lanes read fall in different
-// banks), one warp scans each window row, one warp each period.
-__global__ void __launch_bounds__(kDetectThreads) detect_kernel(DetectArgs a) {
+// When the length grew by exactly one row since the previous call, only the new row i = n-1 is
+// examined: thread t compares it with rows i-1-t, i-1-t-T, ... of the window (T threads) and
+// stops at its first match; the comparison with row i-1-t is also period P = t+1's, so the
+// runs cost nothing more when p_min = 1.  Everything the call reads is loaded up front and the
+// CTA meets at two barriers, the first after every warp has reduced its share (latest match,
+// novel rows, shortest verified period, fp64 statistic sums).  Otherwise (first call, after a
+// prune or any other change of the cache) the window and the runs are recomputed: the
+// sketches of the last smem_rows rows are staged in shared memory with a row stride of
+// nwords + 1 words (rows that different lanes read fall in different banks), one warp scans
+// each window row, one warp each period.
+__global__ void __launch_bounds__(kDetectThreads, 1) detect_kernel(DetectArgs a) {
   extern __shared__ __align__(16) uint32_t sk_s[];
-  __shared__ double red_e[kDetectThreads / 32], red_l[kDetectThreads / 32];
-  __shared__ int s_novel, s_novel_tail, s_pstar, s_mismatch, s_trig, s_latest;
-  constexpr int kWarps = kDetectThreads / 32;
+  __shared__ double red_e[kStatWarps], red_l[kStatWarps];
+  __shared__ int w_latest[kDetectWarps], w_nov[kDetectWarps], w_nov_tail[kDetectWarps],
+      w_pstar[kDetectWarps];
+  __shared__ double s_logn;
+  __shared__ int s_sig[4];  // vote 1, vote 2, vote 3, stall
+  __shared__ int s_novel, s_novel_tail, s_pstar, s_mismatch, s_trig;
   const int b = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  if (status_bad(a.c.dev_status)) return;
-  const lg_guard_params &p = a.p;
+  const int32_t *status = a.c.dev_status;
   const int n = a.c.len[b];
   const int B = a.budget[b];
-  const int nw = a.nwords, thr = a.thr, stride = nw + 1;
-  const uint32_t *sk_g = a.c.sketch + a.c.seq_off[b] * nw;
-  const int w = min(p.W, n);
-  const int wlo = n - w;
+  const int64_t off = a.c.seq_off[b];
+  const lg_guard_params &p = a.p;
   const int np = p.p_max - p.p_min + 1;
   int32_t *ds = a.dstate + (int64_t)b * (np + 2);
-  int32_t *run = ds + 2;
-  int32_t *lm = a.dstate + (int64_t)a.c.batch * (np + 2) + a.c.seq_off[b];
-  const bool incr = n >= 1 && ds[0] + 1 == n;
-  // staged rows: the window and the period comparisons of the new row, or (recompute) every
-  // row the window and the period runs read
-  const int lo_s = max(0, n - (incr ? max(p.W, p.p_max + 1) : a.smem_rows));
-
-  // (1) sums of the entropies and suffix masses over every layer and head (fp64)
-  double se = 0.0, sl = 0.0;
-  const int nh = a.c.L * a.H_q;
-  for (int t = tid; t < nh; t += kDetectThreads) {
-    const int layer = t / a.H_q, h = t - layer * a.H_q;
-    const float *st = a.stats + (((int64_t)layer * a.c.batch + b) * a.H_q + h) * 4;
-    se += (double)st[2];
-    sl += (double)st[3];
-  }
-  for (int o = 16; o >= 1; o >>= 1) {
-    se += __shfl_xor_sync(0xffffffffu, se, o);
-    sl += __shfl_xor_sync(0xffffffffu, sl, o);
-  }
-  if (lane == 0) {
-    red_e[warp] = se;
-    red_l[warp] = sl;
-  }
+  const int synced = ds[0];
+  // the sequence's guard state, {t_gen, cd, level, last_trig} and {n_int, pad}, read by the
+  // thread that updates it
+  int4 st_a = make_int4(0, 0, 0, 0), st_b = make_int4(0, 0, 0, 0);
   if (tid == 0) {
-    s_novel = 0;
-    s_novel_tail = 0;
-    s_pstar = 0x7fffffff;
-    s_mismatch = -1;
-    s_latest = -1;
+    st_a = reinterpret_cast<const int4 *>(a.state + b)[0];
+    st_b = reinterpret_cast<const int4 *>(a.state + b)[1];
   }
-  for (int t = tid; t < (n - lo_s) * nw; t += kDetectThreads) {
-    const int r = t / nw;
-    sk_s[r * stride + (t - r * nw)] = sk_g[(int64_t)lo_s * nw + t];
-  }
-  __syncthreads();
-  auto row = [&](int i) -> const uint32_t * {
-    return i >= lo_s ? sk_s + (int64_t)(i - lo_s) * stride : sk_g + (int64_t)i * nw;
-  };
-  // latest j in [lo, i) whose row matches row i, or -1 (one warp, nearest rows first)
-  auto latest_match = [&](int i, int lo) -> int {
-    const uint32_t *ri = row(i);
-    for (int top = i - 1; top >= lo; top -= 32) {
-      const int j = top - lane;
-      const bool m = j >= lo && rows_match(ri, row(j), nw, thr);
-      const unsigned bal = __ballot_sync(0xffffffffu, m);
-      if (bal) return top - (__ffs(bal) - 1);
+  if (status_bad(status)) return;
+  const int nw = a.nwords, thr = a.thr, stride = nw + 1;
+  const uint32_t *sk_g = a.c.sketch + off * nw;
+  const int w = min(p.W, n);
+  const int wlo = n - w;
+  int32_t *run = ds + 2;
+  int32_t *lm = a.dstate + (int64_t)a.c.batch * (np + 2) + off;
+  const bool incr = n >= 1 && synced + 1 == n;
+  const int nh = a.c.L * a.H_q;
+
+  // (1) sums of the entropies and suffix masses over every layer and head (fp64, one warp per
+  // SM sub-partition), and ln n on the fourth sub-partition
+  if (warp < kStatWarps) {
+    double se = 0.0, sl = 0.0;
+    for (int t = tid; t < nh; t += kStatWarps * 32) {
+      const int layer = t / a.H_q, h = t - layer * a.H_q;
+      const float4 st = __ldg(reinterpret_cast<const float4 *>(a.stats) +
+                              ((int64_t)layer * a.c.batch + b) * a.H_q + h);
+      se += widen(st.z);
+      sl += widen(st.w);
     }
-    return -1;
-  };
+    for (int o = 16; o >= 1; o >>= 1) {
+      se += __shfl_xor_sync(0xffffffffu, se, o);
+      sl += __shfl_xor_sync(0xffffffffu, sl, o);
+    }
+    if (lane == 0) {
+      red_e[warp] = se;
+      red_l[warp] = sl;
+    }
+  } else if (warp == kStatWarps && lane == 0) {
+    s_logn = n >= 2 ? log((double)n) : 1.0;
+  }
 
   if (incr) {
-    // (2) the new row n-1: its latest match in the window (one candidate row per thread),
-    // and every period's run
+    // (2) the new row against the window and the periods, reduced per warp
     const int i = n - 1;
-    const uint32_t *ri = row(i);
-    for (int j = i - 1 - tid; j >= wlo; j -= kDetectThreads)
-      if (rows_match(ri, row(j), nw, thr)) {
-        atomicMax(&s_latest, j);
-        break;
-      }
+    const uint32_t *ri = sk_g + (int64_t)i * nw;
+    const int j0 = i - 1 - tid;
+    bool m0 = false;
+    int latest = -1;
+    if (j0 >= 0) {
+      m0 = hamming(ri, sk_g + (int64_t)j0 * nw, nw) <= thr;
+      if (m0 && j0 >= wlo) latest = j0;
+    }
+    if (latest < 0)
+      for (int j = j0 - kDetectThreads; j >= wlo; j -= kDetectThreads)
+        if (hamming(ri, sk_g + (int64_t)j * nw, nw) <= thr) {
+          latest = j;
+          break;
+        }
+    // novel rows of the window other than the new one
+    int nov = 0, nov_tail = 0;
+    for (int r = wlo + tid; r < i; r += kDetectThreads) {
+      const int novel = lm[r] < wlo;
+      nov += novel;
+      if (r >= n - p.stall_len) nov_tail += novel;
+    }
+    // period runs; P ascends with the thread index, so the first qualifying P of a warp is
+    // its lowest lane's and a thread's first qualifying P is its smallest
+    int pstar = 0x7fffffff;
     for (int pi = tid; pi < np; pi += kDetectThreads) {
       const int P = p.p_min + pi;
       const int cap = max(p.m_rep * P, p.l_min);
-      const bool m = i - P >= 0 && rows_match(ri, row(i - P), nw, thr);
-      run[pi] = m ? min(run[pi] + 1, cap) : 0;
+      const int j = i - P;
+      const bool m = j >= 0 && (P == tid + 1 ? m0 : hamming(ri, sk_g + (int64_t)j * nw, nw) <= thr);
+      const int r = m ? min(run[pi] + 1, cap) : 0;
+      run[pi] = r;
+      if (pstar == 0x7fffffff && n >= cap + P && r >= cap) pstar = P;
+    }
+    latest = __reduce_max_sync(0xffffffffu, latest);
+    nov = __reduce_add_sync(0xffffffffu, nov);
+    nov_tail = __reduce_add_sync(0xffffffffu, nov_tail);
+    pstar = (int)__reduce_min_sync(0xffffffffu, (unsigned)pstar);
+    if (lane == 0) {
+      w_latest[warp] = latest;
+      w_nov[warp] = nov;
+      w_nov_tail[warp] = nov_tail;
+      w_pstar[warp] = pstar;
     }
     __syncthreads();
-    if (tid == 0) lm[i] = s_latest;
-  } else {
-    // (2') recompute: every window row's latest match, every period's trailing run
-    for (int i = wlo + warp; i < n; i += kWarps) {
-      const int j = latest_match(i, wlo);
-      if (lane == 0) lm[i] = j;
+    if (tid == 0) {
+      int lt = -1, nv = 0, nt = 0, ps = 0x7fffffff;
+      for (int k = 0; k < kDetectWarps; ++k) {
+        lt = max(lt, w_latest[k]);
+        nv += w_nov[k];
+        nt += w_nov_tail[k];
+        ps = min(ps, w_pstar[k]);
+      }
+      lm[i] = lt;
+      const int novel = lt < wlo;
+      s_novel = nv + novel;
+      s_novel_tail = nt + (p.stall_len >= 1 ? novel : 0);
+      s_pstar = ps;
     }
-    for (int pi = warp; pi < np; pi += kWarps) {
+  } else {
+    // (2') recompute: every window row's latest match, every period's trailing run, from rows
+    // staged in shared memory
+    const int lo_s = max(0, n - a.smem_rows);
+    for (int t = tid; t < (n - lo_s) * nw; t += kDetectThreads) {
+      const int r = t / nw;
+      sk_s[r * stride + (t - r * nw)] = sk_g[(int64_t)lo_s * nw + t];
+    }
+    if (tid == 0) {
+      s_novel = 0;
+      s_novel_tail = 0;
+      s_pstar = 0x7fffffff;
+    }
+    __syncthreads();
+    auto row = [=](int r) -> const uint32_t * {
+      return r >= lo_s ? sk_s + (int64_t)(r - lo_s) * stride : sk_g + (int64_t)r * nw;
+    };
+    for (int r = wlo + warp; r < n; r += kDetectWarps) {
+      // latest j in [wlo, r) whose row matches row r, or -1 (one warp, nearest rows first)
+      const uint32_t *rr = row(r);
+      int found = -1;
+      for (int top = r - 1; top >= wlo; top -= 32) {
+        const int j = top - lane;
+        const bool m = j >= wlo && rows_match(rr, row(j), nw, thr);
+        const unsigned bal = __ballot_sync(0xffffffffu, m);
+        if (bal) {
+          found = top - (__ffs(bal) - 1);
+          break;
+        }
+      }
+      if (lane == 0) lm[r] = found;
+    }
+    for (int pi = warp; pi < np; pi += kDetectWarps) {
       const int P = p.p_min + pi;
       const int cap = max(p.m_rep * P, p.l_min);
       int r = cap;
@@ -262,16 +354,12 @@ __global__ void __launch_bounds__(kDetectThreads) detect_kernel(DetectArgs a) {
       }
       if (lane == 0) run[pi] = r;
     }
-  }
-  __syncthreads();
-
-  // (3) novelty of the window rows, stall, and the smallest period with a full verified run
-  {
+    __syncthreads();
     int nov = 0, nov_tail = 0;
-    for (int i = wlo + tid; i < n; i += kDetectThreads) {
-      const int novel = lm[i] < wlo;
+    for (int r = wlo + tid; r < n; r += kDetectThreads) {
+      const int novel = lm[r] < wlo;
       nov += novel;
-      if (i >= n - p.stall_len) nov_tail += novel;
+      if (r >= n - p.stall_len) nov_tail += novel;
     }
     nov = __reduce_add_sync(0xffffffffu, nov);
     nov_tail = __reduce_add_sync(0xffffffffu, nov_tail);
@@ -285,34 +373,45 @@ __global__ void __launch_bounds__(kDetectThreads) detect_kernel(DetectArgs a) {
   }
   __syncthreads();
 
-  // (5) votes, gates and the trigger
-  if (tid == 0) {
-    double e_sum = 0.0, l_sum = 0.0;
-    for (int k = 0; k < kDetectThreads / 32; ++k) {
-      e_sum += red_e[k];
-      l_sum += red_l[k];
+  // (3) the votes and the stall gate, one quotient per warp (different sub-partitions)
+  const int Ws = min(p.suffix_w, n);
+  if (lane == 0 && warp < 4 && n >= 1) {
+    if (warp == 0) {
+      // vote 2: mean of H / ln n over every layer and head
+      double e_sum = 0.0;
+      for (int k = 0; k < kStatWarps; ++k) e_sum += red_e[k];
+      const double ebar = n >= 2 ? e_sum / ((double)nh * s_logn) : 1.0;
+      s_sig[1] = ebar < p.theta_ent;
+      if (a.diag) a.diag[8 * b] = ebar;
+    } else if (warp == 1) {
+      // vote 3: mean of S * n / W_s over every layer and head
+      double l_sum = 0.0;
+      for (int k = 0; k < kStatWarps; ++k) l_sum += red_l[k];
+      const double lbar = l_sum * (double)n / ((double)Ws * (double)nh);
+      s_sig[2] = lbar >= p.theta_lift;
+      if (a.diag) a.diag[8 * b + 1] = lbar;
+    } else if (warp == 2) {
+      // vote 1: novel-row fraction of the window
+      const double ttr = (double)s_novel / (double)w;
+      s_sig[0] = ttr < p.theta_ttr;
+      if (a.diag) a.diag[8 * b + 2] = ttr;
+    } else {
+      s_sig[3] = w >= p.stall_len && p.stall_len > 0 &&
+                 (double)s_novel_tail / (double)p.stall_len < p.theta_nov;
     }
+  }
+  __syncthreads();
+
+  // (4) gates and the trigger
+  if (tid == 0) {
     int trig = 0;
     if (n >= 1) {
-      // mean of H / ln n and of S * n / W_s over every layer and head
-      const int Ws = min(p.suffix_w, n);
-      const double ebar = n >= 2 ? e_sum / ((double)nh * log((double)n)) : 1.0;
-      const double lbar = l_sum * (double)n / ((double)Ws * (double)nh);
-      const double ttr = (double)s_novel / (double)w;
-      const int sig1 = ttr < p.theta_ttr;
-      const int sig2 = ebar < p.theta_ent;
-      const int sig3 = lbar >= p.theta_lift;
+      const int sig1 = s_sig[0], sig2 = s_sig[1], sig3 = s_sig[2], stall = s_sig[3];
       const int warn = sig1 + sig2 + sig3 >= p.K;
-      const int stall = w >= p.stall_len && p.stall_len > 0 &&
-                        (double)s_novel_tail / (double)p.stall_len < p.theta_nov;
       const int tailrep = s_pstar != 0x7fffffff;
-      const lg_guard_state st = a.state[b];
-      trig = st.t_gen >= p.t_min && st.cd == 0 && warn && (stall || tailrep);
+      trig = st_a.x >= p.t_min && st_a.y == 0 && warn && (stall || tailrep);
       if (a.diag) {
         double *dg = a.diag + 8 * b;
-        dg[0] = ebar;
-        dg[1] = lbar;
-        dg[2] = ttr;
         dg[3] = sig1;
         dg[4] = sig2;
         dg[5] = sig3;
@@ -321,10 +420,11 @@ __global__ void __launch_bounds__(kDetectThreads) detect_kernel(DetectArgs a) {
       }
     }
     s_trig = trig;
+    s_mismatch = -1;
   }
   __syncthreads();
 
-  // (6) span: extend the verified tail back while rows keep matching the row P* earlier
+  // (5) span: extend the verified tail back while rows keep matching the row P* earlier
   const int trig = s_trig;
   const int Pstar = s_pstar;
   const int R = B / 2;
@@ -338,7 +438,8 @@ __global__ void __launch_bounds__(kDetectThreads) detect_kernel(DetectArgs a) {
     } else {
       for (int hi = s; hi > lo_ext; hi -= kDetectThreads) {
         const int i = hi - 1 - tid;
-        if (i >= lo_ext && !rows_match(row(i), row(i - Pstar), nw, thr)) atomicMax(&s_mismatch, i);
+        if (i >= lo_ext && hamming(sk_g + (int64_t)i * nw, sk_g + (int64_t)(i - Pstar) * nw, nw) > thr)
+          atomicMax(&s_mismatch, i);
         __syncthreads();
         const int found = s_mismatch;
         __syncthreads();
@@ -357,18 +458,19 @@ __global__ void __launch_bounds__(kDetectThreads) detect_kernel(DetectArgs a) {
     a.flags[b] = trig;
     a.spans[2 * b] = lo;
     a.spans[2 * b + 1] = hi;
-    lg_guard_state st = a.state[b];
+    // x = t_gen, y = cd, z = level, w = last_trig; st_b.x = n_int
     if (trig) {
-      const bool quick = st.t_gen - st.last_trig <= p.retrig_window;
-      st.level = quick ? min(st.level + 1, p.level_max) : 0;
-      st.last_trig = st.t_gen;
-      st.cd = p.cooldown;
-      st.n_int += 1;
-    } else if (st.cd > 0) {
-      st.cd -= 1;
+      const bool quick = st_a.x - st_a.w <= p.retrig_window;
+      st_a.z = quick ? min(st_a.z + 1, p.level_max) : 0;
+      st_a.w = st_a.x;
+      st_a.y = p.cooldown;
+      st_b.x += 1;
+    } else if (st_a.y > 0) {
+      st_a.y -= 1;
     }
-    st.t_gen += 1;
-    a.state[b] = st;
+    st_a.x += 1;
+    reinterpret_cast<int4 *>(a.state + b)[0] = st_a;
+    reinterpret_cast<int4 *>(a.state + b)[1] = st_b;
     ds[0] = n;
   }
 }
@@ -779,14 +881,15 @@ cudaError_t launch_append(const lg_cache &c, int layer0, int n_layers, const voi
   const int row_blocks = (int)((total + 255) / 256);
   const bool sk = c.sketch && guard_layer >= layer0 && guard_layer < layer0 + n_layers;
   const int grid = row_blocks + (sk ? c.batch : 0);
-  if (c.dtype == LG_BF16)
+  if (c.dtype == LG_BF16) {
     append_kernel<__nv_bfloat16><<<grid, 256, 0, s>>>(c, layer0, n_layers, (const uint4 *)k_new,
                                                       (const uint4 *)v_new, pos_new, row_blocks,
                                                       guard_layer - layer0);
-  else
+  } else {
     append_kernel<float><<<grid, 256, 0, s>>>(c, layer0, n_layers, (const uint4 *)k_new,
                                               (const uint4 *)v_new, pos_new, row_blocks,
                                               guard_layer - layer0);
+  }
   return cudaGetLastError();
 }
 
@@ -797,10 +900,11 @@ cudaError_t launch_sketch_build(const lg_cache &c, int guard_layer, int max_len,
   if (gx > 1024) gx = 1024;
   if (gx < 1) gx = 1;
   dim3 grid(gx, c.batch);
-  if (c.dtype == LG_BF16)
+  if (c.dtype == LG_BF16) {
     sketch_build_kernel<__nv_bfloat16><<<grid, 256, 0, s>>>(c, guard_layer, max_len);
-  else
+  } else {
     sketch_build_kernel<float><<<grid, 256, 0, s>>>(c, guard_layer, max_len);
+  }
   return cudaGetLastError();
 }
 

@@ -255,10 +255,10 @@ class Cache:
         self.nwords = H_kv * d // 32
         self.sketch = None
         self.h2o = self.pos = None
-        if policy in ("loopguard", "full"):
+        if policy == "loopguard":
             self.sketch = torch.zeros((self.S_total, self.nwords), dtype=torch.int32,
                                       device=self.device)
-        if policy in ("h2o", "streaming"):
+        if policy in ("h2o", "streaming", "full"):
             self.h2o = torch.zeros((L, H_kv, self.S_total), dtype=torch.float32,
                                    device=self.device)
             self.pos = torch.zeros((L, H_kv, self.S_total), dtype=torch.int32,

@@ -16,6 +16,7 @@ budget, Sec. 6.1) at the five benchmark shapes:
   3  small-model long context, 28 layers, 12/2 heads, b=32, n=32768, B=8192, sinks
   4  ragged serving batch, b=64, n log-uniform in [1024, 65536], B=min(n+256, 16384)
   5  bandwidth sweep, 32 layers, 64/8 heads, b=16, n=131072, B=32768
+  6  the paper's setting: Qwen3-1.7B shape, one 3853-token prompt, B=1024, T_max 2500
 
 ``make_workload(i, **overrides)`` returns one of them; overrides shrink a
 workload for tests while keeping its structure.
@@ -163,7 +164,7 @@ def _seqs(batch):
 
 
 def make_workload(i: int, **ov) -> Workload:
-    """Benchmark workload i (1..5); keyword overrides shrink it for tests."""
+    """Benchmark workload i (1..6); keyword overrides shrink it for tests."""
     if i == 1:
         n = ov.get("n", 512)
         loop_len = ov.get("loop_len", 192)
@@ -248,7 +249,27 @@ def make_workload(i: int, **ov) -> Workload:
                         "n=%d, B=%d" % (L, b, n, B)),
             L=L, H_q=64, H_kv=8, d=128, dtype="bf16", batch=b, n0=[n] * b, budget=[B] * b,
             steps=ov.get("steps", 2), seed=seed, seqs=seqs)
-    raise ValueError("workload index must be 1..5")
+    if i == 6:
+        # The paper's own setting (Sec. 6.1, App. C): a 1-2B model (Qwen3-1.7B shape: 28 layers,
+        # 16 query / 8 kv heads, d=128), a LoopBench-DC-length prompt (3853 tokens on average),
+        # budget 1024, generation capped at T_max = 2500; one loop whose onset falls where
+        # most of the paper's interventions happen (800-1300 generated tokens, Fig. 4).
+        b = ov.get("batch", 1); seed = ov.get("seed", 5)
+        n = ov.get("n", 3853); B = ov.get("budget", 1024)
+        L = ov.get("L", 28)
+        on_lo, on_hi = ov.get("onset", (800, 1300))
+        p_lo, p_hi = ov.get("periods", (16, 64))
+        seqs = _seqs(b)
+        for s in range(b):
+            P = _randint(seed, 2, s, p_lo, p_hi)
+            onset = _randint(seed, 3, s, on_lo, on_hi)
+            seqs[s] = (1, n + onset, P, NEVER)
+        return Workload(
+            name=ov.get("name", "paper-shaped guard: Qwen3-1.7B shape (%d layers, 16/8 heads, "
+                        "d=128), bf16, b=%d, prompt %d, B=%d, T_max 2500" % (L, b, n, B)),
+            L=L, H_q=16, H_kv=8, d=128, dtype="bf16", batch=b, n0=[n] * b, budget=[B] * b,
+            steps=ov.get("steps", 2500), seed=seed, seqs=seqs)
+    raise ValueError("workload index must be 1..6")
 
 
 # ----------------------------------------------------------------------------- host generator

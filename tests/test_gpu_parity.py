@@ -115,3 +115,12 @@ def test_streaming_comparator(cuda):
     w = synth.make_workload(4, L=2, batch=4, len_range=(100, 900), budget_max=384, steps=4,
                             periods=(4, 8), onset_max=2)
     run_streaming(w, cuda)
+
+
+def test_paper_shaped_guard(cuda):
+    """workload 6 structure (the paper's setting: 16/8 heads, one 3853-token prompt, B=1024):
+    the first budget cut from 3854 rows, periodic budget cuts every B - T_keep steps, and a
+    planted loop that triggers, at 2 layers and an early onset"""
+    w = synth.make_workload(6, L=2, onset=(90, 110), steps=200)
+    c = run_loopguard(w, cuda)
+    assert c["triggers"] >= 1 and c["prunes"] >= 3
