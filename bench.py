@@ -232,8 +232,10 @@ class GpuBench:
         self.sel((self.qA[t], self.kA[t], self.vA[t]), (self.qB[t], self.kB[t], self.vB[t]),
                  self.s)
 
-    def step(self, t, ev=None):
-        """one guarded decode step; ev = (a0, a1, p0, p1) events around attend and prune"""
+    def step(self, t, ev=None, split=False):
+        """one guarded decode step; ev = (a0, a1, p0, p1) events around attend and the guard
+        (a1 -> p1); split: the loop-onset test and the compaction as separate calls
+        (lg_detect, lg_prune_compact: the same results) with p0 between them"""
         lg, c, g, p, w = self.lg, self.cache, self.guard, self.p, self.w
         h2o = self.policy == "h2o"
         guard_path = self.policy == "loopguard"
@@ -249,16 +251,21 @@ class GpuBench:
                                 1 if h2o else 0, g.max_len, g.ws, self.s)
         if ev:
             ev[1].record(self.stream)
-        if guard_path:
+        if guard_path and not split:
+            # loop-onset test and retained set in one kernel, then the compaction
+            lg.lg_detect_prune(c, g.stats, w.H_q, g.state, self.budget_d, p, g.flags, g.spans,
+                               None, g.dstate, g.kept_idx, g.kept_count, g.max_keep, g.max_len,
+                               self.s)
+        elif guard_path:
             lg.lg_detect(c, g.stats, w.H_q, g.state, self.budget_d, p, g.flags, g.spans, None,
                          g.dstate, self.s)
         if ev:
             ev[2].record(self.stream)
-        if h2o:
-            lg.lg_h2o_evict(c, self.budget_d, pos_t, g.max_len, self.s)
-        elif guard_path:
+        if guard_path and split:
             lg.lg_prune_compact(c, g.flags, g.spans, g.state, self.budget_d, p, g.kept_idx,
                                 g.kept_count, g.max_keep, g.max_len, self.s)
+        elif h2o:
+            lg.lg_h2o_evict(c, self.budget_d, pos_t, g.max_len, self.s)
         elif self.policy == "streaming":
             lg.lg_streaming_evict(c, self.budget_d, pos_t, lg.N_SINK, g.max_len, self.s)
         if ev:
@@ -274,29 +281,33 @@ class GpuBench:
             path = 1 + 1 + 2 * calls + 2
         elif self.policy == "full":        # begin, append, attend (partial, combine)
             path = 1 + 1 + 2 * calls
-        else:                      # begin, append (+sketch), attend (partial, combine), detect,
-            path = 1 + 1 + 2 * calls + 1 + 2        # keep + compact
+        else:                      # begin, append (+sketch), attend (partial, combine),
+            path = 1 + 1 + 2 * calls + 2            # detect + keep, compact
         harness = 1 + 1                             # select, advance
         return path, harness
 
     def replay_log(self, K, fresh=False):
-        """replay the timed trajectory untimed, recording per-step lengths and kept lists
-        (the decisions are deterministic, so they are the timed run's)"""
+        """replay the timed trajectory (the decisions are deterministic, so they are the
+        timed run's), recording per-step lengths and kept lists, with the guard split into
+        lg_detect and lg_prune_compact and events around the compaction; returns
+        (lens, kept, compaction ms per step)"""
         torch = self.torch
         self.reset()
-        lens, kept = [], []
+        lens, kept, evs = [], [], []
         for t in range(K):
             if fresh:
                 self.reset()
             lens.append(self.cache.len.clone())
-            self.step(0 if fresh else t)
+            ev = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
+            self.step(0 if fresh else t, ev, split=True)
+            evs.append(ev)
             if self.policy != "loopguard":
                 kept.append((None, None))
                 continue
             kc = self.guard.kept_count.clone()
             kept.append((kc, self.guard.kept_idx.clone() if int((kc >= 0).sum()) else None))
         torch.cuda.synchronize()
-        return lens, kept
+        return lens, kept, [e[2].elapsed_time(e[3]) for e in evs]
 
 
 def attend_bytes(w, n_rows, h2o=False):
@@ -449,11 +460,10 @@ def run_gpu(args, ws, rank, local):
         raise RuntimeError("device status %d after the timed run" % status)
     ms = max_over_ranks(ms_local, ws)
     attend_ms = [e[0].elapsed_time(e[1]) for e in evs]
-    detect_ms = [e[1].elapsed_time(e[2]) for e in evs]
-    prune_ms = [e[2].elapsed_time(e[3]) for e in evs]
+    guard_ms = [e[1].elapsed_time(e[3]) for e in evs]
 
-    # algorithmic bytes of the same trajectory (untimed, deterministic replay)
-    lens, kept = bench.replay_log(K, fresh)
+    # algorithmic bytes of the same trajectory (deterministic replay, not the timed region)
+    lens, kept, prune_ms = bench.replay_log(K, fresh)
     a_bytes, c_bytes, c_ms = [], [], []
     triggers = 0
     for t in range(K):
@@ -513,10 +523,8 @@ def run_gpu(args, ws, rank, local):
                               "ms_per_event": round(sum(c_ms) / len(c_ms), 4) if c_ms else None,
                               "moved_bytes_per_event": int(sum(c_bytes) / len(c_bytes))
                               if c_bytes else 0},
-            "detect_ms_per_step": round(sum(detect_ms) / K, 4),
-            "cache_update_ms_per_step": round(sum(prune_ms) / K, 4),
-            "other_ms_per_step": round((ms_local - sum(attend_ms) - sum(detect_ms) -
-                                        sum(prune_ms)) / K, 4)},
+            "guard_ms_per_step": round(sum(guard_ms) / K, 4),
+            "other_ms_per_step": round((ms_local - sum(attend_ms) - sum(guard_ms)) / K, 4)},
         "eager_ms_per_step": round(eager_ms / K, 4) if eager_ms is not None else None,
         "gpu_launches": (path_l + harness_l) * K,
         "gpu_launches_detail": {"path_per_step": path_l, "harness_per_step": harness_l},

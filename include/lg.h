@@ -10,6 +10,7 @@
  *
  * A decode step on this ABI:
  *   lg_begin_step -> lg_append -> lg_decode_attend -> lg_detect -> lg_prune_compact
+ *   (lg_detect_prune fuses the last two)
  * or, on the comparator path:
  *   lg_begin_step -> lg_append -> lg_decode_attend(accumulate_h2o=1) -> lg_h2o_evict
  *
@@ -214,6 +215,15 @@ LG_API lg_status lg_prune_compact(const lg_cache *c, const int32_t *flags, const
                            const lg_guard_state *state, const int32_t *budget,
                            const lg_guard_params *p, int32_t *kept_idx, int32_t *kept_count,
                            int max_keep, int max_len, cudaStream_t s);
+
+/* lg_detect followed by lg_prune_compact (same arguments, same results, same device state),
+   with the retained set formed by the loop-onset test's own kernel: two kernel launches instead
+   of three.  Validation is the union of both calls'; dstate and the kept lists as there. */
+LG_API lg_status lg_detect_prune(const lg_cache *c, const float *stats, int H_q,
+                                 lg_guard_state *state, const int32_t *budget,
+                                 const lg_guard_params *p, int32_t *flags, int32_t *spans,
+                                 double *diag, void *dstate, int32_t *kept_idx,
+                                 int32_t *kept_count, int max_keep, int max_len, cudaStream_t s);
 
 /* H2O comparator state: pos[l][h][slot] = slot and h2o = 0 for slots [0, len[b]) (after a
    prefill whose rows are in token order). */

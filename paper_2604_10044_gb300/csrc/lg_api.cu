@@ -215,8 +215,27 @@ lg_status lg_detect(const lg_cache *c, const float *stats, int H_q, lg_guard_sta
   if (((uintptr_t)dstate & 3u) || ((uintptr_t)stats & 15u)) return LG_ERR_INVALID_ARG;
   if (H_q < 1 || H_q % c->H_kv) return LG_ERR_INVALID_ARG;
   if (lg::detect_smem_bytes(*p, c->H_kv * c->d / 32) > 200 * 1024) return LG_ERR_UNSUPPORTED;
-  return cuda_status(
-      lg::launch_detect(*c, stats, H_q, state, budget, *p, flags, spans, diag, dstate, s));
+  return cuda_status(lg::launch_detect(*c, stats, H_q, state, budget, *p, flags, spans, diag,
+                                       dstate, nullptr, nullptr, 0, 0, s));
+}
+
+lg_status lg_detect_prune(const lg_cache *c, const float *stats, int H_q, lg_guard_state *state,
+                          const int32_t *budget, const lg_guard_params *p, int32_t *flags,
+                          int32_t *spans, double *diag, void *dstate, int32_t *kept_idx,
+                          int32_t *kept_count, int max_keep, int max_len, cudaStream_t s) {
+  lg_status st = check_cache(c);
+  if (st != LG_OK) return st;
+  if ((st = check_params(p)) != LG_OK) return st;
+  if (!c->sketch || !stats || !state || !budget || !flags || !spans || !dstate)
+    return LG_ERR_INVALID_ARG;
+  if (!kept_idx || !kept_count || max_keep < 1 || max_len < 0) return LG_ERR_INVALID_ARG;
+  if (((uintptr_t)dstate & 3u) || ((uintptr_t)stats & 15u)) return LG_ERR_INVALID_ARG;
+  if (H_q < 1 || H_q % c->H_kv) return LG_ERR_INVALID_ARG;
+  if (lg::detect_smem_bytes(*p, c->H_kv * c->d / 32) > 200 * 1024) return LG_ERR_UNSUPPORTED;
+  st = cuda_status(lg::launch_detect(*c, stats, H_q, state, budget, *p, flags, spans, diag,
+                                     dstate, kept_idx, kept_count, max_keep, max_len, s));
+  if (st != LG_OK) return st;
+  return cuda_status(lg::launch_compact(*c, kept_idx, kept_count, max_keep, s));
 }
 
 size_t lg_detect_state_size(const lg_cache *c, const lg_guard_params *p) {

@@ -112,6 +112,100 @@ __global__ void state_init_kernel(int batch, lg_guard_state *state, int t_gen0) 
   state[b] = s;
 }
 
+// ------------------------------------------------------------------ retained set I_keep
+
+// I_keep of one sequence in closed form (Sec. 5.3, Eq. 10, Eq. 11).  Its three pieces are
+// disjoint ranges of slots taken in ascending order:
+//   anchors   [0, cA), cA = min(N_anchor, n)
+//   lattice   N_anchor + floor(j n_c / B_sparse), j < B_sparse, over the n_c rows between the
+//             anchors and W^recent = [max(N_anchor, n - R), n); every such row if n_c <= B_sparse
+//   recent    the last B_recent(level) rows of W^recent outside the span I_bad: the rows above
+//             the span first, then, if they are fewer, the top rows below it
+// so slot j of the kept list is a function of j alone and every thread writes its own slots.
+struct KeepPlan {
+  int count;              // rows kept
+  int cA, cL;             // anchors, lattice rows
+  int na, n_c, B_sp;      // lattice geometry
+  int lo_start, lo_cnt;   // recent rows below the span
+  int hi_start;           // recent rows above the span (up to n)
+};
+
+// false when the budget leaves no room for the pieces (B_sparse < 0)
+__device__ __forceinline__ bool keep_plan(int n, int B, int flag, int span_lo, int span_hi,
+                                          int level, const lg_guard_params &p, KeepPlan &k) {
+  const int hd = min(p.headroom, B / 4);
+  const int T = B - hd;
+  const int R = B / 2;
+  const int B_rec = (B / 4) >> (flag ? level : 0);  // a budget event prunes at level 0
+  const int B_sp = T - p.n_anchor - B / 4;
+  if (B_sp < 0) return false;
+  const int na = p.n_anchor;
+  const int rw_lo = min(max(na, n - R), n);
+  k.na = na;
+  k.B_sp = B_sp;
+  k.cA = min(na, n);
+  k.n_c = max(0, rw_lo - na);
+  k.cL = min(k.n_c, B_sp);
+  // the span clipped to W^recent; a budget event has none
+  const int blo = flag ? max(span_lo, rw_lo) : 0;
+  const int bhi = flag ? min(span_hi, n) : 0;
+  int cR;
+  if (blo < bhi) {
+    const int above = n - bhi;
+    if (above >= B_rec) {
+      k.lo_start = blo;
+      k.lo_cnt = 0;
+      k.hi_start = n - B_rec;
+      cR = B_rec;
+    } else {
+      const int below = min(B_rec - above, blo - rw_lo);
+      k.lo_start = blo - below;
+      k.lo_cnt = below;
+      k.hi_start = bhi;
+      cR = below + above;
+    }
+  } else {
+    cR = min(B_rec, n - rw_lo);
+    k.lo_start = n;
+    k.lo_cnt = 0;
+    k.hi_start = n - cR;
+  }
+  k.count = k.cA + k.cL + cR;
+  return true;
+}
+
+__device__ __forceinline__ int keep_row(const KeepPlan &k, int j) {
+  if (j < k.cA) return j;
+  j -= k.cA;
+  if (j < k.cL) return k.na + (k.n_c <= k.B_sp ? j : (int)(((int64_t)j * k.n_c) / k.B_sp));
+  j -= k.cL;
+  return j < k.lo_cnt ? k.lo_start + j : k.hi_start + (j - k.lo_cnt);
+}
+
+// One sequence's prune decision and kept list, written by the nthreads threads of a CTA:
+// no prune (no trigger and n <= B) -> kept_count = -1; otherwise the kept list, its size,
+// and len = that size.  Returns the status code to raise (0 = none).
+__device__ __forceinline__ int write_keep(const lg_cache &c, int b, int n, int B, int flag,
+                                          int span_lo, int span_hi, int level,
+                                          const lg_guard_params &p, int32_t *kept_idx,
+                                          int32_t *kept_count, int max_keep, int max_len,
+                                          int tid, int nthreads) {
+  if (!flag && n <= B) {
+    if (tid == 0) kept_count[b] = -1;
+    return 0;
+  }
+  if (n > max_len) return LG_ERR_CAPACITY;
+  KeepPlan k;
+  if (!keep_plan(n, B, flag, span_lo, span_hi, level, p, k) || B > max_keep) return LG_ERR_BUDGET;
+  int32_t *out = kept_idx + (int64_t)b * max_keep;
+  for (int j = tid; j < k.count; j += nthreads) out[j] = keep_row(k, j);
+  if (tid == 0) {
+    kept_count[b] = k.count;
+    c.len[b] = k.count;
+  }
+  return 0;
+}
+
 // ------------------------------------------------------------------ loop-onset test
 
 struct DetectArgs {
@@ -125,6 +219,9 @@ struct DetectArgs {
   double *diag;
   int32_t *dstate;
   int nwords, thr, smem_rows;
+  // nullable: when set, the same CTA goes on to the retained set (see write_keep)
+  int32_t *kept_idx, *kept_count;
+  int max_keep, max_len;
 };
 
 constexpr int kDetectThreads = 512;
@@ -195,7 +292,8 @@ __global__ void __launch_bounds__(kDetectThreads, 1) detect_kernel(DetectArgs a)
       w_pstar[kDetectWarps];
   __shared__ double s_logn;
   __shared__ int s_sig[4];  // vote 1, vote 2, vote 3, stall
-  __shared__ int s_novel, s_novel_tail, s_pstar, s_mismatch, s_trig;
+  __shared__ int s_novel, s_novel_tail, s_pstar, s_mismatch, s_trig, s_span_lo, s_span_hi,
+      s_level;
   const int b = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int32_t *status = a.c.dev_status;
   const int n = a.c.len[b];
@@ -472,6 +570,17 @@ __global__ void __launch_bounds__(kDetectThreads, 1) detect_kernel(DetectArgs a)
     reinterpret_cast<int4 *>(a.state + b)[0] = st_a;
     reinterpret_cast<int4 *>(a.state + b)[1] = st_b;
     ds[0] = n;
+    s_span_lo = lo;
+    s_span_hi = hi;
+    s_level = st_a.z;
+  }
+  if (a.kept_idx) {
+    // (6) the retained set of this sequence from the decision just taken
+    __syncthreads();
+    const int code = write_keep(a.c, b, n, B, trig, s_span_lo, s_span_hi, s_level, p,
+                                a.kept_idx, a.kept_count, a.max_keep, a.max_len, tid,
+                                kDetectThreads);
+    if (code && tid == 0) set_status(a.c.dev_status, code);
   }
 }
 
@@ -504,89 +613,17 @@ struct KeepArgs {
 constexpr int kKeepThreads = 1024;
 
 __global__ void __launch_bounds__(kKeepThreads) keep_set_kernel(KeepArgs a) {
-  __shared__ int warp_tot[kKeepThreads / 32];
-  __shared__ int s_base;
-  const int b = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  if (status_bad(a.c.dev_status)) return;
+  const int b = blockIdx.x, tid = threadIdx.x;
+  const int32_t *status = a.c.dev_status;
   const int n = a.c.len[b];
   const int B = a.budget[b];
   const int flag = a.flags ? a.flags[b] : 0;
-  if (!flag && n <= B) {
-    if (tid == 0) a.kept_count[b] = -1;
-    return;
-  }
-  if (n > a.max_len) {
-    if (tid == 0) set_status(a.c.dev_status, LG_ERR_CAPACITY);
-    return;
-  }
-  const lg_guard_params &p = a.p;
-  const int level = flag ? a.state[b].level : 0;
-  const int hd = min(p.headroom, B / 4);
-  const int T = B - hd;
-  const int R = B / 2;
-  const int B_rec = (B / 4) >> level;
-  const int B_sp = T - p.n_anchor - B / 4;
-  if (B_sp < 0 || B > a.max_keep) {
-    if (tid == 0) set_status(a.c.dev_status, LG_ERR_BUDGET);
-    return;
-  }
-  const int na = p.n_anchor;
-  const int rw_lo = min(max(na, n - R), n);
-  const int n_c = max(0, rw_lo - na);
-  int blo = 0, bhi = 0;
-  if (flag) {
-    blo = max(a.spans[2 * b], rw_lo);
-    bhi = min(a.spans[2 * b + 1], n);
-    if (blo > bhi) blo = bhi;
-  }
-  int32_t *out = a.kept_idx + (int64_t)b * a.max_keep;
-  if (tid == 0) s_base = 0;
-  __syncthreads();
-  for (int c0 = 0; c0 < n; c0 += kKeepThreads) {
-    const int i = c0 + tid;
-    bool keep = false;
-    if (i < n) {
-      if (i < na) {
-        keep = true;  // anchors
-      } else if (i < rw_lo) {
-        // sparse lattice na + floor(j n_c / B_sp), j < B_sp
-        if (n_c <= B_sp) {
-          keep = true;
-        } else {
-          const int64_t x = i - na;
-          const int64_t j = (x * B_sp + n_c - 1) / n_c;
-          keep = j < B_sp && (j * n_c) / B_sp == x;
-        }
-      } else if (!(i >= blo && i < bhi)) {
-        // tail-cleaned recent rows: rank from the end among W^recent minus the span
-        const int overlap = max(0, bhi - max(blo, i + 1));
-        const int rank = (n - 1 - i) - overlap;
-        keep = rank < B_rec;
-      }
-    }
-    const unsigned bal = __ballot_sync(0xffffffffu, keep);
-    if (lane == 0) warp_tot[warp] = __popc(bal);
-    __syncthreads();
-    if (warp == 0) {
-      int v = warp_tot[lane];
-      int incl = v;
-      for (int o = 1; o < 32; o <<= 1) {
-        const int y = __shfl_up_sync(0xffffffffu, incl, o);
-        if (lane >= o) incl += y;
-      }
-      warp_tot[lane] = incl - v;  // exclusive
-    }
-    __syncthreads();
-    const int base = s_base;
-    if (keep) out[base + warp_tot[warp] + __popc(bal & ((1u << lane) - 1u))] = i;
-    __syncthreads();
-    if (tid == kKeepThreads - 1) s_base = base + warp_tot[warp] + __popc(bal);
-    __syncthreads();
-  }
-  if (tid == 0) {
-    a.kept_count[b] = s_base;
-    a.c.len[b] = s_base;
-  }
+  const int span_lo = a.spans ? a.spans[2 * b] : 0, span_hi = a.spans ? a.spans[2 * b + 1] : 0;
+  const int level = a.flags ? a.state[b].level : 0;  // state may be null without flags
+  if (status_bad(status)) return;
+  const int code = write_keep(a.c, b, n, B, flag, span_lo, span_hi, level, a.p, a.kept_idx,
+                              a.kept_count, a.max_keep, a.max_len, tid, kKeepThreads);
+  if (code && tid == 0) set_status(a.c.dev_status, code);
 }
 
 // ------------------------------------------------------------------ ordered in-place gather
@@ -915,8 +952,13 @@ cudaError_t launch_state_init(const lg_cache &c, lg_guard_state *state, int t_ge
 
 cudaError_t launch_detect(const lg_cache &c, const float *stats, int H_q, lg_guard_state *state,
                           const int32_t *budget, const lg_guard_params &p, int32_t *flags,
-                          int32_t *spans, double *diag, void *dstate, cudaStream_t s) {
+                          int32_t *spans, double *diag, void *dstate, int32_t *kept_idx,
+                          int32_t *kept_count, int max_keep, int max_len, cudaStream_t s) {
   DetectArgs a;
+  a.kept_idx = kept_idx;
+  a.kept_count = kept_count;
+  a.max_keep = max_keep;
+  a.max_len = max_len;
   a.c = c;
   a.stats = stats;
   a.H_q = H_q;
@@ -956,6 +998,11 @@ cudaError_t launch_prune_compact(const lg_cache &c, const int32_t *flags, const 
   keep_set_kernel<<<c.batch, kKeepThreads, 0, s>>>(a);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
+  return launch_compact(c, kept_idx, kept_count, max_keep, s);
+}
+
+cudaError_t launch_compact(const lg_cache &c, const int32_t *kept_idx, const int32_t *kept_count,
+                           int max_keep, cudaStream_t s) {
   int dev = 0, sms = 152;
   if (cudaGetDevice(&dev) == cudaSuccess)
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);

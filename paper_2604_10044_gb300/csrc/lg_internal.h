@@ -41,9 +41,11 @@ cudaError_t launch_append(const lg_cache &c, int layer0, int n_layers, const voi
 cudaError_t launch_sketch_build(const lg_cache &c, int guard_layer, int max_len, cudaStream_t s);
 cudaError_t launch_state_init(const lg_cache &c, lg_guard_state *state, int t_gen0,
                               cudaStream_t s);
+// kept_idx nullable: when set, the retained set is formed in the same kernel (no compaction)
 cudaError_t launch_detect(const lg_cache &c, const float *stats, int H_q, lg_guard_state *state,
                           const int32_t *budget, const lg_guard_params &p, int32_t *flags,
-                          int32_t *spans, double *diag, void *dstate, cudaStream_t s);
+                          int32_t *spans, double *diag, void *dstate, int32_t *kept_idx,
+                          int32_t *kept_count, int max_keep, int max_len, cudaStream_t s);
 size_t detect_state_bytes(const lg_cache &c, const lg_guard_params &p);
 int detect_smem_rows(const lg_guard_params &p);
 size_t detect_smem_bytes(const lg_guard_params &p, int nwords);
@@ -51,6 +53,8 @@ cudaError_t launch_prune_compact(const lg_cache &c, const int32_t *flags, const 
                                  const lg_guard_state *state, const int32_t *budget,
                                  const lg_guard_params &p, int32_t *kept_idx,
                                  int32_t *kept_count, int max_keep, int max_len, cudaStream_t s);
+cudaError_t launch_compact(const lg_cache &c, const int32_t *kept_idx, const int32_t *kept_count,
+                           int max_keep, cudaStream_t s);
 cudaError_t launch_h2o_reset(const lg_cache &c, int max_len, cudaStream_t s);
 cudaError_t launch_h2o_evict(const lg_cache &c, const int32_t *budget, const int32_t *pos_now,
                              int max_len, cudaStream_t s);

@@ -69,6 +69,8 @@ def lib():
                                  i32, vp, ctypes.c_size_t, vp],
             "lg_detect": [P(LgCache), vp, i32, vp, vp, P(LgGuardParams), vp, vp, vp, vp, vp],
             "lg_detect_state_size": [P(LgCache), P(LgGuardParams)],
+            "lg_detect_prune": [P(LgCache), vp, i32, vp, vp, P(LgGuardParams), vp, vp, vp, vp,
+                                vp, vp, i32, i32, vp],
             "lg_prune_compact": [P(LgCache), vp, vp, vp, vp, P(LgGuardParams), vp, vp, i32, i32,
                                  vp],
             "lg_h2o_reset": [P(LgCache), i32, vp],
@@ -95,7 +97,8 @@ def exported_symbols():
     return ["lg_default_params", "lg_status_string", "lg_workspace_size", "lg_state_init",
             "lg_begin_step", "lg_append", "lg_sketch_build", "lg_decode_attend", "lg_detect",
             "lg_prune_compact", "lg_h2o_reset", "lg_h2o_evict", "lg_read_device_status",
-            "lg_decode_attend_noalloc", "lg_detect_state_size", "lg_streaming_evict"]
+            "lg_decode_attend_noalloc", "lg_detect_state_size", "lg_streaming_evict",
+            "lg_detect_prune"]
 
 NOALLOC_SCRATCH_BYTES = 32 << 20  # LG_NOALLOC_SCRATCH_BYTES in include/lg.h
 
@@ -182,6 +185,13 @@ def lg_detect(cache, stats, H_q, state, budget, params, flags, spans, diag, dsta
     _call("lg_detect", ctypes.byref(cache.c), _ptr(stats), H_q, _ptr(state), _ptr(budget),
           ctypes.byref(params), _ptr(flags), _ptr(spans), _ptr(diag), _ptr(dstate),
           _stream(stream))
+
+
+def lg_detect_prune(cache, stats, H_q, state, budget, params, flags, spans, diag, dstate,
+                    kept_idx, kept_count, max_keep, max_len, stream=None):
+    _call("lg_detect_prune", ctypes.byref(cache.c), _ptr(stats), H_q, _ptr(state), _ptr(budget),
+          ctypes.byref(params), _ptr(flags), _ptr(spans), _ptr(diag), _ptr(dstate),
+          _ptr(kept_idx), _ptr(kept_count), max_keep, max_len, _stream(stream))
 
 
 def lg_prune_compact(cache, flags, spans, state, budget, params, kept_idx, kept_count, max_keep,
@@ -297,8 +307,10 @@ class Guard:
     """Device buffers and call order of one guarded decode step (lg.h) for a Cache."""
 
     def __init__(self, cache: Cache, H_q: int, params: LgGuardParams | None = None,
-                 policy="loopguard", max_len=None, t_gen0=64, n_layers_per_call=None):
+                 policy="loopguard", max_len=None, t_gen0=64, n_layers_per_call=None,
+                 fused_prune=True):
         self.cache = cache
+        self.fused_prune = fused_prune  # lg_detect_prune, else lg_detect + lg_prune_compact
         self.H_q = H_q
         self.p = params or lg_default_params()
         self.policy = policy
@@ -336,7 +348,11 @@ class Guard:
             lg_decode_attend(c, l0, nl, q[l0:l0 + nl], self.H_q, self.scale, self.out[l0:l0 + nl],
                              self.stats[l0:l0 + nl], p.suffix_w, 1 if self.policy == "h2o" else 0,
                              self.max_len, self.ws, stream)
-        if self.policy == "loopguard":
+        if self.policy == "loopguard" and self.fused_prune:
+            lg_detect_prune(c, self.stats, self.H_q, self.state, budget, p, self.flags,
+                            self.spans, self.diag, self.dstate, self.kept_idx, self.kept_count,
+                            self.max_keep, self.max_len, stream)
+        elif self.policy == "loopguard":
             lg_detect(c, self.stats, self.H_q, self.state, budget, p, self.flags, self.spans,
                       self.diag, self.dstate, stream)
             lg_prune_compact(c, self.flags, self.spans, self.state, budget, p, self.kept_idx,

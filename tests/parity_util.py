@@ -40,8 +40,10 @@ def compare_cache(w, ref, cache, lens, what):
             assert np.array_equal(sk[o:o + n], ref.sk[o:o + n]), "%s sketch seq %d" % (what, b)
 
 
-def run_loopguard(w, device, steps=None, n_layers_per_call=None, params=None, check_cache=True):
-    """The guarded decode path of workload w on the GPU and in the oracle, compared each step.
+def run_loopguard(w, device, steps=None, n_layers_per_call=None, params=None, check_cache=True,
+                  fused_prune=True):
+    """The guarded decode path of workload w on the GPU and in the oracle, compared each step
+    (fused_prune: lg_detect_prune, else lg_detect + lg_prune_compact).
     Returns counters of what the run exercised."""
     steps = w.steps if steps is None else steps
     K, V = synth.host_cache(w)
@@ -49,7 +51,8 @@ def run_loopguard(w, device, steps=None, n_layers_per_call=None, params=None, ch
     prm_g = lg.lg_default_params(**(params or {}))
     ref = oracle.OracleGuard(w, K.copy(), V.copy(), prm_o)
     cache = lg.Cache.from_host(w, K, V, device, params=prm_g)
-    guard = lg.Guard(cache, w.H_q, prm_g, n_layers_per_call=n_layers_per_call)
+    guard = lg.Guard(cache, w.H_q, prm_g, n_layers_per_call=n_layers_per_call,
+                     fused_prune=fused_prune)
     seqs = w.seqs.copy()
     pos = w.n0.astype(np.int64)
     rt, ra = OUT_TOL[w.dtype]

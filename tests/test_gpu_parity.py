@@ -37,6 +37,15 @@ def test_per_layer_calls_match(cuda):
     run_loopguard(w, cuda, n_layers_per_call=1)
 
 
+def test_separate_detect_and_prune_calls(cuda):
+    """lg_detect then lg_prune_compact (the retained set in its own kernel) on the workload 2
+    structure: the same results as the fused call"""
+    w = synth.make_workload(2, L=2, batch=4, n=1200, budget=768, steps=40, tail=(300, 500),
+                            periods=(8, 40))
+    c = run_loopguard(w, cuda, fused_prune=False)
+    assert c["triggers"] >= 1 and c["prunes"] >= 4
+
+
 def test_small_model_sinks_gqa6(cuda):
     """workload 3 structure: 12/2 heads (GQA 6), attention sinks x8, loops after 75% of n"""
     w = synth.make_workload(3, L=2, batch=5, n=1500, budget=512, steps=12, periods=(8, 24))
