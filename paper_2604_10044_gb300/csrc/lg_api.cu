@@ -69,7 +69,7 @@ AttendLayout attend_layout(const lg_cache *c, int H_q, int n_layers, int max_len
   L.logits_bytes =
       h2o ? round256((size_t)n_layers * c->H_kv * c->S_total * (H_q / c->H_kv) * sizeof(float))
           : 0;
-  L.counter_bytes = 256;
+  L.counter_bytes = round256((size_t)(1 + (int64_t)n_layers * c->batch * c->H_kv) * sizeof(int));
   L.total = L.partial_bytes + L.final_bytes + L.logits_bytes + L.counter_bytes;
   return L;
 }
@@ -187,6 +187,9 @@ lg_status lg_decode_attend(const lg_cache *c, int layer0, int n_layers, const vo
   float *final_ml = accumulate_h2o ? (float *)((char *)ws + L.partial_bytes) : nullptr;
   a.logits = accumulate_h2o ? (float *)((char *)ws + L.partial_bytes + L.final_bytes) : nullptr;
   a.counter = (int *)((char *)ws + L.partial_bytes + L.final_bytes + L.logits_bytes);
+  a.out = out;
+  a.stats = stats;
+  a.final_ml = final_ml;
   a.S_total = c->S_total;
   a.layer0 = layer0;
   a.n_layers = n_layers;

@@ -78,7 +78,7 @@ attend_partial_kernel(AttendArgs a) {
   const int chunk = blockIdx.x, kvh = blockIdx.y;
   const int b = blockIdx.z % a.batch, lloc = blockIdx.z / a.batch;
   const int layer = a.layer0 + lloc;
-  if (status_bad(a.status)) return;
+  if (cta_status_bad(a.status)) return;
   const int n = a.len[b];
   if (n > a.max_len || n < 0) {
     if (threadIdx.x == 0) set_status(a.status, LG_ERR_CAPACITY);
@@ -382,10 +382,13 @@ static cudaError_t launch_typed(const AttendArgs &a, int64_t rows_total, void *o
     kp<<<grid, C::kThreads, C::kSmem, s>>>(a);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
   }
-  const int64_t heads = (int64_t)a.n_layers * a.batch * a.H_q;
-  attend_combine_kernel<T, D><<<(unsigned)((heads + 7) / 8), 256, 0, s>>>(a, out, stats,
-                                                                          final_ml);
-  if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  if (Elem<T>::kDtype != LG_BF16) {
+    // the tensor-core pass merges its chunk partials itself
+    const int64_t heads = (int64_t)a.n_layers * a.batch * a.H_q;
+    attend_combine_kernel<T, D><<<(unsigned)((heads + 7) / 8), 256, 0, s>>>(a, out, stats,
+                                                                            final_ml);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  }
   if (h2o) {
     int gx = (a.max_len + 255) / 256;
     if (gx > 64) gx = 64;

@@ -1,8 +1,9 @@
 // Decode attention over a bf16 KV cache fused with the guard's per-head statistics (LoopGuard
 // Sec. 3.1, Eq. 1; statistics read by Sec. 5.2), on tensor cores.
 //
-// Persistent CTAs (one per SM) take chunks from a shared counter, each CHUNK consecutive rows
-// of one (layer, sequence, kv-head).  A producer warp streams 128-row K and V tiles into a 3-stage
+// Persistent CTAs (one per SM) take chunks from a shared counter, each a run of consecutive rows
+// of one (layer, sequence, kv-head), sized at launch from the lengths of the call (about eight
+// chunks per CTA).  A producer warp streams 128-row K and V tiles into a 3-stage
 // shared-memory ring with 2-D tensor copies (cp.async.bulk.tensor, 128-byte swizzle, one box
 // per 64 columns) completing on mbarriers.  Each of four consumer warps owns 32 rows of a tile
 // and all g query heads of the kv-head (padded to 8):
@@ -12,9 +13,10 @@
 //                                               P split into bf16 hi + lo (two MMAs)
 // The suffix mass, the entropy term and the normaliser accumulate beside the softmax.  At the
 // end of a chunk the four warps merge through shared memory into one partial per head
-// {M, l, u, sigma, o[d]}; lg_attend.cu merges the chunk partials and emits out and the
-// statistics.  Rows past the end of a sequence (ragged last tile) are masked to zero weight,
-// and their stale V rows are zeroed in shared memory before the P.V product.
+// {M, l, u, sigma, o[d]} and hand the chunk to one of four merger warps, which count the
+// arrivals of each (layer, sequence, kv-head) group; the arrival that completes a group merges
+// the group's chunk partials into out and the statistics while the consumers go on streaming.  Rows past the end of a sequence (ragged last tile) are masked to zero
+// weight, and their stale V rows are zeroed in shared memory before the P.V product.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 #include <cuda_bf16.h>
@@ -32,7 +34,13 @@ namespace {
 constexpr int kTile = 128;          // rows per tile (TMA box height)
 constexpr int kBoxBytes = kTile * 128;  // one box: 128 rows x 64 bf16
 constexpr int kConsumerWarps = 4;
-constexpr int kThreads = (kConsumerWarps + 1) * 32;
+constexpr int kProducerWarp = kConsumerWarps;
+constexpr int kMergerWarp0 = kConsumerWarps + 1;
+constexpr int kMergers = 4;   // merger warps; ticket k goes to merger k % kMergers
+constexpr int kThreads = (kConsumerWarps + 1 + kMergers) * 32;
+constexpr int kTickets = 2 * kMergers;  // finished chunks queued from the consumers to the mergers
+constexpr int kMaxChunkRows = 4096;  // chunk rows at most (the tail of a call is about one chunk)
+constexpr int kStagedSeqs = 256;     // lengths and offsets kept in shared memory up to this batch
 
 template <int D>
 struct MmaCfg {
@@ -41,7 +49,8 @@ struct MmaCfg {
   static constexpr int kStages = D == 128 ? 3 : 6;
   static constexpr int kRingBytes = kStages * kStageBytes;
   static constexpr int kMergeBytes = kConsumerWarps * 8 * D * 4 + kConsumerWarps * 8 * 4 * 4;
-  static constexpr int kSmem = kRingBytes + kMergeBytes + 1024;  // + alignment slack
+  static constexpr int kQBytes = 8 * D * 2;  // a stage's query rows (up to 8 heads), bf16
+  static constexpr int kSmem = kRingBytes + kMergeBytes + kStages * kQBytes + 1024;  // + slack
   static constexpr int kKSteps = D / 16;
 };
 
@@ -97,10 +106,35 @@ struct ChunkId {
   int lloc, b, kvh, ch;
 };
 
-__device__ __forceinline__ ChunkId decode_chunk(const AttendArgs &a, int c) {
+// Chunk geometry of one call, from the lengths it attends over (the host sizes the workspace
+// for max_len, which can be far above them): chunk rows a multiple of the tile, about eight
+// chunks per CTA, and never more chunks per group than the workspace holds (max_chunks).
+struct Geom {
+  int rows;     // rows per chunk
+  int per_grp;  // chunk ids per (layer, sequence, kv-head)
+  int total;    // chunk ids of the call
+};
+
+__device__ __forceinline__ Geom make_geom(const AttendArgs &a, int n_max, int64_t len_sum,
+                                          int ctas) {
+  const int64_t rows_all = len_sum * a.H_kv * a.n_layers;
+  const int64_t target = (int64_t)ctas * 8;
+  int64_t c = (rows_all + target - 1) / target;
+  const int64_t fit = (n_max + a.max_chunks - 1) / a.max_chunks;
+  c = min(c, (int64_t)kMaxChunkRows);
+  c = max(max(c, fit), (int64_t)kTile);
+  c = (c + kTile - 1) / kTile * kTile;
+  Geom gm;
+  gm.rows = (int)c;
+  gm.per_grp = max(1, (int)((n_max + c - 1) / c));
+  gm.total = a.n_layers * a.batch * a.H_kv * gm.per_grp;
+  return gm;
+}
+
+__device__ __forceinline__ ChunkId decode_chunk(const AttendArgs &a, int c, int per_grp) {
   ChunkId id;
-  id.ch = c % a.max_chunks;
-  int r = c / a.max_chunks;
+  id.ch = c % per_grp;
+  int r = c / per_grp;
   id.kvh = r % a.H_kv;
   r /= a.H_kv;
   id.b = r % a.batch;
@@ -108,57 +142,246 @@ __device__ __forceinline__ ChunkId decode_chunk(const AttendArgs &a, int c) {
   return id;
 }
 
+// Split-K merge of one group's chunk partials (all G heads, one warp):
+//   M = max_j M_j, f_j = 2^(M_j - M), l = sum f_j l_j, u = sum f_j (u_j + (M_j - M) l_j),
+//   sigma = sum f_j sigma_j, o = sum f_j o_j / l
+// out = o, stats = {M ln 2, l, ln l - u ln 2 / l, sigma / l}.  The partials were written by
+// other CTAs of this launch: read through L2.  Lane j holds chunk j's {M, l, u, sigma} (up to
+// 32 chunks; more are read again per block), and the o slices of kBlk chunks are loaded with
+// them, so a head of a group of at most kBlk chunks costs one round trip.
+template <int D, int G>
+__device__ __forceinline__ void merge_group(const AttendArgs &a, int64_t head0, int n,
+                                            int chunk_rows, int lane) {
+  constexpr int EPL = D / 32;
+  constexpr int kBlk = 8;
+  const int nch = (n + chunk_rows - 1) / chunk_rows;
+  for (int h = 0; h < G; ++h) {
+    const int64_t head = head0 + h;
+    const float *pp = a.partial + head * a.max_chunks * (D + 8);
+    float ob[kBlk][EPL];
+#pragma unroll
+    for (int jj = 0; jj < kBlk; ++jj)
+#pragma unroll
+      for (int k = 0; k < EPL; ++k)
+        ob[jj][k] = jj < nch ? __ldcg(pp + (int64_t)jj * (D + 8) + 8 + lane + 32 * k) : 0.f;
+    float4 sl = make_float4(-INFINITY, 0.f, 0.f, 0.f);  // this lane's chunk (j = lane)
+    if (lane < nch) sl = __ldcg(reinterpret_cast<const float4 *>(pp + (int64_t)lane * (D + 8)));
+    float M = sl.x;
+    for (int j = lane + 32; j < nch; j += 32) M = fmaxf(M, __ldcg(pp + (int64_t)j * (D + 8)));
+#pragma unroll
+    for (int o = 16; o >= 1; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
+    float l = 0.f, u = 0.f, sg = 0.f, acc[EPL];
+#pragma unroll
+    for (int k = 0; k < EPL; ++k) acc[k] = 0.f;
+    for (int j0 = 0; j0 < nch; j0 += kBlk) {
+      if (j0 > 0) {
+#pragma unroll
+        for (int jj = 0; jj < kBlk; ++jj)
+#pragma unroll
+          for (int k = 0; k < EPL; ++k)
+            ob[jj][k] = j0 + jj < nch
+                            ? __ldcg(pp + (int64_t)(j0 + jj) * (D + 8) + 8 + lane + 32 * k)
+                            : 0.f;
+      }
+      // weights of this block's chunks: lane jj < kBlk takes chunk j0 + jj (held by lane
+      // j0 + jj when that is below 32, read again otherwise)
+      const int j = j0 + lane;
+      float4 sv = make_float4(__shfl_sync(0xffffffffu, sl.x, j & 31),
+                              __shfl_sync(0xffffffffu, sl.y, j & 31),
+                              __shfl_sync(0xffffffffu, sl.z, j & 31),
+                              __shfl_sync(0xffffffffu, sl.w, j & 31));
+      float f = 0.f;
+      if (lane < kBlk && j < nch) {
+        if (j >= 32) sv = __ldcg(reinterpret_cast<const float4 *>(pp + (int64_t)j * (D + 8)));
+        f = exp2f(sv.x - M);
+        l += f * sv.y;
+        u += f * (sv.z + (sv.x - M) * sv.y);
+        sg += f * sv.w;
+      }
+#pragma unroll
+      for (int jj = 0; jj < kBlk; ++jj) {
+        const float fj = __shfl_sync(0xffffffffu, f, jj);
+#pragma unroll
+        for (int k = 0; k < EPL; ++k) acc[k] += fj * ob[jj][k];
+      }
+    }
+#pragma unroll
+    for (int o = 16; o >= 1; o >>= 1) {
+      l += __shfl_xor_sync(0xffffffffu, l, o);
+      u += __shfl_xor_sync(0xffffffffu, u, o);
+      sg += __shfl_xor_sync(0xffffffffu, sg, o);
+    }
+    const float inv_l = 1.f / l;
+    __nv_bfloat16 *out = reinterpret_cast<__nv_bfloat16 *>(a.out) + head * D;
+#pragma unroll
+    for (int k = 0; k < EPL; ++k) out[lane + 32 * k] = __float2bfloat16_rn(acc[k] * inv_l);
+    if (lane == 0) {
+      constexpr float kLn2 = 0.69314718055994530942f;
+      float *st = a.stats + head * 4;
+      st[0] = M * kLn2;
+      st[1] = l;
+      st[2] = logf(l) - u * kLn2 * inv_l;
+      st[3] = sg * inv_l;
+      if (a.final_ml) {
+        a.final_ml[head * 2] = M;
+        a.final_ml[head * 2 + 1] = l;
+      }
+    }
+  }
+}
+
 }  // namespace
 
 template <int D, int G>
 __global__ void __launch_bounds__(kThreads, 1)
 attend_mma_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
-                  AttendArgs a, int total_chunks, int *next_chunk) {
+                  AttendArgs a, int *next_chunk) {
   using C = MmaCfg<D>;
   extern __shared__ unsigned char smem_raw[];
   __shared__ __align__(8) uint64_t full_bar[C::kStages];
   __shared__ __align__(8) uint64_t empty_bar[C::kStages];
   __shared__ int stage_chunk[C::kStages];  // chunk of the tile in each stage, -1: no more work
   __shared__ int stage_tile[C::kStages];   // tile index within that chunk
+  __shared__ int stage_n[C::kStages];      // the chunk's sequence length
+  __shared__ long long stage_lrow0[C::kStages];  // its first row in the logits layout
+  __shared__ __align__(8) uint64_t tfull[kTickets];   // consumer -> merger: a finished chunk
+  __shared__ __align__(8) uint64_t tempty[kTickets];  // merger -> consumer: the slot is free
+  __shared__ int t_grp[kTickets], t_n[kTickets];      // its group (-1: no more) and length
+  __shared__ int red_max[kThreads / 32];
+  __shared__ long long red_sum[kThreads / 32];
+  __shared__ int s_len[kStagedSeqs];         // len[b] and seq_off[b] of a batch up to kStagedSeqs
+  __shared__ long long s_off[kStagedSeqs];
+  __shared__ int s_bad;                      // the device status at entry (one read per CTA)
   unsigned char *smem = reinterpret_cast<unsigned char *>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   float *merge_o = reinterpret_cast<float *>(smem + C::kRingBytes);  // [warps][8][D]
+  unsigned char *qbuf = smem + C::kRingBytes + C::kMergeBytes;         // [stages][8][D] bf16
   float *merge_s = merge_o + kConsumerWarps * 8 * D;                  // [warps][8][4]
 
-  if (status_bad(a.status)) return;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  // the first chunk claim and the length reads below are in flight together
+  int c_first = 0;
+  if (warp == kProducerWarp && lane == 0) c_first = atomicAdd(next_chunk, 1);
   if (threadIdx.x == 0) {
+    s_bad = status_bad(a.status);
     for (int s = 0; s < C::kStages; ++s) {
       mbar_init(&full_bar[s], 1);
       mbar_init(&empty_bar[s], kConsumerWarps);
     }
+    for (int s = 0; s < kTickets; ++s) {
+      mbar_init(&tfull[s], 1);
+      mbar_init(&tempty[s], 1);
+    }
     mbar_fence_init();
   }
+  {
+    // longest and total length of the batch (lengths past max_len count as max_len)
+    int nmx = 0;
+    long long sum = 0;
+    for (int b = threadIdx.x; b < a.batch; b += kThreads) {
+      const int nb = a.len[b];
+      if (b < kStagedSeqs) {
+        s_len[b] = nb;
+        s_off[b] = a.seq_off[b];
+      }
+      const int n = min(nb, a.max_len);
+      nmx = max(nmx, n);
+      sum += n;
+    }
+    nmx = __reduce_max_sync(0xffffffffu, nmx);
+#pragma unroll
+    for (int o = 16; o >= 1; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
+    if (lane == 0) {
+      red_max[warp] = nmx;
+      red_sum[warp] = sum;
+    }
+  }
   __syncthreads();
+  if (s_bad) return;  // the same decision in every thread of the CTA
+  const bool staged = a.batch <= kStagedSeqs;
+  int n_max = 0;
+  long long len_sum = 0;
+#pragma unroll
+  for (int w = 0; w < kThreads / 32; ++w) {
+    n_max = max(n_max, red_max[w]);
+    len_sum += red_sum[w];
+  }
+  const Geom gm = make_geom(a, n_max, len_sum, gridDim.x);
 
-  if (warp == kConsumerWarps) {
+  if (warp >= kMergerWarp0) {
+    // ------------------------------------------------------------ mergers
+    // One ticket per finished chunk, dealt round-robin to the merger warps.  The consumers'
+    // partial stores are ordered before the ticket (their barrier, the mbarrier's release and
+    // acquire); the fence makes them visible to the GPU before the group's arrival count
+    // moves, and the arrival that completes the group (acquire fence after it) reads every
+    // chunk partial of the group.
+    for (uint32_t tk = warp - kMergerWarp0;; tk += kMergers) {
+      const int slot = tk % kTickets;
+      if (!mbar_wait(&tfull[slot], (tk / kTickets) & 1)) {
+        set_status(a.status, LG_ERR_TIMEOUT);
+        return;
+      }
+      const int grp = t_grp[slot], n = t_n[slot];
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&tempty[slot]);
+      if (grp < 0) break;
+      int last = 0;
+      if (lane == 0) {
+        __threadfence();
+        const int nch = (n + gm.rows - 1) / gm.rows;
+        last = atomicAdd(a.counter + 1 + grp, 1) == nch - 1;
+      }
+      last = __shfl_sync(0xffffffffu, last, 0);
+      __syncwarp();
+      if (last) {
+        __threadfence();
+        const int64_t head0 = (int64_t)(grp / a.H_kv) * a.H_q + (int64_t)(grp % a.H_kv) * G;
+        merge_group<D, G>(a, head0, n, gm.rows, lane);
+      }
+    }
+    return;
+  }
+
+  if (warp == kProducerWarp) {
     // ------------------------------------------------------------ producer
-    // Chunks are taken from a shared counter (ragged lengths balance across CTAs); each
-    // stage carries its chunk and tile index to the consumers.
+    // Chunks are taken from a shared counter (ragged lengths balance across CTAs), one claim
+    // ahead so that its round trip overlaps the current chunk; each stage carries its chunk,
+    // tile index, length and logits row to the consumers, and a chunk's first stage also
+    // brings the chunk's query rows (one bulk copy on the same barrier).
     if (lane == 0) {
       asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmK)) : "memory");
       asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmV)) : "memory");
       uint32_t it = 0;
-      bool alive = true;
-      while (alive) {
-        const int c = atomicAdd(next_chunk, 1);
-        int ntiles = 0, grow = 0;
-        if (c < total_chunks) {
-          const ChunkId id = decode_chunk(a, c);
-          const int n = a.len[id.b];
-          const int row0 = id.ch * a.chunk_rows;
+      int c = c_first;
+      while (true) {
+        const bool alive = c < gm.total;
+        int ntiles = 0, grow = 0, n = 0, c_next = 0;
+        int64_t lrow0 = 0, head0 = 0;
+        if (alive) {
+          c_next = atomicAdd(next_chunk, 1);
+          const ChunkId id = decode_chunk(a, c, gm.per_grp);
+          n = staged ? s_len[id.b] : a.len[id.b];
+          const int64_t off = staged ? s_off[id.b] : a.seq_off[id.b];
+          const int row0 = id.ch * gm.rows;
+          head0 = ((int64_t)id.lloc * a.batch + id.b) * a.H_q + (int64_t)id.kvh * G;
           if (n > a.max_len) set_status(a.status, LG_ERR_CAPACITY);
-          if (n > a.max_len || row0 >= n) continue;
-          ntiles = (min(a.chunk_rows, n - row0) + kTile - 1) / kTile;
-          grow = (int)(((int64_t)(a.layer0 + id.lloc) * a.H_kv + id.kvh) * a.S_total +
-                       a.seq_off[id.b] + row0);
-        } else {
-          alive = false;
+          if (n == 0 && id.ch == 0) {
+            // empty sequence: no chunk to merge; zero output, m = -inf, l = H = S = 0
+            __nv_bfloat16 *out = reinterpret_cast<__nv_bfloat16 *>(a.out) + head0 * D;
+            for (int e = 0; e < G * D; ++e) out[e] = __float2bfloat16_rn(0.f);
+            for (int h = 0; h < G; ++h) {
+              a.stats[(head0 + h) * 4] = -INFINITY;
+              a.stats[(head0 + h) * 4 + 1] = a.stats[(head0 + h) * 4 + 2] =
+                  a.stats[(head0 + h) * 4 + 3] = 0.f;
+            }
+          }
+          if (n > a.max_len || row0 >= n) {
+            c = c_next;
+            continue;
+          }
+          ntiles = (min(gm.rows, n - row0) + kTile - 1) / kTile;
+          grow = (int)(((int64_t)(a.layer0 + id.lloc) * a.H_kv + id.kvh) * a.S_total + off + row0);
+          lrow0 = ((int64_t)id.lloc * a.H_kv + id.kvh) * a.S_total + off + row0;
         }
         for (int t = 0; t < (alive ? ntiles : 1); ++t, ++it) {
           const int st = it % C::kStages;
@@ -169,19 +392,27 @@ attend_mma_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant
           }
           stage_chunk[st] = alive ? c : -1;
           stage_tile[st] = t;
+          stage_n[st] = n;
+          stage_lrow0[st] = lrow0;
           if (!alive) {
             mbar_arrive(&full_bar[st]);  // end of work: completes the phase without a copy
             break;
           }
           unsigned char *stage = smem + (size_t)st * C::kStageBytes;
-          mbar_arrive_expect_tx(&full_bar[st], C::kStageBytes);
+          mbar_arrive_expect_tx(&full_bar[st], C::kStageBytes + (t == 0 ? G * D * 2 : 0));
 #pragma unroll
           for (int h = 0; h < C::kHalves; ++h) {
             tma_load_2d(stage + h * kBoxBytes, &tmK, h * 64, grow + t * kTile, &full_bar[st]);
             tma_load_2d(stage + (C::kHalves + h) * kBoxBytes, &tmV, h * 64, grow + t * kTile,
                         &full_bar[st]);
           }
+          if (t == 0)
+            bulk_load(qbuf + st * C::kQBytes,
+                      reinterpret_cast<const __nv_bfloat16 *>(a.q) + head0 * D, G * D * 2,
+                      &full_bar[st]);
         }
+        if (!alive) break;
+        c = c_next;
       }
     }
     return;
@@ -197,6 +428,8 @@ attend_mma_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant
   float o[C::kKSteps][4];
   float m2[2], l2[2], u2[2], sg2[2];
   float *logits = a.logits;
+  uint32_t tk = 0;        // tickets issued (thread 0)
+  bool handoff = true;    // false once a ticket slot was not released in time (thread 0)
   for (uint32_t it = 0;; ++it) {
     const int st = it % C::kStages;
     if (!mbar_wait(&full_bar[st], (it / C::kStages) & 1)) {
@@ -208,17 +441,15 @@ attend_mma_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant
     const int t = stage_tile[st];
     if (t == 0) {
       // first tile of a chunk: its geometry, the q^T fragments, fresh softmax state
-      id = decode_chunk(a, c);
-      n = a.len[id.b];
-      row0 = id.ch * a.chunk_rows;
-      rows = min(a.chunk_rows, n - row0);
+      id = decode_chunk(a, c, gm.per_grp);
+      n = stage_n[st];
+      row0 = id.ch * gm.rows;
+      rows = min(gm.rows, n - row0);
       ntiles = (rows + kTile - 1) / kTile;
       suffix_lo = n - min(a.suffix_w, n);
-      lrow0 = ((int64_t)id.lloc * a.H_kv + id.kvh) * a.S_total + a.seq_off[id.b] + row0;
+      lrow0 = stage_lrow0[st];
       // B fragments of q^T: head g (zero for padded heads), d = 16 ks + 2 t4 (+1, +8, +9)
-      const int64_t qh = ((int64_t)id.lloc * a.batch + id.b) * a.H_q + (int64_t)id.kvh * G + g;
-      const uint32_t *qp = reinterpret_cast<const uint32_t *>(
-          reinterpret_cast<const __nv_bfloat16 *>(a.q) + qh * D);
+      const uint32_t *qp = reinterpret_cast<const uint32_t *>(qbuf + st * C::kQBytes) + g * (D / 2);
 #pragma unroll
       for (int ks = 0; ks < C::kKSteps; ++ks) {
         qf[ks][0] = g < G ? qp[ks * 8 + t4] : 0u;
@@ -410,7 +641,33 @@ attend_mma_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant
         pp[3] = sg;
       }
     }
+    // every partial store of the chunk is done: hand the chunk to the merger warp
     asm volatile("bar.sync 1, %0;" ::"n"(kConsumerWarps * 32) : "memory");
+    if (threadIdx.x == 0 && handoff) {
+      const int slot = tk % kTickets;
+      if (tk >= (uint32_t)kTickets && !mbar_wait(&tempty[slot], ((tk / kTickets) - 1) & 1)) {
+        set_status(a.status, LG_ERR_TIMEOUT);
+        handoff = false;
+      } else {
+        t_grp[slot] = (int)(((int64_t)id.lloc * a.batch + id.b) * a.H_kv + id.kvh);
+        t_n[slot] = n;
+        mbar_arrive(&tfull[slot]);
+        ++tk;
+      }
+    }
+  }
+  if (threadIdx.x == 0 && handoff) {
+    // no more chunks: one last ticket for each merger
+    for (int m = 0; m < kMergers; ++m, ++tk) {
+      const int slot = tk % kTickets;
+      if (tk >= (uint32_t)kTickets && !mbar_wait(&tempty[slot], ((tk / kTickets) - 1) & 1)) {
+        set_status(a.status, LG_ERR_TIMEOUT);
+        break;
+      }
+      t_grp[slot] = -1;
+      t_n[slot] = 0;
+      mbar_arrive(&tfull[slot]);
+    }
   }
 }
 
@@ -446,27 +703,27 @@ bool make_map(CUtensorMap *m, const void *base, int d, int64_t rows) {
 
 template <int D, int G>
 cudaError_t launch_mma_typed(const CUtensorMap &mk, const CUtensorMap &mv, const AttendArgs &a,
-                             int total, int grid, int *counter, cudaStream_t s) {
+                             int grid, int *counter, cudaStream_t s) {
   auto kern = attend_mma_kernel<D, G>;
   cudaError_t e =
       cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, MmaCfg<D>::kSmem);
   if (e != cudaSuccess) return e;
-  kern<<<grid, kThreads, MmaCfg<D>::kSmem, s>>>(mk, mv, a, total, counter);
+  kern<<<grid, kThreads, MmaCfg<D>::kSmem, s>>>(mk, mv, a, counter);
   return cudaGetLastError();
 }
 
 template <int D>
 cudaError_t launch_mma_d(const CUtensorMap &mk, const CUtensorMap &mv, const AttendArgs &a, int g,
-                         int total, int grid, int *counter, cudaStream_t s) {
+                         int grid, int *counter, cudaStream_t s) {
   switch (g) {
-    case 1: return launch_mma_typed<D, 1>(mk, mv, a, total, grid, counter, s);
-    case 2: return launch_mma_typed<D, 2>(mk, mv, a, total, grid, counter, s);
-    case 3: return launch_mma_typed<D, 3>(mk, mv, a, total, grid, counter, s);
-    case 4: return launch_mma_typed<D, 4>(mk, mv, a, total, grid, counter, s);
-    case 5: return launch_mma_typed<D, 5>(mk, mv, a, total, grid, counter, s);
-    case 6: return launch_mma_typed<D, 6>(mk, mv, a, total, grid, counter, s);
-    case 7: return launch_mma_typed<D, 7>(mk, mv, a, total, grid, counter, s);
-    case 8: return launch_mma_typed<D, 8>(mk, mv, a, total, grid, counter, s);
+    case 1: return launch_mma_typed<D, 1>(mk, mv, a, grid, counter, s);
+    case 2: return launch_mma_typed<D, 2>(mk, mv, a, grid, counter, s);
+    case 3: return launch_mma_typed<D, 3>(mk, mv, a, grid, counter, s);
+    case 4: return launch_mma_typed<D, 4>(mk, mv, a, grid, counter, s);
+    case 5: return launch_mma_typed<D, 5>(mk, mv, a, grid, counter, s);
+    case 6: return launch_mma_typed<D, 6>(mk, mv, a, grid, counter, s);
+    case 7: return launch_mma_typed<D, 7>(mk, mv, a, grid, counter, s);
+    case 8: return launch_mma_typed<D, 8>(mk, mv, a, grid, counter, s);
   }
   return cudaErrorInvalidValue;
 }
@@ -484,12 +741,14 @@ cudaError_t launch_attend_mma_partial(const AttendArgs &a, int d, int g, int64_t
   cudaError_t e = cudaGetDevice(&dev);
   if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   if (e != cudaSuccess) return e;
+  // an upper bound of the chunk ids (the kernel sizes its chunks from the lengths it reads)
   const int total = a.n_layers * a.batch * a.H_kv * a.max_chunks;
   const int grid = total < sms ? total : sms;
   if (!a.counter) return cudaErrorInvalidValue;
-  if ((e = cudaMemsetAsync(a.counter, 0, sizeof(int), s)) != cudaSuccess) return e;
-  if (d == 128) return launch_mma_d<128>(mk, mv, a, g, total, grid, a.counter, s);
-  if (d == 64) return launch_mma_d<64>(mk, mv, a, g, total, grid, a.counter, s);
+  const size_t counters = (size_t)(1 + (int64_t)a.n_layers * a.batch * a.H_kv) * sizeof(int);
+  if ((e = cudaMemsetAsync(a.counter, 0, counters, s)) != cudaSuccess) return e;
+  if (d == 128) return launch_mma_d<128>(mk, mv, a, g, grid, a.counter, s);
+  if (d == 64) return launch_mma_d<64>(mk, mv, a, g, grid, a.counter, s);
   return cudaErrorInvalidValue;
 }
 

@@ -20,6 +20,16 @@ __device__ __forceinline__ bool status_bad(const int32_t *status) {
   return status && *(volatile const int32_t *)status != 0;
 }
 
+// The device status as one decision for the whole CTA: thread 0 reads it and a barrier hands it
+// to every thread, so that a status another CTA sets meanwhile cannot split the CTA between an
+// early return and a later barrier.  Every thread of the CTA calls it.
+__device__ __forceinline__ bool cta_status_bad(const int32_t *status) {
+  __shared__ int s_status_bad;
+  if (threadIdx.x == 0) s_status_bad = status_bad(status);
+  __syncthreads();
+  return s_status_bad != 0;
+}
+
 __device__ __forceinline__ uint64_t global_ns() {
   uint64_t t;
   asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));

@@ -310,7 +310,7 @@ __global__ void __launch_bounds__(kDetectThreads, 1) detect_kernel(DetectArgs a)
     st_a = reinterpret_cast<const int4 *>(a.state + b)[0];
     st_b = reinterpret_cast<const int4 *>(a.state + b)[1];
   }
-  if (status_bad(status)) return;
+  if (cta_status_bad(status)) return;
   const int nw = a.nwords, thr = a.thr, stride = nw + 1;
   const uint32_t *sk_g = a.c.sketch + off * nw;
   const int w = min(p.W, n);
@@ -640,7 +640,7 @@ __global__ void __launch_bounds__(kCompactThreads) compact_kernel(lg_cache c,
                                                                   const int32_t *kept_count,
                                                                   int max_keep) {
   const int tid = threadIdx.x;
-  if (status_bad(c.dev_status)) return;
+  if (cta_status_bad(c.dev_status)) return;
   const int row_bytes_kv = c.d * (c.dtype == LG_BF16 ? 2 : 4);
   const int nwords = c.H_kv * c.d / 32;
   const int n_kv = 2 * c.L * c.H_kv;
@@ -742,7 +742,7 @@ __global__ void __launch_bounds__(kH2OThreads) evict_kernel(lg_cache c, const in
   __shared__ unsigned long long s_prefix;
   __shared__ int s_remaining;
   const int lh = blockIdx.x, b = blockIdx.y, tid = threadIdx.x;
-  if (status_bad(c.dev_status)) return;
+  if (cta_status_bad(c.dev_status)) return;
   const int n = c.len[b], B = budget[b];
   if (n <= B) return;
   if (n > max_len) {

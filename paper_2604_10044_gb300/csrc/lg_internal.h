@@ -15,7 +15,11 @@ struct AttendArgs {
   int32_t *status;
   float *partial;          // [n_layers][batch][H_q][max_chunks][d + 8]
   float *logits;           // nullable [n_layers][H_kv][S_total][g], log2 units
-  int *counter;            // work counter of the persistent tensor-core pass (bf16)
+  int *counter;            // [1 + n_layers * batch * H_kv], zeroed by each call (bf16 pass):
+                           // the chunk counter, then chunks done per (layer, sequence, kv-head)
+  void *out;               // [n_layers][batch][H_q][d] dtype
+  float *stats;            // [n_layers][batch][H_q][4]
+  float *final_ml;         // nullable [n_layers][batch][H_q][2]: merged (M, l), log2 units
   int64_t S_total;
   int layer0, n_layers, batch, H_kv, H_q;
   int chunk_rows;          // rows per CTA, a multiple of the tile
