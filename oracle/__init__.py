@@ -51,6 +51,31 @@ DEFAULTS = dict(W=256, K=2, t_min=64, cooldown=32, n_anchor=32, stall_len=4, p_m
 NEVER_TRIGGERED = -(1 << 30)
 
 
+class TokenParams(ctypes.Structure):
+    _fields_ = [("cr_every", ctypes.c_int32), ("theta_streak", ctypes.c_int32),
+                ("hist", ctypes.c_int32), ("pad", ctypes.c_int32),
+                ("theta_cr", ctypes.c_double), ("theta_conf", ctypes.c_double)]
+
+
+class TokenState(ctypes.Structure):
+    _fields_ = [("streak", ctypes.c_int32), ("synced", ctypes.c_int32),
+                ("appended", ctypes.c_int32), ("pad", ctypes.c_int32), ("cr", ctypes.c_double)]
+
+
+# App. B.2 thresholds of the token-level monitor; cr_every and hist are the build's readings.
+TOKEN_DEFAULTS = dict(cr_every=16, theta_streak=6, hist=512, theta_cr=0.12, theta_conf=0.9)
+
+
+def token_params(**over) -> TokenParams:
+    d = dict(TOKEN_DEFAULTS)
+    d.update(over)
+    return TokenParams(**d)
+
+
+def new_token_state() -> TokenState:
+    return TokenState(streak=0, synced=-1, appended=0, pad=0, cr=1.0)
+
+
 def params(**over) -> Params:
     d = dict(DEFAULTS)
     d.update(over)
@@ -94,6 +119,10 @@ def lib():
         L.lgref_h2o_argmin.argtypes = [i32, vp, vp, i32, ctypes.c_int32]
         L.lgref_streaming_select.argtypes = [i32, vp, i32, i32, ctypes.c_int32, vp]
         L.lgref_streaming_oldest.argtypes = [i32, vp, i32]
+        L.lgref_lz77_phrases.argtypes = [vp, i32]
+        L.lgref_token_detect.argtypes = [vp, i32, dbl, i32, i32, ctypes.POINTER(Params),
+                                         ctypes.POINTER(TokenParams), ctypes.POINTER(State),
+                                         ctypes.POINTER(TokenState), vp, vp, vp]
         _lib = L
     return _lib
 
@@ -160,6 +189,32 @@ def detect(stats, sketches, budget, prm: Params, st: State):
         raise ValueError("lgref_detect rejected its arguments")
     keys = ("ebar", "lbar", "ttr", "sig1", "sig2", "sig3", "warn", "stall", "P", "trigger")
     return int(flag[0]), (int(span[0]), int(span[1])), dict(zip(keys, diag.tolist()))
+
+
+def lz77_phrases(x) -> int:
+    """phrases of the greedy LZ77 parse of a token sequence (Sec. 4.2's comp, read as LZ77)"""
+    x = np.ascontiguousarray(x, dtype=np.int32)
+    return int(lib().lgref_lz77_phrases(_p(x), x.size))
+
+
+TOKEN_DIAG_KEYS = ("ttr", "cr", "streak", "sig1", "sig2", "sig3", "warn", "stall", "P", "trigger")
+
+
+def token_detect(tokens, pmax, n, budget, prm: Params, tp: TokenParams, st: State,
+                 ts: TokenState):
+    """Token-level monitor for one sequence and one step: tokens = every generated token so far
+    (the last is this step's), pmax this step's top-1 probability, n the cache length after the
+    step's append.  Returns (flag, (lo, hi) in cache slots, diag dict); st, ts updated."""
+    y = np.ascontiguousarray(tokens, dtype=np.int32)
+    flag = np.zeros(1, dtype=np.int32)
+    span = np.zeros(2, dtype=np.int32)
+    diag = np.zeros(10)
+    rc = lib().lgref_token_detect(_p(y), y.size, float(pmax), int(n), int(budget),
+                                  ctypes.byref(prm), ctypes.byref(tp), ctypes.byref(st),
+                                  ctypes.byref(ts), _p(flag), _p(span), _p(diag))
+    if rc:
+        raise ValueError("lgref_token_detect rejected its arguments")
+    return int(flag[0]), (int(span[0]), int(span[1])), dict(zip(TOKEN_DIAG_KEYS, diag.tolist()))
 
 
 def keep_set(n, budget, flag, span, level, prm: Params) -> np.ndarray:

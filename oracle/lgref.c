@@ -16,6 +16,7 @@
  *   progressive aggressiveness, gather ....... Sec. 5.3
  *   H2O comparator (cited, not defined) ...... Sec. 2.2, Sec. 6.1
  *   StreamingLLM comparator (cited) .......... Sec. 2.2, Sec. 6.1
+ *   token-level monitor (TTR, CR, p_max) ..... Sec. 4.2, Sec. 5.2, Eq. 8, Eq. 9, App. B.2
  *
  * The paper's detector reads generated token ids and top-1 probabilities; the
  * decode path carries only K/V caches and attention, so each signal is
@@ -421,4 +422,118 @@ int lgref_streaming_oldest(int n, const int32_t *pos, int n_sink) {
     if (best < 0 || pos[i] < pos[best]) best = i;
   }
   return best;
+}
+
+/* ---------------------------------------------------------------- token-level monitor */
+
+int lgref_lz77_phrases(const int32_t *x, int w) {
+  int phrases = 0;
+  for (int i = 0; i < w;) {
+    int best = 0;
+    for (int j = 0; j < i; ++j) {
+      int k = 0;
+      while (i + k < w && x[j + k] == x[i + k]) ++k;
+      if (k > best) best = k;
+    }
+    ++phrases;
+    i += best >= 2 ? best : 1;
+  }
+  return phrases;
+}
+
+int lgref_token_detect(const int32_t *tokens, int T, double pmax, int n, int budget,
+                       const lgref_params *p, const lgref_token_params *tp, lgref_state *st,
+                       lgref_token_state *ts, int32_t *flag, int32_t *span, double *diag) {
+  if (T < 1 || n < 1 || !p || !tp || !st || !ts || tp->cr_every < 1) return -1;
+  const int32_t *y = tokens;
+  const int t = T - 1; /* this step's token */
+
+  /* cache rows that are consecutive generated tokens: one more after an append, else only
+     this step's row (the cache changed otherwise since the previous step) */
+  ts->appended = (ts->synced >= 0 && n == ts->synced + 1) ? ts->appended + 1 : 1;
+  if (ts->appended > n) ts->appended = n;
+  ts->synced = n;
+
+  /* the window W_t: the last min(W, T) generated tokens */
+  const int w = p->W < T ? p->W : T;
+  const int lo = T - w;
+  /* diversity (TTR): distinct tokens of the window over its length; a token is novel when no
+     earlier token of the window equals it */
+  int n_distinct = 0, novel_tail = 0;
+  for (int i = lo; i < T; ++i) {
+    int novel = 1;
+    for (int j = lo; j < i && novel; ++j) novel = y[j] != y[i];
+    n_distinct += novel;
+    if (i >= T - p->stall_len) novel_tail += novel;
+  }
+  const double ttr = (double)n_distinct / (double)w;
+  /* redundancy (CR): LZ77 phrases of the window over its length, evaluated every cr_every
+     tokens and held in between */
+  if (t % tp->cr_every == 0) ts->cr = (double)lgref_lz77_phrases(y + lo, w) / (double)w;
+  /* confidence collapse: consecutive steps with p_max above theta_conf */
+  ts->streak = pmax > tp->theta_conf ? ts->streak + 1 : 0;
+  /* novelty stagnation: novel fraction of the last theta_stall tokens below theta_nov */
+  int stall = 0;
+  if (w >= p->stall_len && p->stall_len > 0)
+    stall = (double)novel_tail / (double)p->stall_len < p->theta_nov;
+  /* suffix self-alignment: smallest period P whose last max(m_rep P, l_min) tokens each equal
+     the token P earlier */
+  int tailrep = 0, Pstar = 0;
+  for (int P = p->p_min; P <= p->p_max && !tailrep; ++P) {
+    int span_len = p->m_rep * P > p->l_min ? p->m_rep * P : p->l_min;
+    if (T < span_len + P) continue;
+    int all = 1;
+    for (int i = T - span_len; i < T && all; ++i) all = y[i] == y[i - P];
+    if (all) {
+      tailrep = 1;
+      Pstar = P;
+    }
+  }
+  const int sig1 = ttr < p->theta_ttr;
+  const int sig2 = ts->cr < tp->theta_cr;
+  const int sig3 = ts->streak >= tp->theta_streak;
+  const int warn = sig1 + sig2 + sig3 >= p->K;
+  const int trigger = st->t_gen >= p->t_min && st->cd == 0 && warn && (stall || tailrep);
+
+  span[0] = 0;
+  span[1] = 0;
+  if (trigger && tailrep) {
+    /* the repetitive tail in generated tokens: the verified run extended back while tokens
+       keep equalling the token P* earlier (within the kept history), plus its first period;
+       mapped onto the trailing cache rows that hold consecutive generated tokens */
+    int span_len = p->m_rep * Pstar > p->l_min ? p->m_rep * Pstar : p->l_min;
+    int lim = T - tp->hist > 0 ? T - tp->hist : 0;
+    int s = T - span_len;
+    while (s - 1 - Pstar >= lim && y[s - 1] == y[s - 1 - Pstar]) --s;
+    int bad = T - (s - Pstar);
+    if (bad > ts->appended) bad = ts->appended;
+    span[0] = n - bad;
+    span[1] = n;
+  }
+  *flag = trigger;
+
+  if (trigger) {
+    int quick = st->t_gen - st->last_trig <= p->retrig_window;
+    st->level = quick ? (st->level + 1 < p->level_max ? st->level + 1 : p->level_max) : 0;
+    st->last_trig = st->t_gen;
+    st->cd = p->cooldown;
+    st->n_int += 1;
+  } else if (st->cd > 0) {
+    st->cd -= 1;
+  }
+  st->t_gen += 1;
+
+  if (diag) {
+    diag[0] = ttr;
+    diag[1] = ts->cr;
+    diag[2] = ts->streak;
+    diag[3] = sig1;
+    diag[4] = sig2;
+    diag[5] = sig3;
+    diag[6] = warn;
+    diag[7] = stall;
+    diag[8] = tailrep ? Pstar : 0;
+    diag[9] = trigger;
+  }
+  return 0;
 }

@@ -115,6 +115,39 @@ int lgref_streaming_select(int n, const int32_t *pos, int budget, int n_sink, in
 /* StreamingLLM comparator, one row over budget: the slot of the oldest position >= n_sink. */
 int lgref_streaming_oldest(int n, const int32_t *pos, int n_sink);
 
+/* ---- token-level monitor (Sec. 5.2, Eq. 8, Eq. 9, App. B.2) on generated token ids ---- */
+
+typedef struct {
+  int32_t cr_every;      /* the compression ratio is evaluated every cr_every tokens      */
+  int32_t theta_streak;  /* confidence-collapse streak, steps (App. B.2: 6)                */
+  int32_t hist;          /* generated tokens the span extension may reach back over        */
+  int32_t pad;
+  double theta_cr;       /* redundancy threshold (App. B.2: 0.12)                           */
+  double theta_conf;     /* top-1 probability threshold (App. B.2: 0.9)                     */
+} lgref_token_params;
+
+typedef struct {
+  int32_t streak;        /* consecutive steps with p_max > theta_conf                       */
+  int32_t synced;        /* cache length seen by the previous step (-1 before the first)    */
+  int32_t appended;      /* trailing cache rows that are consecutive generated tokens       */
+  int32_t pad;
+  double cr;             /* the last evaluated compression ratio                            */
+} lgref_token_state;
+
+/* Phrases of the greedy LZ77 parse of x[0..w): at each position the longest earlier match
+   (overlap allowed, up to the end) becomes one phrase when it covers at least 2 tokens, else
+   the token is one literal phrase. */
+int lgref_lz77_phrases(const int32_t *x, int w);
+
+/* One decode step of the token-level monitor.  tokens[0..T) are every generated token so far
+   (tokens[T-1] is this step's), pmax this step's top-1 probability, n the cache length after
+   this step's append.  Writes the trigger flag and the span [lo, hi) of cache slots (empty
+   [0,0) without a tail period) and updates the guard and monitor state.  diag nullable [10]:
+   {ttr, cr, streak, vote1, vote2, vote3, warn, stall, P*, trigger}. */
+int lgref_token_detect(const int32_t *tokens, int T, double pmax, int n, int budget,
+                       const lgref_params *p, const lgref_token_params *tp, lgref_state *st,
+                       lgref_token_state *ts, int32_t *flag, int32_t *span, double *diag);
+
 #ifdef __cplusplus
 }
 #endif
