@@ -185,7 +185,8 @@ LG_API lg_status lg_decode_attend(const lg_cache *c, int layer0, int n_layers, c
    On a trigger with TailRep the span [lo, hi) of I_bad covers every copy of the period
    extended back while rows keep matching, clipped to W^recent = [n - budget/2, n).
    stats: device [L][batch][H_q][4], 16-byte aligned (lg_decode_attend's output for all
-   layers); state: device [batch]; budget: device [batch]; flags: device [batch] (1 = trigger);
+   layers); state: device [batch], 16-byte aligned; budget: device [batch]; flags: device
+   [batch] (1 = trigger);
    spans: device [batch][2] ([0,0) when empty).
    diag: nullable device [batch][8] fp64, per sequence {mean normalised entropy, mean suffix
    lift, novel fraction, vote 1, vote 2, vote 3, Stall, P* (0 = no tail repetition)}.
@@ -197,6 +198,55 @@ LG_API lg_status lg_decode_attend(const lg_cache *c, int layer0, int n_layers, c
 LG_API lg_status lg_detect(const lg_cache *c, const float *stats, int H_q, lg_guard_state *state,
                            const int32_t *budget, const lg_guard_params *p, int32_t *flags,
                            int32_t *spans, double *diag, void *dstate, cudaStream_t s);
+
+/* Parameters of the token-level monitor (lg_token_detect). */
+typedef struct {
+  int32_t cr_every;      /* the compression ratio is evaluated every cr_every tokens      */
+  int32_t theta_streak;  /* confidence-collapse streak, steps (App. B.2: 6)                */
+  int32_t hist;          /* generated tokens kept per sequence (>= W and >= p_max +
+                            max(m_rep p_max, l_min)); the span reaches back at most as far */
+  int32_t pad;
+  double theta_cr;       /* redundancy threshold (App. B.2: 0.12)                           */
+  double theta_conf;     /* top-1 probability threshold (App. B.2: 0.9)                     */
+} lg_token_params;
+
+/* Fills *tp with the defaults: cr_every 16, theta_streak 6, hist 512, theta_cr 0.12,
+   theta_conf 0.9. */
+LG_API lg_status lg_default_token_params(lg_token_params *tp);
+
+/* Bytes of lg_token_detect's tstate: batch times (16 + 2 hist + p_max - p_min + 1) 32-bit
+   words rounded up to a multiple of 4; 0 on invalid arguments. */
+LG_API size_t lg_token_state_size(const lg_cache *c, const lg_guard_params *p,
+                                  const lg_token_params *tp);
+
+/* Token-level loop-onset monitor (Sec. 5.2, Eq. 8, Eq. 9, App. B.2; indicators of Sec. 4.2),
+   one step per call, for callers that have the generated token ids and top-1 probabilities:
+     window W_t = the last min(W, t) generated tokens; a token of W_t is novel when no earlier
+       token of W_t equals it;
+     vote 1: novel tokens / |W_t| (TTR) < theta_ttr;
+     vote 2: greedy LZ77 phrases of W_t / |W_t| (CR; a phrase is the longest earlier match of
+       >= 2 tokens, overlap allowed, else one literal token), evaluated every cr_every tokens
+       and held in between, < theta_cr;
+     vote 3: consecutive steps with p_max > theta_conf >= theta_streak;
+     Stall: novel fraction of the last stall_len tokens < theta_nov;
+     TailRep: smallest P in [p_min, p_max] whose last max(m_rep P, l_min) tokens each equal
+       the token P earlier (P*);
+     Trigger = t_gen >= t_min and cd = 0 and votes >= K and (Stall or TailRep).
+   On a trigger with TailRep the span [lo, hi) covers the verified run extended back while
+   tokens keep equalling the token P* earlier (at most hist tokens back) plus its first period,
+   mapped onto the trailing cache rows appended one per step since the cache last changed
+   otherwise (hi = len[b]).  The span is not clipped here: lg_prune_compact, which takes
+   flags, spans and state as from lg_detect, clips it to W^recent.
+   tokens: device [batch] int32, this step's generated token; pmax: device [batch] fp32.
+   state (16-byte aligned), flags, spans as for lg_detect; diag: nullable device [batch][8]
+   fp64 {TTR, CR, streak, vote 1, vote 2, vote 3, Stall, P* (0 = none)}.
+   tstate: device, lg_token_state_size bytes, 8-byte aligned, zero-filled before the first
+   call.  Call it once per decode step after the step's append (len[b] counts this step's
+   row). */
+LG_API lg_status lg_token_detect(const lg_cache *c, const int32_t *tokens, const float *pmax,
+                                 lg_guard_state *state, const lg_guard_params *p,
+                                 const lg_token_params *tp, int32_t *flags, int32_t *spans,
+                                 double *diag, void *tstate, cudaStream_t s);
 
 /* Bytes of lg_detect's dstate: (batch * (p_max - p_min + 3) + S_total) 32-bit words. */
 LG_API size_t lg_detect_state_size(const lg_cache *c, const lg_guard_params *p);

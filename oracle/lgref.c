@@ -441,8 +441,8 @@ int lgref_lz77_phrases(const int32_t *x, int w) {
   return phrases;
 }
 
-int lgref_token_detect(const int32_t *tokens, int T, double pmax, int n, int budget,
-                       const lgref_params *p, const lgref_token_params *tp, lgref_state *st,
+int lgref_token_detect(const int32_t *tokens, int T, double pmax, int n, const lgref_params *p,
+                       const lgref_token_params *tp, lgref_state *st,
                        lgref_token_state *ts, int32_t *flag, int32_t *span, double *diag) {
   if (T < 1 || n < 1 || !p || !tp || !st || !ts || tp->cr_every < 1) return -1;
   const int32_t *y = tokens;

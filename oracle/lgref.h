@@ -144,8 +144,8 @@ int lgref_lz77_phrases(const int32_t *x, int w);
    this step's append.  Writes the trigger flag and the span [lo, hi) of cache slots (empty
    [0,0) without a tail period) and updates the guard and monitor state.  diag nullable [10]:
    {ttr, cr, streak, vote1, vote2, vote3, warn, stall, P*, trigger}. */
-int lgref_token_detect(const int32_t *tokens, int T, double pmax, int n, int budget,
-                       const lgref_params *p, const lgref_token_params *tp, lgref_state *st,
+int lgref_token_detect(const int32_t *tokens, int T, double pmax, int n, const lgref_params *p,
+                       const lgref_token_params *tp, lgref_state *st,
                        lgref_token_state *ts, int32_t *flag, int32_t *span, double *diag);
 
 #ifdef __cplusplus

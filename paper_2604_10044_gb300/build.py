@@ -11,7 +11,8 @@ ROOT = os.path.dirname(_HERE)
 CSRC = os.path.join(_HERE, "csrc")
 BUILD = os.path.join(_HERE, "_build")
 LIB = os.path.join(_HERE, "liblg.so")
-SOURCES = ["lg_attend.cu", "lg_attend_mma.cu", "lg_guard.cu", "lg_api.cu", "lg_noalloc.cu"]
+SOURCES = ["lg_attend.cu", "lg_attend_mma.cu", "lg_guard.cu", "lg_token.cu", "lg_api.cu",
+           "lg_noalloc.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC,-fvisibility=hidden",
          "-I" + os.path.join(ROOT, "include"), "-I" + CSRC]

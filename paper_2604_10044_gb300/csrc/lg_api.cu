@@ -35,6 +35,19 @@ lg_status check_params(const lg_guard_params *p) {
 
 lg_status cuda_status(cudaError_t e) { return e == cudaSuccess ? LG_OK : LG_ERR_CUDA; }
 
+// the token monitor's history must hold the window and every period test's reads
+lg_status check_token_params(const lg_guard_params *p, const lg_token_params *tp) {
+  if (!tp) return LG_ERR_INVALID_ARG;
+  if (tp->cr_every < 1 || tp->theta_streak < 0 || !(tp->theta_cr >= 0.0) ||
+      !(tp->theta_conf >= 0.0))
+    return LG_ERR_INVALID_ARG;
+  const int64_t tail = p->m_rep * (int64_t)p->p_max > p->l_min ? p->m_rep * (int64_t)p->p_max
+                                                               : (int64_t)p->l_min;
+  if (tp->hist < p->W || tp->hist < p->p_max + tail || tp->hist > 8192 || p->W > 4096)
+    return LG_ERR_UNSUPPORTED;
+  return LG_OK;
+}
+
 // rows per chunk (one work item: one CTA of the fp32 path, one loop trip of a persistent CTA
 // of the bf16 path): a multiple of the staging tile, about eight chunks per SM of a 152-SM
 // GB300 for the bf16 path and twelve CTAs per SM for the fp32 path, at most 4096 rows
@@ -215,7 +228,8 @@ lg_status lg_detect(const lg_cache *c, const float *stats, int H_q, lg_guard_sta
   if ((st = check_params(p)) != LG_OK) return st;
   if (!c->sketch || !stats || !state || !budget || !flags || !spans || !dstate)
     return LG_ERR_INVALID_ARG;
-  if (((uintptr_t)dstate & 3u) || ((uintptr_t)stats & 15u)) return LG_ERR_INVALID_ARG;
+  if (((uintptr_t)dstate & 3u) || ((uintptr_t)stats & 15u) || ((uintptr_t)state & 15u))
+    return LG_ERR_INVALID_ARG;
   if (H_q < 1 || H_q % c->H_kv) return LG_ERR_INVALID_ARG;
   if (lg::detect_smem_bytes(*p, c->H_kv * c->d / 32) > 200 * 1024) return LG_ERR_UNSUPPORTED;
   return cuda_status(lg::launch_detect(*c, stats, H_q, state, budget, *p, flags, spans, diag,
@@ -232,13 +246,46 @@ lg_status lg_detect_prune(const lg_cache *c, const float *stats, int H_q, lg_gua
   if (!c->sketch || !stats || !state || !budget || !flags || !spans || !dstate)
     return LG_ERR_INVALID_ARG;
   if (!kept_idx || !kept_count || max_keep < 1 || max_len < 0) return LG_ERR_INVALID_ARG;
-  if (((uintptr_t)dstate & 3u) || ((uintptr_t)stats & 15u)) return LG_ERR_INVALID_ARG;
+  if (((uintptr_t)dstate & 3u) || ((uintptr_t)stats & 15u) || ((uintptr_t)state & 15u))
+    return LG_ERR_INVALID_ARG;
   if (H_q < 1 || H_q % c->H_kv) return LG_ERR_INVALID_ARG;
   if (lg::detect_smem_bytes(*p, c->H_kv * c->d / 32) > 200 * 1024) return LG_ERR_UNSUPPORTED;
   st = cuda_status(lg::launch_detect(*c, stats, H_q, state, budget, *p, flags, spans, diag,
                                      dstate, kept_idx, kept_count, max_keep, max_len, s));
   if (st != LG_OK) return st;
   return cuda_status(lg::launch_compact(*c, kept_idx, kept_count, max_keep, s));
+}
+
+lg_status lg_default_token_params(lg_token_params *tp) {
+  if (!tp) return LG_ERR_INVALID_ARG;
+  memset(tp, 0, sizeof(*tp));
+  tp->cr_every = 16;
+  tp->theta_streak = 6;    // App. B.2
+  tp->hist = 512;
+  tp->theta_cr = 0.12;     // App. B.2
+  tp->theta_conf = 0.9;    // App. B.2
+  return LG_OK;
+}
+
+size_t lg_token_state_size(const lg_cache *c, const lg_guard_params *p,
+                           const lg_token_params *tp) {
+  if (check_cache(c) != LG_OK || check_params(p) != LG_OK || check_token_params(p, tp) != LG_OK)
+    return 0;
+  return (size_t)c->batch * lg::token_state_words(*p, *tp) * sizeof(int32_t);
+}
+
+lg_status lg_token_detect(const lg_cache *c, const int32_t *tokens, const float *pmax,
+                          lg_guard_state *state, const lg_guard_params *p,
+                          const lg_token_params *tp, int32_t *flags, int32_t *spans, double *diag,
+                          void *tstate, cudaStream_t s) {
+  lg_status st = check_cache(c);
+  if (st != LG_OK) return st;
+  if ((st = check_params(p)) != LG_OK) return st;
+  if ((st = check_token_params(p, tp)) != LG_OK) return st;
+  if (!tokens || !pmax || !state || !flags || !spans || !tstate) return LG_ERR_INVALID_ARG;
+  if (((uintptr_t)state & 15u) || ((uintptr_t)tstate & 7u)) return LG_ERR_INVALID_ARG;
+  return cuda_status(lg::launch_token_detect(*c, tokens, pmax, state, *p, *tp, flags, spans,
+                                             diag, tstate, s));
 }
 
 size_t lg_detect_state_size(const lg_cache *c, const lg_guard_params *p) {

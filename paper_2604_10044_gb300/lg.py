@@ -45,6 +45,12 @@ class LgGuardParams(ctypes.Structure):
                                          "tau_ham")]
 
 
+class LgTokenParams(ctypes.Structure):
+    _fields_ = [("cr_every", ctypes.c_int32), ("theta_streak", ctypes.c_int32),
+                ("hist", ctypes.c_int32), ("pad", ctypes.c_int32),
+                ("theta_cr", ctypes.c_double), ("theta_conf", ctypes.c_double)]
+
+
 STATE_BYTES = 32  # lg_guard_state: 8 x int32
 
 _lib = None
@@ -71,6 +77,10 @@ def lib():
             "lg_detect_state_size": [P(LgCache), P(LgGuardParams)],
             "lg_detect_prune": [P(LgCache), vp, i32, vp, vp, P(LgGuardParams), vp, vp, vp, vp,
                                 vp, vp, i32, i32, vp],
+            "lg_default_token_params": [P(LgTokenParams)],
+            "lg_token_state_size": [P(LgCache), P(LgGuardParams), P(LgTokenParams)],
+            "lg_token_detect": [P(LgCache), vp, vp, vp, P(LgGuardParams), P(LgTokenParams), vp,
+                                vp, vp, vp, vp],
             "lg_prune_compact": [P(LgCache), vp, vp, vp, vp, P(LgGuardParams), vp, vp, i32, i32,
                                  vp],
             "lg_h2o_reset": [P(LgCache), i32, vp],
@@ -87,6 +97,7 @@ def lib():
             f.restype = ctypes.c_int
         L.lg_workspace_size.restype = ctypes.c_size_t
         L.lg_detect_state_size.restype = ctypes.c_size_t
+        L.lg_token_state_size.restype = ctypes.c_size_t
         L.lg_status_string.restype = ctypes.c_char_p
         _lib = L
     return _lib
@@ -98,7 +109,8 @@ def exported_symbols():
             "lg_begin_step", "lg_append", "lg_sketch_build", "lg_decode_attend", "lg_detect",
             "lg_prune_compact", "lg_h2o_reset", "lg_h2o_evict", "lg_read_device_status",
             "lg_decode_attend_noalloc", "lg_detect_state_size", "lg_streaming_evict",
-            "lg_detect_prune"]
+            "lg_detect_prune", "lg_default_token_params", "lg_token_state_size",
+            "lg_token_detect"]
 
 NOALLOC_SCRATCH_BYTES = 32 << 20  # LG_NOALLOC_SCRATCH_BYTES in include/lg.h
 
@@ -179,6 +191,26 @@ def lg_decode_attend_noalloc(cache, layer0, n_layers, q, H_q, scale, out, stats,
 
 def lg_detect_state_size(cache, params) -> int:
     return int(lib().lg_detect_state_size(ctypes.byref(cache.c), ctypes.byref(params)))
+
+
+def lg_default_token_params(**over) -> LgTokenParams:
+    tp = LgTokenParams()
+    _call("lg_default_token_params", ctypes.byref(tp))
+    for k, v in over.items():
+        setattr(tp, k, v)
+    return tp
+
+
+def lg_token_state_size(cache, params, tparams) -> int:
+    return int(lib().lg_token_state_size(ctypes.byref(cache.c), ctypes.byref(params),
+                                         ctypes.byref(tparams)))
+
+
+def lg_token_detect(cache, tokens, pmax, state, params, tparams, flags, spans, diag, tstate,
+                    stream=None):
+    _call("lg_token_detect", ctypes.byref(cache.c), _ptr(tokens), _ptr(pmax), _ptr(state),
+          ctypes.byref(params), ctypes.byref(tparams), _ptr(flags), _ptr(spans), _ptr(diag),
+          _ptr(tstate), _stream(stream))
 
 
 def lg_detect(cache, stats, H_q, state, budget, params, flags, spans, diag, dstate, stream=None):

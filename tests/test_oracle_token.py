@@ -51,7 +51,7 @@ def test_lz77_bounds():
 
 # --------------------------------------------------------------------------- the monitor
 
-def _run(tokens, pmax, n0=4000, budget=1024, prm=None, tp=None, t_gen0=0, stop_at_trigger=True):
+def _run(tokens, pmax, n0=4000, prm=None, tp=None, t_gen0=0, stop_at_trigger=True):
     """feed tokens one step at a time; the cache grows by one row per step from n0"""
     prm = prm or oracle.params()
     tp = tp or oracle.token_params()
@@ -59,7 +59,7 @@ def _run(tokens, pmax, n0=4000, budget=1024, prm=None, tp=None, t_gen0=0, stop_a
     events = []
     for t in range(len(tokens)):
         n = n0 + t + 1
-        f, span, dg = oracle.token_detect(tokens[:t + 1], pmax[t], n, budget, prm, tp, st, ts)
+        f, span, dg = oracle.token_detect(tokens[:t + 1], pmax[t], n, prm, tp, st, ts)
         if f:
             events.append((t, span, dg, n))
             if stop_at_trigger:
@@ -118,7 +118,7 @@ def test_streak_is_strict_and_resets():
     y = np.arange(len(seq), dtype=np.int32)
     streaks = []
     for t, p in enumerate(seq):
-        _, _, dg = oracle.token_detect(y[:t + 1], p, 100 + t, 1024, prm, tp, st, ts)
+        _, _, dg = oracle.token_detect(y[:t + 1], p, 100 + t, prm, tp, st, ts)
         streaks.append(dg["streak"])
     assert streaks == [1, 2, 3, 4, 5, 0, 1, 2, 3, 4, 5, 6, 7, 0, 1, 2, 3]
 
@@ -131,7 +131,7 @@ def test_ttr_and_stall_definitions():
     y = np.array([1, 2, 3, 4, 5, 6, 7, 8, 1, 2, 3, 4, 9, 9, 9, 9, 9], dtype=np.int32)
     got = []
     for t in range(len(y)):
-        _, _, dg = oracle.token_detect(y[:t + 1], 0.5, 50 + t, 1024, prm, tp, st, ts)
+        _, _, dg = oracle.token_detect(y[:t + 1], 0.5, 50 + t, prm, tp, st, ts)
         got.append((dg["ttr"], dg["stall"]))
     # t = 7: window 1..8 all distinct; t = 11: window 5 6 7 8 1 2 3 4 all distinct (the
     # repeats are outside the window); t = 15: 1 2 3 4 9 9 9 9 -> 5 distinct
@@ -154,7 +154,7 @@ def test_span_clipped_to_appended_rows():
     cut = len(y) - 50          # the cache is pruned (shrinks) before this token's step
     for t in range(len(y)):
         n = n + 1 if t != cut else 900
-        f, span, dg = oracle.token_detect(y[:t + 1], pm[t], n, 1024, prm, tp, st, ts)
+        f, span, dg = oracle.token_detect(y[:t + 1], pm[t], n, prm, tp, st, ts)
     assert f == 1 and span == (n - 50, n)
 
 
