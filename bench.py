@@ -58,6 +58,10 @@ def parse():
     ap.add_argument("--fresh-each-step", action="store_true",
                     help="time every step from a freshly generated cache (the first decode "
                          "step: attention over the full prefill and the budget prune)")
+    ap.add_argument("--detector", default="kv", choices=["kv", "token"],
+                    help="loop-onset test of the LoopGuard policy: over attention statistics and "
+                         "V-row sketches (lg_detect_prune), or over the generated token ids and "
+                         "top-1 probabilities (lg_token_detect + lg_prune_compact)")
     ap.add_argument("--eager", action="store_true",
                     help="time the steps as eager launches instead of one CUDA graph replay")
     ap.add_argument("--profile-steps", type=int, default=0,
@@ -170,10 +174,11 @@ class Clocks:
 class GpuBench:
     """Device buffers, the per-step input variants and one guarded step on the C ABI."""
 
-    def __init__(self, w, dev, total_steps, layers_per_call, policy="loopguard"):
+    def __init__(self, w, dev, total_steps, layers_per_call, policy="loopguard", detector="kv"):
         import torch
         from paper_2604_10044_gb300 import lg
         self.torch, self.lg = torch, lg
+        self.detector = detector
         self.w, self.dev = w, dev
         self.policy = policy
         self.stream = torch.cuda.current_stream()
@@ -210,6 +215,16 @@ class GpuBench:
         e = self.esz
         self.sel = synth.Select3(w, self.seqs_d, self.pos_d, (self.q, self.kn, self.vn),
                                  (w.H_q * w.d * e, w.H_kv * w.d * e, w.H_kv * w.d * e))
+        if detector == "token":
+            # generated token ids and top-1 probabilities of every step, both variants
+            tl, tf, pl, pf = synth.token_streams(w, S)
+            self.tokA, self.tokB = (torch.as_tensor(x, device=dev) for x in (tl, tf))
+            self.pmA, self.pmB = (torch.as_tensor(x, device=dev) for x in (pl, pf))
+            self.tok = torch.zeros(b, dtype=torch.int32, device=dev)
+            self.pm = torch.zeros(b, dtype=torch.float32, device=dev)
+            self.tp = lg.lg_default_token_params()
+            self.tstate = torch.zeros(lg.lg_token_state_size(self.cache, self.guard.p, self.tp) // 4,
+                                      dtype=torch.int32, device=dev)
         torch.cuda.synchronize()
 
     def reset(self):
@@ -222,8 +237,12 @@ class GpuBench:
             lg.lg_h2o_reset(self.cache, int(w.n0.max()))
         else:
             lg.lg_sketch_build(self.cache, self.p, int(w.n0.max()))
-        lg.lg_state_init(self.cache, self.guard.state, 64)
+        # the token monitor counts generated tokens from 0; the KV-space test counts the
+        # prompt as seen (its window starts full)
+        lg.lg_state_init(self.cache, self.guard.state, 0 if self.detector == "token" else 64)
         self.guard.dstate.zero_()
+        if self.detector == "token":
+            self.tstate.zero_()
         self.pos_d.copy_(self.n0_d.to(torch.int64))
         self.cache.status.zero_()
         torch.cuda.synchronize()
@@ -251,7 +270,14 @@ class GpuBench:
                                 1 if h2o else 0, g.max_len, g.ws, self.s)
         if ev:
             ev[1].record(self.stream)
-        if guard_path and not split:
+        token = guard_path and self.detector == "token"
+        if token:
+            # the caller's generated token and top-1 probability, then the token-level monitor
+            synth.dev_select_tokens(w, self.seqs_d, self.pos_d, self.tokA[t], self.tokB[t],
+                                    self.pmA[t], self.pmB[t], self.tok, self.pm, self.s)
+            lg.lg_token_detect(c, self.tok, self.pm, g.state, p, self.tp, g.flags, g.spans,
+                               None, self.tstate, self.s)
+        elif guard_path and not split:
             # loop-onset test and retained set in one kernel, then the compaction
             lg.lg_detect_prune(c, g.stats, w.H_q, g.state, self.budget_d, p, g.flags, g.spans,
                                None, g.dstate, g.kept_idx, g.kept_count, g.max_keep, g.max_len,
@@ -261,7 +287,7 @@ class GpuBench:
                          g.dstate, self.s)
         if ev:
             ev[2].record(self.stream)
-        if guard_path and split:
+        if guard_path and (split or token):
             lg.lg_prune_compact(c, g.flags, g.spans, g.state, self.budget_d, p, g.kept_idx,
                                 g.kept_count, g.max_keep, g.max_len, self.s)
         elif h2o:
@@ -275,15 +301,18 @@ class GpuBench:
     # launches of this repository's kernels per step (harness + path)
     def launches_per_step(self):
         calls = math.ceil(self.w.L / self.nl)
-        if self.policy == "h2o":   # begin, append, attend (partial, combine, accumulate), evict x2
-            path = 1 + 1 + 3 * calls + 2
-        elif self.policy == "streaming":   # begin, append, attend (partial, combine), evict x2
-            path = 1 + 1 + 2 * calls + 2
-        elif self.policy == "full":        # begin, append, attend (partial, combine)
-            path = 1 + 1 + 2 * calls
-        else:                      # begin, append (+sketch), attend (partial, combine),
-            path = 1 + 1 + 2 * calls + 2            # detect + keep, compact
+        # one attention kernel per call on the tensor-core path (it merges its own partials),
+        # a partial pass and a merge on the fp32 path; the H2O path adds the score update
+        attend = (1 if self.w.dtype == "bf16" else 2) + (1 if self.policy == "h2o" else 0)
+        path = 1 + 1 + attend * calls               # begin, append (+sketch), attend
         harness = 1 + 1                             # select, advance
+        if self.policy in ("h2o", "streaming"):     # evict, lengths
+            path += 2
+        elif self.policy == "loopguard" and self.detector == "token":
+            path += 3                               # token monitor, keep set, compact
+            harness += 1                            # the step's token and p_max
+        elif self.policy == "loopguard":
+            path += 2                               # detect + keep, compact
         return path, harness
 
     def replay_log(self, K, fresh=False):
@@ -383,7 +412,8 @@ def run_gpu(args, ws, rank, local):
     # every launch of the run goes to one side stream (stream capture needs a non-default one)
     side = torch.cuda.Stream(device=dev)
     torch.cuda.set_stream(side)
-    bench = GpuBench(w, dev, 1 if fresh else max(K, W, 1), args.layers_per_call, args.policy)
+    bench = GpuBench(w, dev, 1 if fresh else max(K, W, 1), args.layers_per_call, args.policy,
+                     args.detector)
 
     # warm-up on the trajectory's first W steps, then a fresh cache for the timed run
     bench.reset()
@@ -503,7 +533,10 @@ def run_gpu(args, ws, rank, local):
                        else "consecutive decode steps from a fresh cache",
                        launch="eager" if graph is None else
                        "one CUDA graph replay of the K steps (captured before timing)",
-                       layers_per_attend_call=bench.nl, parallelism="dp%d (independent batches, "
+                       layers_per_attend_call=bench.nl,
+                       detector="token ids and p_max (lg_token_detect)"
+                       if args.detector == "token" else "attention statistics and V-row sketches",
+                       parallelism="dp%d (independent batches, "
                        "no collective)" % ws, tokens_per_step=w.batch * ws),
         "roofline": {"bound": "hbm", "achieved": round(attend_gbs, 1), "peak": hbm_peak,
                      "unit": "GB/s", "frac": round(attend_gbs / hbm_peak, 4),
@@ -544,6 +577,11 @@ def run_e2e(bench, K, ws):
     hq = [bench.qA[:K].cpu().pin_memory(), bench.qB[:K].cpu().pin_memory()]
     hk = [bench.kA[:K].cpu().pin_memory(), bench.kB[:K].cpu().pin_memory()]
     hv = [bench.vA[:K].cpu().pin_memory(), bench.vB[:K].cpu().pin_memory()]
+    pairs_tok = []
+    if bench.detector == "token":
+        # the generated token ids and top-1 probabilities of the step, both variants
+        for dev_t in (bench.tokA, bench.tokB, bench.pmA, bench.pmB):
+            pairs_tok.append((dev_t, dev_t[:K].cpu().pin_memory()))
     g = bench.guard
     out_h = torch.empty(g.out.shape, dtype=g.out.dtype).pin_memory()
     small_h = torch.empty(4 * w.batch, dtype=torch.int32).pin_memory()
@@ -555,7 +593,8 @@ def run_e2e(bench, K, ws):
     for t in range(K):
         # H2D: this step's input variants into the device staging slots the harness reads
         for dst, src in ((bench.qA, hq[0]), (bench.qB, hq[1]), (bench.kA, hk[0]),
-                         (bench.kB, hk[1]), (bench.vA, hv[0]), (bench.vB, hv[1])):
+                         (bench.kB, hk[1]), (bench.vA, hv[0]), (bench.vB, hv[1])) + tuple(
+                             pairs_tok):
             dst[t].copy_(src[t], non_blocking=True)
         bench.step(t)
         out_h.copy_(g.out, non_blocking=True)
@@ -566,6 +605,7 @@ def run_e2e(bench, K, ws):
         bench.stream.synchronize()
     dt = max_over_ranks(time.perf_counter() - t0, ws)
     h2d = 2 * (hq[0][0].numel() + hk[0][0].numel() + hv[0][0].numel()) * hq[0].element_size()
+    h2d += sum(h[0].numel() * h.element_size() for _, h in pairs_tok)
     d2h = out_h.numel() * out_h.element_size() + small_h.numel() * 4
     return {"value": round(sum_over_ranks(K, ws) / dt, 3), "unit": UNIT,
             "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),

@@ -373,8 +373,9 @@ def dev_lib():
         lib.syn_dev_advance.argtypes = [vp, i32, vp, vp, vp]
         lib.syn_dev_select.argtypes = [vp, i32, vp, i32, i64, vp, vp, vp, vp]
         lib.syn_dev_select3.argtypes = [vp, i32, vp, i32, vp, vp, vp, vp, vp]
+        lib.syn_dev_select_tokens.argtypes = [vp, i32, vp, vp, vp, vp, vp, vp, vp, vp]
         for f in (lib.syn_dev_fill_cache, lib.syn_dev_step, lib.syn_dev_advance,
-                  lib.syn_dev_select, lib.syn_dev_select3):
+                  lib.syn_dev_select, lib.syn_dev_select3, lib.syn_dev_select_tokens):
             f.restype = ctypes.c_int
         _dev = lib
     return _dev
@@ -417,6 +418,54 @@ def dev_select(w: Workload, seqs_dev, pos_dev, rowlen_bytes: int, loop_buf, fres
     _check(dev_lib().syn_dev_select(seqs_dev.data_ptr(), w.batch, pos_dev.data_ptr(), w.L,
                                     rowlen_bytes, loop_buf.data_ptr(), fresh_buf.data_ptr(),
                                     out.data_ptr(), stream), "syn_dev_select")
+
+
+def dev_select_tokens(w: Workload, seqs_dev, pos_dev, tok_loop, tok_fresh, pm_loop, pm_fresh,
+                      tok, pm, stream):
+    _check(dev_lib().syn_dev_select_tokens(seqs_dev.data_ptr(), w.batch, pos_dev.data_ptr(),
+                                           tok_loop.data_ptr(), tok_fresh.data_ptr(),
+                                           pm_loop.data_ptr(), pm_fresh.data_ptr(),
+                                           tok.data_ptr(), pm.data_ptr(), stream),
+           "syn_dev_select_tokens")
+
+
+TOKEN_VOCAB = 50_000
+
+
+def _token_at(seed: int, seq: int, pos: int) -> int:
+    return (mix64(mix64(seed ^ 0x70C3E5) ^ (seq << 32) ^ pos) >> 40) % TOKEN_VOCAB
+
+
+def _pmax_at(seed: int, seq: int, pos: int) -> float:
+    return 0.2 + 0.6 * ((mix64(mix64(seed ^ 0x9B1A) ^ (seq << 32) ^ pos) >> 40) / float(1 << 24))
+
+
+def token_streams(w: Workload, steps: int):
+    """Generated token ids and top-1 probabilities of every step, for a caller of the
+    token-level monitor, in the two variants the decode inputs have: (tok_loop, tok_fresh,
+    pm_loop, pm_fresh), each [steps][batch].  A healthy token is a hash of (sequence,
+    position) over a 50 000-token vocabulary with p_max in [0.2, 0.8); a sequence inside its
+    planted loop (position >= start) repeats the `period` tokens before the start, with
+    p_max 0.95, in the loop-continuing variant."""
+    tl = np.zeros((steps, w.batch), dtype=np.int32)
+    tf = np.zeros_like(tl)
+    pl = np.zeros((steps, w.batch), dtype=np.float32)
+    pf = np.zeros_like(pl)
+    for b in range(w.batch):
+        sq = w.seqs[b]
+        for t in range(steps):
+            pos = int(w.n0[b]) + t
+            tf[t, b] = _token_at(w.seed, b, pos)
+            pf[t, b] = _pmax_at(w.seed, b, pos)
+            if sq["looping"] and pos >= sq["start"]:
+                P = int(sq["period"])
+                src = int(sq["start"]) - P + (pos - int(sq["start"])) % P
+                tl[t, b] = _token_at(w.seed, b, src)
+                pl[t, b] = 0.95
+            else:
+                tl[t, b] = tf[t, b]
+                pl[t, b] = pf[t, b]
+    return tl, tf, pl, pf
 
 
 class Select3:

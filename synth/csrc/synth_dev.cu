@@ -109,6 +109,19 @@ __global__ void select3_kernel(const syn_seq *seqs, int batch, const int64_t *po
   }
 }
 
+// each sequence's token id and top-1 probability of the step: the loop-continuing variant
+// until the guard has intervened (pos >= fresh_from), the loop-free one after
+__global__ void select_tokens_kernel(const syn_seq *seqs, int batch, const int64_t *pos,
+                                     const int32_t *tok_loop, const int32_t *tok_fresh,
+                                     const float *pm_loop, const float *pm_fresh, int32_t *tok,
+                                     float *pm) {
+  const int b = blockIdx.x * blockDim.x + threadIdx.x;
+  if (b >= batch) return;
+  const bool fresh = pos[b] >= seqs[b].fresh_from;
+  tok[b] = fresh ? tok_fresh[b] : tok_loop[b];
+  pm[b] = fresh ? pm_fresh[b] : pm_loop[b];
+}
+
 }  // namespace
 
 extern "C" {
@@ -169,6 +182,14 @@ int syn_dev_select(const syn_seq *seqs_dev, int batch, const int64_t *pos_dev, i
   select_kernel<<<(unsigned)((total + 255) / 256), 256, 0, stream>>>(
       seqs_dev, batch, pos_dev, L, rowlen_bytes, (const char *)loop_buf, (const char *)fresh_buf,
       (char *)out);
+  return cudaGetLastError() == cudaSuccess ? 0 : 2;
+}
+
+int syn_dev_select_tokens(const syn_seq *seqs_dev, int batch, const int64_t *pos_dev,
+                          const int32_t *tok_loop, const int32_t *tok_fresh, const float *pm_loop,
+                          const float *pm_fresh, int32_t *tok, float *pm, cudaStream_t stream) {
+  select_tokens_kernel<<<(batch + 127) / 128, 128, 0, stream>>>(
+      seqs_dev, batch, pos_dev, tok_loop, tok_fresh, pm_loop, pm_fresh, tok, pm);
   return cudaGetLastError() == cudaSuccess ? 0 : 2;
 }
 
