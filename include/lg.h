@@ -219,7 +219,7 @@ LG_API lg_status lg_default_token_params(lg_token_params *tp);
 LG_API size_t lg_token_state_size(const lg_cache *c, const lg_guard_params *p,
                                   const lg_token_params *tp);
 
-/* Token-level loop-onset monitor (Sec. 5.2, Eq. 8, Eq. 9, App. B.2; indicators of Sec. 4.2),
+/* Token-level loop-onset monitor (Sec. 5.2, Eq. 8, Eq. 9, App. B.2; indicators of Sec. 4.3),
    one step per call, for callers that have the generated token ids and top-1 probabilities:
      window W_t = the last min(W, t) generated tokens; a token of W_t is novel when no earlier
        token of W_t equals it;

@@ -192,7 +192,7 @@ def detect(stats, sketches, budget, prm: Params, st: State):
 
 
 def lz77_phrases(x) -> int:
-    """phrases of the greedy LZ77 parse of a token sequence (Sec. 4.2's comp, read as LZ77)"""
+    """phrases of the greedy LZ77 parse of a token sequence (Sec. 4.3's comp(), read as LZ77)"""
     x = np.ascontiguousarray(x, dtype=np.int32)
     return int(lib().lgref_lz77_phrases(_p(x), x.size))
 

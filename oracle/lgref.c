@@ -16,7 +16,7 @@
  *   progressive aggressiveness, gather ....... Sec. 5.3
  *   H2O comparator (cited, not defined) ...... Sec. 2.2, Sec. 6.1
  *   StreamingLLM comparator (cited) .......... Sec. 2.2, Sec. 6.1
- *   token-level monitor (TTR, CR, p_max) ..... Sec. 4.2, Sec. 5.2, Eq. 8, Eq. 9, App. B.2
+ *   token-level monitor (TTR, CR, p_max) ..... Sec. 4.3, Sec. 5.2, Eq. 8, Eq. 9, App. B.2
  *
  * The paper's detector reads generated token ids and top-1 probabilities; the
  * decode path carries only K/V caches and attention, so each signal is

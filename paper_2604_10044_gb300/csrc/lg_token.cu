@@ -1,5 +1,5 @@
 // Token-level loop-onset monitor (LoopGuard Sec. 5.2, Eq. 8, Eq. 9, App. B.2; indicators of
-// Sec. 4.2) over the generated token ids and top-1 probabilities the caller passes each step.
+// Sec. 4.3) over the generated token ids and top-1 probabilities the caller passes each step.
 //
 // One CTA per sequence.  The monitor state (tstate) of a sequence keeps the last `hist` tokens
 // and, for each, the latest earlier equal token of the window as it was when the token arrived

@@ -253,7 +253,7 @@ def make_workload(i: int, **ov) -> Workload:
         # The paper's own setting (Sec. 6.1, App. C): a 1-2B model (Qwen3-1.7B shape: 28 layers,
         # 16 query / 8 kv heads, d=128), a LoopBench-DC-length prompt (3853 tokens on average),
         # budget 1024, generation capped at T_max = 2500; one loop whose onset falls where
-        # most of the paper's interventions happen (800-1300 generated tokens, Fig. 4).
+        # most of the paper's interventions happen (800-1300 generated tokens, Sec. 6.4, Fig. 4).
         b = ov.get("batch", 1); seed = ov.get("seed", 5)
         n = ov.get("n", 3853); B = ov.get("budget", 1024)
         L = ov.get("L", 28)

@@ -1,4 +1,4 @@
-"""Pins of the oracle's token-level monitor (Sec. 4.2, Sec. 5.2, Eq. 8, Eq. 9, App. B.2) against
+"""Pins of the oracle's token-level monitor (Sec. 4.3, Sec. 5.2, Eq. 8, Eq. 9, App. B.2) against
 hand-worked parses, closed forms and invariants; nothing here re-types the oracle's loops.
 
 Readings: comp() of the CR indicator is the greedy LZ77 parse over token ids (a phrase is the
