@@ -62,6 +62,10 @@ def parse():
                     help="loop-onset test of the LoopGuard policy: over attention statistics and "
                          "V-row sketches (lg_detect_prune), or over the generated token ids and "
                          "top-1 probabilities (lg_token_detect + lg_prune_compact)")
+    ap.add_argument("--ablation", action="store_true",
+                    help="run the synthetic analog of the paper's ablation (no guard, always-on "
+                         "pruning, the confidence streak alone, the full guard) on the GPU path and "
+                         "print its measures instead of the step benchmark")
     ap.add_argument("--eager", action="store_true",
                     help="time the steps as eager launches instead of one CUDA graph replay")
     ap.add_argument("--profile-steps", type=int, default=0,
@@ -276,7 +280,7 @@ class GpuBench:
             synth.dev_select_tokens(w, self.seqs_d, self.pos_d, self.tokA[t], self.tokB[t],
                                     self.pmA[t], self.pmB[t], self.tok, self.pm, self.s)
             lg.lg_token_detect(c, self.tok, self.pm, g.state, p, self.tp, g.flags, g.spans,
-                               None, self.tstate, self.s)
+                               None, self.tstate, g.kept_idx, g.kept_count, self.s)
         elif guard_path and not split:
             # loop-onset test and retained set in one kernel, then the compaction
             lg.lg_detect_prune(c, g.stats, w.H_q, g.state, self.budget_d, p, g.flags, g.spans,
@@ -699,9 +703,38 @@ def run_reference(args, ws, rank):
     print(json.dumps(line), flush=True)
 
 
+def run_ablation(args, local):
+    """the ablation analog (synth.ablation) at the paper's setting: B = 1024, a 3853-token
+    prompt, T_max = 2500, loops starting at 800-1300 generated tokens with periods 16..64"""
+    import torch
+    import synth.ablation as A
+    from paper_2604_10044_gb300.ablation import run_variant
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    streams = A.LoopStreams(args.batch or 64, 3853, 2500)
+    res = {}
+    for name, over in A.VARIANTS.items():
+        t0 = time.perf_counter()
+        m, _ = run_variant(streams, over, dev)
+        m["wall_s"] = round(time.perf_counter() - t0, 2)
+        res[name] = m
+    print(json.dumps({
+        "metric": "synthetic ablation of the guard variants (Table 3 analog)",
+        "unit": "loop rate %, interventions per sequence, early interventions %",
+        "variants": res, "data": "synthetic",
+        "config": {"sequences": streams.batch, "prompt": 3853, "budget": 1024,
+                   "steps": streams.steps, "onset": "U{800..1300}", "period": "U{16..64}",
+                   "detector": "token-level monitor (lg_token_detect) + lg_prune_compact"}}),
+        flush=True)
+
+
 def main():
     args = parse()
     ws, rank, local = dist_setup()
+    if args.ablation:
+        if rank == 0:
+            run_ablation(args, local)
+        return
     if ws != args.gpus:
         raise SystemExit("--gpus %d but WORLD_SIZE=%d" % (args.gpus, ws))
     if args.impl == "reference":

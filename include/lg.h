@@ -234,17 +234,23 @@ LG_API size_t lg_token_state_size(const lg_cache *c, const lg_guard_params *p,
      Trigger = t_gen >= t_min and cd = 0 and votes >= K and (Stall or TailRep).
    On a trigger with TailRep the span [lo, hi) covers the verified run extended back while
    tokens keep equalling the token P* earlier (at most hist tokens back) plus its first period,
-   mapped onto the trailing cache rows appended one per step since the cache last changed
-   otherwise (hi = len[b]).  The span is not clipped here: lg_prune_compact, which takes
+   mapped onto the trailing cache rows that hold consecutive generated tokens (hi = len[b]):
+   the rows appended one per step since the cache last changed otherwise, or, when the caller
+   passes the retained lists of the prune that followed the previous call, also the kept rows
+   that end the kept list one after another up to the old last row (a budget cut keeps its
+   recent rows so).  The span is not clipped here: lg_prune_compact, which takes
    flags, spans and state as from lg_detect, clips it to W^recent.
    tokens: device [batch] int32, this step's generated token; pmax: device [batch] fp32.
-   state (16-byte aligned), flags, spans as for lg_detect; diag: nullable device [batch][8]
+   kept_idx, kept_count, max_keep: nullable (both or neither): the kept_idx/kept_count buffers
+   lg_prune_compact wrote after the previous call (kept_count -1 = not pruned), as laid out
+   there.  state (16-byte aligned), flags, spans as for lg_detect; diag: nullable device [batch][8]
    fp64 {TTR, CR, streak, vote 1, vote 2, vote 3, Stall, P* (0 = none)}.
    tstate: device, lg_token_state_size bytes, 8-byte aligned, zero-filled before the first
    call.  Call it once per decode step after the step's append (len[b] counts this step's
    row). */
 LG_API lg_status lg_token_detect(const lg_cache *c, const int32_t *tokens, const float *pmax,
-                                 lg_guard_state *state, const lg_guard_params *p,
+                                 const int32_t *kept_idx, const int32_t *kept_count,
+                                 int max_keep, lg_guard_state *state, const lg_guard_params *p,
                                  const lg_token_params *tp, int32_t *flags, int32_t *spans,
                                  double *diag, void *tstate, cudaStream_t s);
 

@@ -120,7 +120,7 @@ def lib():
         L.lgref_streaming_select.argtypes = [i32, vp, i32, i32, ctypes.c_int32, vp]
         L.lgref_streaming_oldest.argtypes = [i32, vp, i32]
         L.lgref_lz77_phrases.argtypes = [vp, i32]
-        L.lgref_token_detect.argtypes = [vp, i32, dbl, i32, ctypes.POINTER(Params),
+        L.lgref_token_detect.argtypes = [vp, i32, dbl, i32, vp, i32, ctypes.POINTER(Params),
                                          ctypes.POINTER(TokenParams), ctypes.POINTER(State),
                                          ctypes.POINTER(TokenState), vp, vp, vp]
         _lib = L
@@ -200,15 +200,20 @@ def lz77_phrases(x) -> int:
 TOKEN_DIAG_KEYS = ("ttr", "cr", "streak", "sig1", "sig2", "sig3", "warn", "stall", "P", "trigger")
 
 
-def token_detect(tokens, pmax, n, prm: Params, tp: TokenParams, st: State, ts: TokenState):
+def token_detect(tokens, pmax, n, prm: Params, tp: TokenParams, st: State, ts: TokenState,
+                 kept=None):
     """Token-level monitor for one sequence and one step: tokens = every generated token so far
     (the last is this step's), pmax this step's top-1 probability, n the cache length after the
-    step's append.  Returns (flag, (lo, hi) in cache slots, diag dict); st, ts updated."""
+    step's append, kept the retained slots of the prune after the previous step (None if there
+    was none).  Returns (flag, (lo, hi) in cache slots, diag dict); st, ts updated."""
     y = np.ascontiguousarray(tokens, dtype=np.int32)
     flag = np.zeros(1, dtype=np.int32)
     span = np.zeros(2, dtype=np.int32)
     diag = np.zeros(10)
-    rc = lib().lgref_token_detect(_p(y), y.size, float(pmax), int(n), ctypes.byref(prm), ctypes.byref(tp), ctypes.byref(st),
+    k = None if kept is None else np.ascontiguousarray(kept, dtype=np.int32)
+    rc = lib().lgref_token_detect(_p(y), y.size, float(pmax), int(n),
+                                  None if k is None or k.size == 0 else _p(k),
+                                  -1 if k is None else int(k.size), ctypes.byref(prm), ctypes.byref(tp), ctypes.byref(st),
                                   ctypes.byref(ts), _p(flag), _p(span), _p(diag))
     if rc:
         raise ValueError("lgref_token_detect rejected its arguments")

@@ -441,16 +441,29 @@ int lgref_lz77_phrases(const int32_t *x, int w) {
   return phrases;
 }
 
-int lgref_token_detect(const int32_t *tokens, int T, double pmax, int n, const lgref_params *p,
-                       const lgref_token_params *tp, lgref_state *st,
-                       lgref_token_state *ts, int32_t *flag, int32_t *span, double *diag) {
+int lgref_token_detect(const int32_t *tokens, int T, double pmax, int n, const int32_t *kept,
+                       int kept_count, const lgref_params *p, const lgref_token_params *tp,
+                       lgref_state *st, lgref_token_state *ts, int32_t *flag, int32_t *span,
+                       double *diag) {
   if (T < 1 || n < 1 || !p || !tp || !st || !ts || tp->cr_every < 1) return -1;
   const int32_t *y = tokens;
   const int t = T - 1; /* this step's token */
 
-  /* cache rows that are consecutive generated tokens: one more after an append, else only
-     this step's row (the cache changed otherwise since the previous step) */
-  ts->appended = (ts->synced >= 0 && n == ts->synced + 1) ? ts->appended + 1 : 1;
+  /* cache rows that are consecutive generated tokens, this step's row included */
+  if (ts->synced >= 0 && kept && kept_count >= 0 && n == kept_count + 1) {
+    /* the cache was pruned after the previous step: the kept rows that end the kept list
+       one after another, up to the old last row, and were consecutive tokens before, still
+       are */
+    int run = 0;
+    for (int j = kept_count - 1; j >= 0; --j) {
+      if (kept[j] != ts->synced - (kept_count - j) || kept[j] < ts->synced - ts->appended) break;
+      ++run;
+    }
+    ts->appended = run + 1;
+  } else {
+    /* one more after an append; only this step's row after any other change */
+    ts->appended = (ts->synced >= 0 && n == ts->synced + 1) ? ts->appended + 1 : 1;
+  }
   if (ts->appended > n) ts->appended = n;
   ts->synced = n;
 

@@ -141,12 +141,15 @@ int lgref_lz77_phrases(const int32_t *x, int w);
 
 /* One decode step of the token-level monitor.  tokens[0..T) are every generated token so far
    (tokens[T-1] is this step's), pmax this step's top-1 probability, n the cache length after
-   this step's append.  Writes the trigger flag and the span [lo, hi) of cache slots (empty
-   [0,0) without a tail period) and updates the guard and monitor state.  diag nullable [10]:
-   {ttr, cr, streak, vote1, vote2, vote3, warn, stall, P*, trigger}. */
-int lgref_token_detect(const int32_t *tokens, int T, double pmax, int n, const lgref_params *p,
-                       const lgref_token_params *tp, lgref_state *st,
-                       lgref_token_state *ts, int32_t *flag, int32_t *span, double *diag);
+   this step's append; kept[0..kept_count) (nullable; kept_count -1 = no prune) the retained
+   slots of the prune that followed the previous step.  Writes the trigger flag and the span
+   [lo, hi) of cache slots (empty [0,0) without a tail period) and updates the guard and
+   monitor state.  diag nullable [10]: {ttr, cr, streak, vote1, vote2, vote3, warn, stall, P*,
+   trigger}. */
+int lgref_token_detect(const int32_t *tokens, int T, double pmax, int n, const int32_t *kept,
+                       int kept_count, const lgref_params *p, const lgref_token_params *tp,
+                       lgref_state *st, lgref_token_state *ts, int32_t *flag, int32_t *span,
+                       double *diag);
 
 #ifdef __cplusplus
 }

@@ -275,6 +275,7 @@ size_t lg_token_state_size(const lg_cache *c, const lg_guard_params *p,
 }
 
 lg_status lg_token_detect(const lg_cache *c, const int32_t *tokens, const float *pmax,
+                          const int32_t *kept_idx, const int32_t *kept_count, int max_keep,
                           lg_guard_state *state, const lg_guard_params *p,
                           const lg_token_params *tp, int32_t *flags, int32_t *spans, double *diag,
                           void *tstate, cudaStream_t s) {
@@ -284,8 +285,10 @@ lg_status lg_token_detect(const lg_cache *c, const int32_t *tokens, const float 
   if ((st = check_token_params(p, tp)) != LG_OK) return st;
   if (!tokens || !pmax || !state || !flags || !spans || !tstate) return LG_ERR_INVALID_ARG;
   if (((uintptr_t)state & 15u) || ((uintptr_t)tstate & 7u)) return LG_ERR_INVALID_ARG;
-  return cuda_status(lg::launch_token_detect(*c, tokens, pmax, state, *p, *tp, flags, spans,
-                                             diag, tstate, s));
+  if ((kept_idx == nullptr) != (kept_count == nullptr) || (kept_idx && max_keep < 1))
+    return LG_ERR_INVALID_ARG;
+  return cuda_status(lg::launch_token_detect(*c, tokens, pmax, kept_idx, kept_count, max_keep,
+                                             state, *p, *tp, flags, spans, diag, tstate, s));
 }
 
 size_t lg_detect_state_size(const lg_cache *c, const lg_guard_params *p) {

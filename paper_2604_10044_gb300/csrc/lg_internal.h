@@ -63,6 +63,7 @@ cudaError_t launch_compact(const lg_cache &c, const int32_t *kept_idx, const int
 size_t token_state_words(const lg_guard_params &p, const lg_token_params &tp);
 size_t token_smem_bytes(const lg_guard_params &p, const lg_token_params &tp);
 cudaError_t launch_token_detect(const lg_cache &c, const int32_t *tokens, const float *pmax,
+                                const int32_t *kept_idx, const int32_t *kept_count, int max_keep,
                                 lg_guard_state *state, const lg_guard_params &p,
                                 const lg_token_params &tp, int32_t *flags, int32_t *spans,
                                 double *diag, void *tstate, cudaStream_t s);

@@ -18,7 +18,8 @@
 //   Trigger t_gen >= t_min and cd = 0 and votes >= K and (Stall or TailRep)
 // On a trigger with TailRep the span is the verified run extended back while tokens keep
 // equalling the token P* earlier (within the kept history), plus its first period, mapped onto
-// the trailing cache rows that hold consecutive generated tokens.
+// the trailing cache rows that hold consecutive generated tokens (kept across a prune when the
+// caller passes the prune's retained lists).
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -37,6 +38,9 @@ struct TokenArgs {
   lg_cache c;
   const int32_t *tokens;  // [batch] this step's token of each sequence
   const float *pmax;      // [batch] this step's top-1 probability
+  const int32_t *kept_idx;    // nullable [batch][max_keep]: the prune after the previous step
+  const int32_t *kept_count;  // nullable [batch], -1 = that sequence was not pruned
+  int max_keep;
   lg_guard_state *state;
   lg_guard_params p;
   lg_token_params tp;
@@ -64,7 +68,8 @@ __device__ __forceinline__ int block_max(int v, int *red, int lane, int warp) {
 __global__ void __launch_bounds__(kTokThreads, 1) token_detect_kernel(TokenArgs a) {
   extern __shared__ __align__(16) int32_t sm[];
   __shared__ int red[kTokWarps];
-  __shared__ int w_latest[kTokWarps], w_nov[kTokWarps], w_tail[kTokWarps], w_pstar[kTokWarps];
+  __shared__ int w_latest[kTokWarps], w_nov[kTokWarps], w_tail[kTokWarps], w_pstar[kTokWarps],
+      w_run[kTokWarps];
   __shared__ int s_mismatch, s_trig, s_P, s_n_tok, s_appended;
   const int b = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const lg_guard_params &p = a.p;
@@ -83,6 +88,8 @@ __global__ void __launch_bounds__(kTokThreads, 1) token_detect_kernel(TokenArgs 
   const int y = a.tokens[b];
   const double pm = (double)a.pmax[b];
   const int t = ts[0];  // tokens before this one: this token is position t
+  const int synced = ts[2] - 1, app_old = ts[3];
+  const int kc = a.kept_count ? a.kept_count[b] : -1;
   int4 st_a = make_int4(0, 0, 0, 0), st_b = make_int4(0, 0, 0, 0);
   if (tid == 0) {
     st_a = reinterpret_cast<const int4 *>(a.state + b)[0];
@@ -136,11 +143,28 @@ __global__ void __launch_bounds__(kTokThreads, 1) token_detect_kernel(TokenArgs 
   nov = __reduce_add_sync(0xffffffffu, nov);
   tail = __reduce_add_sync(0xffffffffu, tail);
   pstar = (int)__reduce_min_sync(0xffffffffu, (unsigned)pstar);
+  // after a prune of this sequence: the kept rows that end the kept list one after another up
+  // to the old last row, and were consecutive tokens before, still are (first break from the end)
+  const bool use_kept = kc >= 0 && synced >= 0 && n == kc + 1;
+  const int run_lim = use_kept ? min(kc, app_old) : 0;
+  int first_bad = 0x7fffffff;
+  if (use_kept) {
+    const int32_t *K = a.kept_idx + (int64_t)b * a.max_keep;
+    for (int jo = tid; jo < run_lim; jo += kTokThreads) {
+      const int v = K[kc - 1 - jo];
+      if (v != synced - 1 - jo || v < synced - app_old) {
+        first_bad = jo;
+        break;
+      }
+    }
+  }
+  first_bad = (int)__reduce_min_sync(0xffffffffu, (unsigned)first_bad);
   if (lane == 0) {
     w_latest[warp] = latest;
     w_nov[warp] = nov;
     w_tail[warp] = tail;
     w_pstar[warp] = pstar;
+    w_run[warp] = first_bad;
   }
 
   // (2) compression ratio of the window, every cr_every tokens
@@ -176,12 +200,13 @@ __global__ void __launch_bounds__(kTokThreads, 1) token_detect_kernel(TokenArgs 
 
   // (3) votes, gates, trigger, state (thread 0)
   if (tid == 0) {
-    int lt = -1, nv = 0, tl = 0, ps = 0x7fffffff;
+    int lt = -1, nv = 0, tl = 0, ps = 0x7fffffff, fb = 0x7fffffff;
     for (int k = 0; k < kTokWarps; ++k) {
       lt = max(lt, w_latest[k]);
       nv += w_nov[k];
       tl += w_tail[k];
       ps = min(ps, w_pstar[k]);
+      fb = min(fb, w_run[k]);
     }
     const int novel = lt < wlo;
     nv += novel;
@@ -203,8 +228,11 @@ __global__ void __launch_bounds__(kTokThreads, 1) token_detect_kernel(TokenArgs 
                       (double)tl / (double)p.stall_len < p.theta_nov;
     const int tailrep = ps != 0x7fffffff;
     const int trig = st_a.x >= p.t_min && st_a.y == 0 && warn && (stall || tailrep);
-    const int synced = ts[2] - 1;
-    int appended = (synced >= 0 && n == synced + 1) ? ts[3] + 1 : 1;
+    int appended;
+    if (use_kept)
+      appended = min(fb, run_lim) + 1;
+    else
+      appended = (synced >= 0 && n == synced + 1) ? app_old + 1 : 1;
     appended = min(appended, n);
     if (a.diag) {
       double *dg = a.diag + 8 * b;
@@ -283,6 +311,7 @@ size_t token_smem_bytes(const lg_guard_params &p, const lg_token_params &tp) {
 }
 
 cudaError_t launch_token_detect(const lg_cache &c, const int32_t *tokens, const float *pmax,
+                                const int32_t *kept_idx, const int32_t *kept_count, int max_keep,
                                 lg_guard_state *state, const lg_guard_params &p,
                                 const lg_token_params &tp, int32_t *flags, int32_t *spans,
                                 double *diag, void *tstate, cudaStream_t s) {
@@ -290,6 +319,9 @@ cudaError_t launch_token_detect(const lg_cache &c, const int32_t *tokens, const 
   a.c = c;
   a.tokens = tokens;
   a.pmax = pmax;
+  a.kept_idx = kept_idx;
+  a.kept_count = kept_count;
+  a.max_keep = max_keep;
   a.state = state;
   a.p = p;
   a.tp = tp;

@@ -79,8 +79,8 @@ def lib():
                                 vp, vp, i32, i32, vp],
             "lg_default_token_params": [P(LgTokenParams)],
             "lg_token_state_size": [P(LgCache), P(LgGuardParams), P(LgTokenParams)],
-            "lg_token_detect": [P(LgCache), vp, vp, vp, P(LgGuardParams), P(LgTokenParams), vp,
-                                vp, vp, vp, vp],
+            "lg_token_detect": [P(LgCache), vp, vp, vp, vp, i32, vp, P(LgGuardParams),
+                                P(LgTokenParams), vp, vp, vp, vp, vp],
             "lg_prune_compact": [P(LgCache), vp, vp, vp, vp, P(LgGuardParams), vp, vp, i32, i32,
                                  vp],
             "lg_h2o_reset": [P(LgCache), i32, vp],
@@ -207,10 +207,13 @@ def lg_token_state_size(cache, params, tparams) -> int:
 
 
 def lg_token_detect(cache, tokens, pmax, state, params, tparams, flags, spans, diag, tstate,
-                    stream=None):
-    _call("lg_token_detect", ctypes.byref(cache.c), _ptr(tokens), _ptr(pmax), _ptr(state),
-          ctypes.byref(params), ctypes.byref(tparams), _ptr(flags), _ptr(spans), _ptr(diag),
-          _ptr(tstate), _stream(stream))
+                    kept_idx=None, kept_count=None, stream=None):
+    """kept_idx / kept_count: the buffers lg_prune_compact wrote after the previous call (or
+    None): the trailing kept rows that are still consecutive tokens keep mapping the span"""
+    max_keep = int(kept_idx.shape[1]) if kept_idx is not None else 0
+    _call("lg_token_detect", ctypes.byref(cache.c), _ptr(tokens), _ptr(pmax), _ptr(kept_idx),
+          _ptr(kept_count), max_keep, _ptr(state), ctypes.byref(params), ctypes.byref(tparams),
+          _ptr(flags), _ptr(spans), _ptr(diag), _ptr(tstate), _stream(stream))
 
 
 def lg_detect(cache, stats, H_q, state, budget, params, flags, spans, diag, dstate, stream=None):

@@ -43,7 +43,10 @@ def _streams(rng):
     return np.stack(toks), np.stack(pm).astype(np.float32)
 
 
-def test_token_monitor_and_prune_match_oracle(cuda):
+@pytest.mark.parametrize("pass_kept", [True, False])
+def test_token_monitor_and_prune_match_oracle(cuda, pass_kept):
+    """pass_kept: the monitor gets the previous prune's retained lists (rows kept in order at
+    the tail stay mapped to their tokens), or not (only rows appended since a prune are)"""
     rng = np.random.default_rng(7)
     toks, pmax = _streams(rng)
     b = toks.shape[0]
@@ -71,13 +74,15 @@ def test_token_monitor_and_prune_match_oracle(cuda):
     st_o = [oracle.new_state(0) for _ in range(b)]
     ts_o = [oracle.new_token_state() for _ in range(b)]
     n_o = n0.astype(np.int64).copy()
+    prev_kept = [None] * b
     triggers = np.zeros(b, dtype=int)
     prunes = 0
     keys = ("ttr", "cr", "streak", "sig1", "sig2", "sig3", "stall", "P")
     for t in range(STEPS):
         lg.lg_begin_step(cache)
         lg.lg_token_detect(cache, toks_d[t], pmax_d[t], state, prm_g, tp_g, flags, spans, diag,
-                           tstate)
+                           tstate, kept_idx if pass_kept else None,
+                           kept_count if pass_kept else None)
         lg.lg_prune_compact(cache, flags, spans, state, budget, prm_g, kept_idx, kept_count,
                             max_keep, int(cap.max()))
         torch.cuda.synchronize()
@@ -87,7 +92,9 @@ def test_token_monitor_and_prune_match_oracle(cuda):
         for s in range(b):
             n_o[s] += 1
             f, sp, dg = oracle.token_detect(toks[s, :t + 1], float(pmax[s, t]), int(n_o[s]),
-                                            prm_o, tp_o, st_o[s], ts_o[s])
+                                            prm_o, tp_o, st_o[s], ts_o[s],
+                                            kept=prev_kept[s] if pass_kept else None)
+            prev_kept[s] = None
             ctx = (t, s, dg, dg_g[s].tolist(), sp, sp_g[s].tolist())
             assert f_g[s] == f and tuple(sp_g[s]) == sp, ctx
             assert [dg[k] for k in keys] == dg_g[s].tolist(), ctx
@@ -100,6 +107,7 @@ def test_token_monitor_and_prune_match_oracle(cuda):
                 assert kc_g[s] == len(kept) and np.array_equal(
                     kept_idx[s, :kc_g[s]].cpu().numpy(), kept), ctx
                 n_o[s] = len(kept)
+                prev_kept[s] = kept
                 prunes += 1
             assert len_g[s] == n_o[s], ctx
             triggers[s] += f
@@ -118,3 +126,6 @@ def test_token_monitor_rejects_short_history(cuda):
     with pytest.raises(lg.LgError):
         lg.lg_token_detect(cache, t, t.float(), t, prm, lg.lg_default_token_params(hist=200),
                            t, t, None, t)
+    with pytest.raises(lg.LgError):   # kept lists without their counts
+        lg.lg_token_detect(cache, t, t.float(), t, prm, lg.lg_default_token_params(), t, t, None,
+                           t, kept_idx=t.view(1, 64), kept_count=None)

@@ -177,3 +177,27 @@ def test_no_trigger_on_healthy_stream():
     pm = rng.uniform(0.1, 0.95, size=700)
     ev, _, _ = _run(y, pm, stop_at_trigger=False)
     assert ev == []
+
+
+def test_span_follows_a_contiguous_kept_tail():
+    """a prune that keeps the cache's last 400 rows in order (a budget cut keeps its recent rows
+    so) leaves them consecutive generated tokens: given the kept list, the monitor keeps
+    counting them, and the span later covers the whole loop (L* = 213 tokens) instead of the
+    rows appended since the prune"""
+    H, P = 300, 8
+    L_star = math.floor(256 + P - 51.2) + 1
+    y = _healthy_then_loop(H, P, L_star)
+    pm = np.where(np.arange(len(y)) >= H, 0.95, 0.5)
+    prm, tp = oracle.params(), oracle.token_params()
+    st, ts = oracle.new_state(0), oracle.new_token_state()
+    n = 5000
+    cut = len(y) - 50
+    for t in range(len(y)):
+        kept = None
+        if t == cut:
+            kept = np.concatenate([np.arange(32), np.arange(n - 400, n)])
+            n = len(kept)
+        n += 1
+        f, span, dg = oracle.token_detect(y[:t + 1], pm[t], n, prm, tp, st, ts, kept=kept)
+    assert f == 1 and span == (n - L_star, n)
+    assert ts.appended == 400 + 50
