@@ -34,6 +34,7 @@ import synth  # noqa: E402
 
 METRIC = "guarded decode steps/s (attend+stats, detect, prune/compact) and achieved HBM GB/s"
 UNIT = "steps/s"
+L2_BYTES = 129e6
 
 
 def parse():
@@ -514,11 +515,20 @@ def run_gpu(args, ws, rank, local):
     attend_gbs = sum(a_bytes) / (sum(attend_ms) * 1e-3) / 1e9
     compact_gbs = (sum(c_bytes) / (sum(c_ms) * 1e-3) / 1e9) if c_ms else None
 
-    e2e = None
+    e2e = e2e_eager = None
     if not args.no_e2e and not fresh and args.policy == "loopguard":
-        e2e = run_e2e(bench, K, ws)
+        e2e, e2e_eager = run_e2e(bench, K, ws, graphs=not args.eager)
 
     value = sum_over_ranks(K, ws) / (ms * 1e-3)
+    # the K/V bytes a step reads against the 129 MB L2 (no flush between steps)
+    step_read = sum(a_bytes) / max(1, len(a_bytes))
+    if step_read > L2_BYTES:
+        l2_note = ("inputs larger than L2: each step reads %.2f GB of K/V (cache %.1f GB per GPU)"
+                   % (step_read / 1e9, w.kv_bytes() / 1e9))
+    else:
+        l2_note = ("each step reads %.0f MB of K/V, less than the 129 MB L2 (cache %.1f GB per GPU, "
+                   "no flush between steps): bandwidth figures include L2 hits"
+                   % (step_read / 1e6, w.kv_bytes() / 1e9))
     path_l, harness_l = bench.launches_per_step()
     prof = traffic_from_profile(source_hash())
     traffic = None
@@ -531,8 +541,7 @@ def run_gpu(args, ws, rank, local):
         "metric": METRIC, "value": round(value, 3), "unit": UNIT, "n_gpus": ws, "steps": K,
         "warmup": W, "ms_per_step": round(ms / K, 4), "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": w.dtype, "data": "synthetic",
-        "config": dict(w.describe(), l2="inputs larger than L2 (K/V cache %.1f GB per GPU)"
-                       % (w.kv_bytes() / 1e9), policy=args.policy,
+        "config": dict(w.describe(), decode_steps=K, l2=l2_note, policy=args.policy,
                        timed_steps="each from a fresh cache" if fresh
                        else "consecutive decode steps from a fresh cache",
                        launch="eager" if graph is None else
@@ -545,8 +554,9 @@ def run_gpu(args, ws, rank, local):
         "roofline": {"bound": "hbm", "achieved": round(attend_gbs, 1), "peak": hbm_peak,
                      "unit": "GB/s", "frac": round(attend_gbs / hbm_peak, 4),
                      "traffic": traffic,
-                     "kernel": "lg_decode_attend (split-K partial + combine), all %d layers per "
-                               "call" % w.L if bench.nl == w.L else "lg_decode_attend",
+                     "kernel": "lg_decode_attend (tensor-core pass with its split-K merge), all "
+                               "%d layers per call" % w.L if bench.nl == w.L
+                               else "lg_decode_attend",
                      "peak_kind": peak_kind + " copy bandwidth"},
         "kernels": {
             "attend_stats": {"GB_per_s": round(attend_gbs, 1),
@@ -569,36 +579,37 @@ def run_gpu(args, ws, rank, local):
     }
     if e2e:
         line["e2e"] = e2e
+        line["e2e_eager"] = {"value": e2e_eager, "unit": UNIT}
     return line, w
 
 
-def run_e2e(bench, K, ws):
+def run_e2e(bench, K, ws, graphs=True):
     """the same steps through the C ABI with host buffers: every step copies its inputs from
-    pinned host memory and reads the outputs back (attention output, flags, spans, lengths)"""
+    pinned host memory, runs the guarded step and reads the outputs back (attention output,
+    flags, spans, lengths), and the host waits for them before the next step.  graphs: each
+    step's copies, calls and read-back are captured once as a CUDA graph (as a serving loop
+    captures its decode step) and replayed in the timed loop; else they are launched eagerly.
+    Returns (line dict, eager steps/s or None)."""
     torch = bench.torch
     w = bench.w
     # both input variants of every step in pinned host memory (filled before timing)
     hq = [bench.qA[:K].cpu().pin_memory(), bench.qB[:K].cpu().pin_memory()]
     hk = [bench.kA[:K].cpu().pin_memory(), bench.kB[:K].cpu().pin_memory()]
     hv = [bench.vA[:K].cpu().pin_memory(), bench.vB[:K].cpu().pin_memory()]
-    pairs_tok = []
+    pairs = [(bench.qA, hq[0]), (bench.qB, hq[1]), (bench.kA, hk[0]), (bench.kB, hk[1]),
+             (bench.vA, hv[0]), (bench.vB, hv[1])]
     if bench.detector == "token":
         # the generated token ids and top-1 probabilities of the step, both variants
         for dev_t in (bench.tokA, bench.tokB, bench.pmA, bench.pmB):
-            pairs_tok.append((dev_t, dev_t[:K].cpu().pin_memory()))
+            pairs.append((dev_t, dev_t[:K].cpu().pin_memory()))
     g = bench.guard
     out_h = torch.empty(g.out.shape, dtype=g.out.dtype).pin_memory()
     small_h = torch.empty(4 * w.batch, dtype=torch.int32).pin_memory()
     small_d = torch.empty(4 * w.batch, dtype=torch.int32, device=bench.dev)
-    bench.reset()
-    barrier(ws)
-    torch.cuda.synchronize()
-    t0 = time.perf_counter()
-    for t in range(K):
-        # H2D: this step's input variants into the device staging slots the harness reads
-        for dst, src in ((bench.qA, hq[0]), (bench.qB, hq[1]), (bench.kA, hk[0]),
-                         (bench.kB, hk[1]), (bench.vA, hv[0]), (bench.vB, hv[1])) + tuple(
-                             pairs_tok):
+
+    def enqueue(t):
+        # H2D: this step's input variants into the device slots the harness reads
+        for dst, src in pairs:
             dst[t].copy_(src[t], non_blocking=True)
         bench.step(t)
         out_h.copy_(g.out, non_blocking=True)
@@ -606,15 +617,36 @@ def run_e2e(bench, K, ws):
         small_d[w.batch:3 * w.batch].copy_(g.spans.view(-1))
         small_d[3 * w.batch:].copy_(bench.cache.len)
         small_h.copy_(small_d, non_blocking=True)
-        bench.stream.synchronize()
-    dt = max_over_ranks(time.perf_counter() - t0, ws)
-    h2d = 2 * (hq[0][0].numel() + hk[0][0].numel() + hv[0][0].numel()) * hq[0].element_size()
-    h2d += sum(h[0].numel() * h.element_size() for _, h in pairs_tok)
+
+    def timed(run_step):
+        bench.reset()
+        barrier(ws)
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        for t in range(K):
+            run_step(t)
+            bench.stream.synchronize()
+        return max_over_ranks(time.perf_counter() - t0, ws)
+
+    dt_eager = timed(enqueue)
+    dt = dt_eager
+    if graphs:
+        step_graphs = []
+        for t in range(K):
+            gr = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(gr, stream=bench.stream, capture_error_mode="thread_local"):
+                enqueue(t)
+            step_graphs.append(gr)
+        dt = timed(lambda t: step_graphs[t].replay())
+    h2d = sum(h[0].numel() * h.element_size() for _, h in pairs)
     d2h = out_h.numel() * out_h.element_size() + small_h.numel() * 4
-    return {"value": round(sum_over_ranks(K, ws) / dt, 3), "unit": UNIT,
+    line = {"value": round(sum_over_ranks(K, ws) / dt, 3), "unit": UNIT,
             "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
+            "launch": "one CUDA graph per step (copies, guarded step, read-back), host waits "
+                      "for each step" if graphs else "eager, host waits for each step",
             "note": "inputs of both sequence modes (loop continues / loop-free) copied every "
                     "step; outputs, flags, spans and lengths read back every step"}
+    return line, round(sum_over_ranks(K, ws) / dt_eager, 3)
 
 
 # ------------------------------------------------------------------ CPU oracle arm
