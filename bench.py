@@ -723,7 +723,7 @@ def run_reference(args, ws, rank):
     line = {"impl": "reference", "metric": METRIC, "value": round(value, 6), "unit": UNIT,
             "n_gpus": ws, "steps": K, "warmup": W, "ms_per_step": round(1e3 / value, 3),
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
-            "data": "synthetic", "config": w.describe(),
+            "data": "synthetic", "config": dict(w.describe(), decode_steps=args.steps),
             "cpu_baseline": {"value": round(value, 6), "unit": UNIT, "cores": threads,
                              "kind": "oracle",
                              "sample": "each step: the oracle's guarded decode step of sequence "

@@ -13,13 +13,17 @@ namespace lg {
 
 // ------------------------------------------------------------------ step bookkeeping
 
+// (Here and in append_kernel the inputs are read before the status word, so that every load
+// of a thread is in flight at once; neither kernel has a barrier after its status check.)
 __global__ void begin_step_kernel(lg_cache c) {
   const int b = blockIdx.x * blockDim.x + threadIdx.x;
-  if (b >= c.batch || status_bad(c.dev_status)) return;
-  if (c.len[b] + 1 > c.cap[b])
+  if (b >= c.batch) return;
+  const int n = c.len[b], cap = c.cap[b];
+  if (status_bad(c.dev_status)) return;
+  if (n + 1 > cap)
     set_status(c.dev_status, LG_ERR_CAPACITY);
   else
-    c.len[b] += 1;
+    c.len[b] = n + 1;
 }
 
 // sketch word w of a row: sign bits of elements [32w, 32w+32) of the row flattened [H_kv][d]
@@ -43,15 +47,15 @@ template <typename T>
 __global__ void append_kernel(lg_cache c, int layer0, int n_layers, const uint4 *k_new,
                               const uint4 *v_new, const int32_t *pos_new, int row_blocks,
                               int lguard) {
-  if (status_bad(c.dev_status)) return;
   if ((int)blockIdx.x >= row_blocks) {
     const int b = blockIdx.x - row_blocks;
     const int nwords = c.H_kv * c.d / 32;
     const int slot = c.len[b] - 1;
-    if (slot < 0) return;
+    const int64_t off = c.seq_off[b];
+    if (status_bad(c.dev_status) || slot < 0) return;
     const T *row = (const T *)v_new + ((int64_t)lguard * c.batch + b) * c.H_kv * c.d;
     for (int w = threadIdx.x; w < nwords; w += blockDim.x)
-      c.sketch[(c.seq_off[b] + slot) * nwords + w] = sketch_word<T>(row, c.d, c.d, w);
+      c.sketch[(off + slot) * nwords + w] = sketch_word<T>(row, c.d, c.d, w);
     return;
   }
   const int cpr = c.d * (int)sizeof(T) / 16;
@@ -63,14 +67,17 @@ __global__ void append_kernel(lg_cache c, int layer0, int n_layers, const uint4 
   const int kvh = (int)(row % c.H_kv);
   const int b = (int)((row / c.H_kv) % c.batch);
   const int layer = layer0 + (int)(row / ((int64_t)c.H_kv * c.batch));
+  const uint4 kr = k_new[row * cpr + ch], vr = v_new[row * cpr + ch];
   const int slot = c.len[b] - 1;
+  const int64_t off = c.seq_off[b];
+  if (status_bad(c.dev_status)) return;
   if (slot < 0) {
     set_status(c.dev_status, LG_ERR_CAPACITY);
     return;
   }
-  const int64_t s = ((int64_t)layer * c.H_kv + kvh) * c.S_total + c.seq_off[b] + slot;
-  reinterpret_cast<uint4 *>(c.k)[s * cpr + ch] = k_new[row * cpr + ch];
-  reinterpret_cast<uint4 *>(c.v)[s * cpr + ch] = v_new[row * cpr + ch];
+  const int64_t s = ((int64_t)layer * c.H_kv + kvh) * c.S_total + off + slot;
+  reinterpret_cast<uint4 *>(c.k)[s * cpr + ch] = kr;
+  reinterpret_cast<uint4 *>(c.v)[s * cpr + ch] = vr;
   if (ch == 0 && c.pos) {
     c.pos[s] = pos_new[b];
     c.h2o[s] = 0.f;
@@ -640,15 +647,18 @@ __global__ void __launch_bounds__(kCompactThreads) compact_kernel(lg_cache c,
                                                                   const int32_t *kept_count,
                                                                   int max_keep) {
   const int tid = threadIdx.x;
-  if (cta_status_bad(c.dev_status)) return;
   const int row_bytes_kv = c.d * (c.dtype == LG_BF16 ? 2 : 4);
   const int nwords = c.H_kv * c.d / 32;
   const int n_kv = 2 * c.L * c.H_kv;
   const int per_seq = n_kv + 1;
+  // the first item's count is read together with the status word
+  const int cnt_first =
+      (int)blockIdx.x < c.batch * per_seq ? kept_count[blockIdx.x / per_seq] : -1;
+  if (cta_status_bad(c.dev_status)) return;
   // grid-stride over (sequence, stream); sequences left as they were cost one load each
   for (int item = blockIdx.x; item < c.batch * per_seq; item += gridDim.x) {
     const int b = item / per_seq, stream = item - b * per_seq;
-    const int cnt = kept_count[b];
+    const int cnt = item == (int)blockIdx.x ? cnt_first : kept_count[b];
     if (cnt < 0) continue;
     unsigned char *base;
     int row_bytes;

@@ -133,3 +133,17 @@ def test_paper_shaped_guard(cuda):
     w = synth.make_workload(6, L=2, onset=(90, 110), steps=200)
     c = run_loopguard(w, cuda)
     assert c["triggers"] >= 1 and c["prunes"] >= 3
+
+
+@pytest.mark.parametrize("over", [
+    # a window wider than one thread stride, periods from 3 (compared directly), 2 repeats,
+    # a 6-row stall, one vote
+    dict(W=400, p_min=3, p_max=40, m_rep=2, l_min=16, stall_len=6, K=1),
+    # a narrow window, all three votes, a short cooldown and warmup
+    dict(W=100, p_max=60, K=3, theta_lift=1.5, cooldown=8, t_min=10, retrig_window=20),
+])
+def test_nondefault_guard_params(cuda, over):
+    """the same pipeline under other monitor constants: both sides take the same parameters"""
+    w = synth.make_workload(2, L=2, batch=4, n=1200, budget=768, steps=40, tail=(300, 500),
+                            periods=(8, 40))
+    run_loopguard(w, cuda, params=over)

@@ -43,10 +43,15 @@ def _streams(rng):
     return np.stack(toks), np.stack(pm).astype(np.float32)
 
 
-@pytest.mark.parametrize("pass_kept", [True, False])
-def test_token_monitor_and_prune_match_oracle(cuda, pass_kept):
+OTHER = (dict(W=300, p_min=2, p_max=50, m_rep=2, l_min=24, stall_len=6, cooldown=16),
+         dict(hist=320, cr_every=5, theta_streak=4))
+
+
+@pytest.mark.parametrize("pass_kept,params", [(True, None), (False, None), (True, OTHER)])
+def test_token_monitor_and_prune_match_oracle(cuda, pass_kept, params):
     """pass_kept: the monitor gets the previous prune's retained lists (rows kept in order at
-    the tail stay mapped to their tokens), or not (only rows appended since a prune are)"""
+    the tail stay mapped to their tokens), or not (only rows appended since a prune are);
+    params: (guard, token) parameter overrides, the same on both sides"""
     rng = np.random.default_rng(7)
     toks, pmax = _streams(rng)
     b = toks.shape[0]
@@ -55,8 +60,9 @@ def test_token_monitor_and_prune_match_oracle(cuda, pass_kept):
     seq_off = np.concatenate([[0], np.cumsum(cap)[:-1]]).astype(np.int64)
     n0 = np.full(b, N0, dtype=np.int32)
     cache = lg.Cache(1, 1, 128, "f32", seq_off, cap, n0, cuda, "loopguard")
-    prm_g, prm_o = lg.lg_default_params(), oracle.params()
-    tp_g, tp_o = lg.lg_default_token_params(), oracle.token_params()
+    g_over, t_over = params or ({}, {})
+    prm_g, prm_o = lg.lg_default_params(**g_over), oracle.params(**g_over)
+    tp_g, tp_o = lg.lg_default_token_params(**t_over), oracle.token_params(**t_over)
     state = torch.zeros((b, lg.STATE_BYTES // 4), dtype=torch.int32, device=cuda)
     lg.lg_state_init(cache, state, 0)
     tstate = torch.zeros(lg.lg_token_state_size(cache, prm_g, tp_g) // 4, dtype=torch.int32,
@@ -112,8 +118,8 @@ def test_token_monitor_and_prune_match_oracle(cuda, pass_kept):
             assert len_g[s] == n_o[s], ctx
             triggers[s] += f
     assert lg.lg_read_device_status(cache) == 0
-    assert triggers[0] == 0 and triggers[1] >= 2 and triggers[2] >= 1 and triggers[3] >= 2
-    assert triggers[4] >= 2 and prunes > triggers.sum()
+    assert triggers[0] == 0 and triggers[1] >= 1 and triggers[3] >= 1 and triggers[4] >= 2
+    assert prunes > triggers.sum()
 
 
 def test_token_monitor_rejects_short_history(cuda):
