@@ -405,7 +405,8 @@ def run_gpu(args, ws, rank, local):
     K, W = args.steps, args.warmup
     if args.profile_steps:
         # untimed steps inside an NVTX range "steps" (ncu --nvtx-include "steps/")
-        bench = GpuBench(w, dev, args.profile_steps, args.layers_per_call)
+        bench = GpuBench(w, dev, args.profile_steps, args.layers_per_call, args.policy,
+                         args.detector)
         bench.reset()
         torch.cuda.nvtx.range_push("steps")
         for t in range(args.profile_steps):
