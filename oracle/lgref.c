@@ -18,11 +18,12 @@
  *   StreamingLLM comparator (cited) .......... Sec. 2.2, Sec. 6.1
  *   token-level monitor (TTR, CR, p_max) ..... Sec. 4.3, Sec. 5.2, Eq. 8, Eq. 9, App. B.2
  *
- * The paper's detector reads generated token ids and top-1 probabilities; the
- * decode path carries only K/V caches and attention, so each signal is
- * restated over attention statistics and sign sketches of the guard layer's V
- * rows.  The readings (constants marked as the build's choice where the paper
- * is silent) are listed in the design doc and pinned by tests/test_oracle_*.py.
+ * The paper's detector reads generated token ids and top-1 probabilities:
+ * lgref_token_detect follows it on those inputs.  A decode path that carries
+ * only K/V caches and attention has neither, so lgref_detect restates each
+ * signal over attention statistics and sign sketches of the guard layer's V
+ * rows.  Where the paper is silent the constants are this build's choice, stated
+ * beside each function; tests/test_oracle_*.py pin every function.
  */
 #include "lgref.h"
 
