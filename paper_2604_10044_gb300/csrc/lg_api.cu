@@ -14,7 +14,7 @@ bool aligned16(const void *p) { return ((uintptr_t)p & 15u) == 0; }
 lg_status check_cache(const lg_cache *c) {
   if (!c || !c->k || !c->v || !c->seq_off || !c->cap || !c->len || !c->dev_status)
     return LG_ERR_INVALID_ARG;
-  if (!aligned16(c->k) || !aligned16(c->v)) return LG_ERR_INVALID_ARG;
+  if (!aligned16(c->k) || !aligned16(c->v) || !aligned16(c->sketch)) return LG_ERR_INVALID_ARG;
   if (c->dtype != LG_BF16 && c->dtype != LG_F32) return LG_ERR_UNSUPPORTED;
   if (c->d != 64 && c->d != 128) return LG_ERR_UNSUPPORTED;
   if (c->L < 1 || c->H_kv < 1 || c->batch < 1 || c->S_total < 1) return LG_ERR_INVALID_ARG;

@@ -637,28 +637,56 @@ __global__ void __launch_bounds__(kKeepThreads) keep_set_kernel(KeepArgs a) {
 
 constexpr int kCompactThreads = 256;
 constexpr int kCompactChunks = 4;  // 16-byte chunks per thread per tile
+constexpr int kCompactSeqList = 1024;  // pruned sequences listed in shared memory up to this batch
 
 // Stream (sequence b, one of 2*L*H_kv K/V streams or the sketch stream): slot j <- row kept[j]
-// for j >= j0, tiles in ascending order; CTAs take (sequence, stream) items grid-stride.  kept[] is strictly increasing with kept[j] >= j,
+// for j >= j0, tiles in ascending order; CTAs take (sequence, stream) items of the pruned
+// sequences grid-stride (each CTA first lists them from one pass over kept_count, so a step
+// that prunes nothing costs that pass).  kept[] is strictly increasing with kept[j] >= j,
 // so a tile reads only rows at or above its own first slot: once every load of the tile is
 // performed (the barrier) its stores cannot clobber a row another tile still needs.
 __global__ void __launch_bounds__(kCompactThreads) compact_kernel(lg_cache c,
                                                                   const int32_t *kept_idx,
                                                                   const int32_t *kept_count,
                                                                   int max_keep) {
-  const int tid = threadIdx.x;
+  __shared__ int s_seq[kCompactSeqList], s_cnt[kCompactSeqList];
+  __shared__ int s_wtot[kCompactThreads / 32];
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int row_bytes_kv = c.d * (c.dtype == LG_BF16 ? 2 : 4);
   const int nwords = c.H_kv * c.d / 32;
   const int n_kv = 2 * c.L * c.H_kv;
   const int per_seq = n_kv + 1;
-  // the first item's count is read together with the status word
-  const int cnt_first =
-      (int)blockIdx.x < c.batch * per_seq ? kept_count[blockIdx.x / per_seq] : -1;
+  // the pruned sequences and their counts, in sequence order (read before the status word)
+  const bool listed = c.batch <= kCompactSeqList;
+  int n_listed = 0;
+  if (listed) {
+    for (int b0 = 0; b0 < c.batch; b0 += kCompactThreads) {
+      const int b = b0 + tid;
+      const int k = b < c.batch ? kept_count[b] : -1;
+      const unsigned bal = __ballot_sync(0xffffffffu, k >= 0);
+      if (lane == 0) s_wtot[warp] = __popc(bal);
+      __syncthreads();
+      int at = n_listed, tot = 0;
+      for (int w = 0; w < kCompactThreads / 32; ++w) {
+        at += w < warp ? s_wtot[w] : 0;
+        tot += s_wtot[w];
+      }
+      if (k >= 0) {
+        at += __popc(bal & ((1u << lane) - 1u));
+        s_seq[at] = b;
+        s_cnt[at] = k;
+      }
+      n_listed += tot;
+      __syncthreads();
+    }
+  }
   if (cta_status_bad(c.dev_status)) return;
-  // grid-stride over (sequence, stream); sequences left as they were cost one load each
-  for (int item = blockIdx.x; item < c.batch * per_seq; item += gridDim.x) {
-    const int b = item / per_seq, stream = item - b * per_seq;
-    const int cnt = item == (int)blockIdx.x ? cnt_first : kept_count[b];
+  const int n_items = (listed ? n_listed : c.batch) * per_seq;
+  // grid-stride over (sequence, stream)
+  for (int item = blockIdx.x; item < n_items; item += gridDim.x) {
+    const int r = item / per_seq, stream = item - r * per_seq;
+    const int b = listed ? s_seq[r] : r;
+    const int cnt = listed ? s_cnt[r] : kept_count[b];
     if (cnt < 0) continue;
     unsigned char *base;
     int row_bytes;
