@@ -192,3 +192,10 @@ def test_bandwidth_sweep_full_size(cuda):
     """workload 5: 32 layers, 64/8 heads (GQA 8), b=16, n=131072, B=32768 (275 GB)"""
     w = synth.make_workload(5)
     assert run_full_size(w, cuda, n_groups=2, n_streams=2) == w.batch
+
+
+def test_paper_shaped_full_size(cuda):
+    """workload 6: the paper's setting at full size (28 layers, 16/8 heads, the 3853-row prompt,
+    B=1024): the first step's attention, detection on seeded statistics and the budget cut"""
+    w = synth.make_workload(6)
+    assert run_full_size(w, cuda, n_groups=4, n_streams=3) == w.batch
