@@ -608,16 +608,22 @@ def run_e2e(bench, K, ws, graphs=True):
     small_h = torch.empty(4 * w.batch, dtype=torch.int32).pin_memory()
     small_d = torch.empty(4 * w.batch, dtype=torch.int32, device=bench.dev)
 
-    def enqueue(t):
+    def copy_in(t):
         # H2D: this step's input variants into the device slots the harness reads
         for dst, src in pairs:
             dst[t].copy_(src[t], non_blocking=True)
-        bench.step(t)
+
+    def copy_out():
         out_h.copy_(g.out, non_blocking=True)
         small_d[:w.batch].copy_(g.flags)
         small_d[w.batch:3 * w.batch].copy_(g.spans.view(-1))
         small_d[3 * w.batch:].copy_(bench.cache.len)
         small_h.copy_(small_d, non_blocking=True)
+
+    def enqueue(t):
+        copy_in(t)
+        bench.step(t)
+        copy_out()
 
     def timed(run_step):
         bench.reset()
@@ -630,24 +636,42 @@ def run_e2e(bench, K, ws, graphs=True):
         return max_over_ranks(time.perf_counter() - t0, ws)
 
     dt_eager = timed(enqueue)
-    dt = dt_eager
+    dt = dt_graph = None
     if graphs:
+        # the step's kernels as one graph per step; the host copies stay stream copies (as
+        # graph nodes, copies from pinned host memory ran several times slower on this system)
         step_graphs = []
         for t in range(K):
             gr = torch.cuda.CUDAGraph()
             with torch.cuda.graph(gr, stream=bench.stream, capture_error_mode="thread_local"):
-                enqueue(t)
+                bench.step(t)
             step_graphs.append(gr)
-        dt = timed(lambda t: step_graphs[t].replay())
+        # one untimed replay of every graph first: the first launch of a graph uploads it
+        bench.reset()
+        for gr in step_graphs:
+            gr.replay()
+        torch.cuda.synchronize()
+
+        def graphed(t):
+            copy_in(t)
+            step_graphs[t].replay()
+            copy_out()
+        dt_graph = timed(graphed)
     h2d = sum(h[0].numel() * h.element_size() for _, h in pairs)
     d2h = out_h.numel() * out_h.element_size() + small_h.numel() * 4
-    line = {"value": round(sum_over_ranks(K, ws) / dt, 3), "unit": UNIT,
+    rate = lambda d: round(sum_over_ranks(K, ws) / d, 3) if d else None
+    # the faster of the two ways a serving loop can drive the calls (both reported)
+    use_graph = dt_graph is not None and dt_graph < dt_eager
+    line = {"value": rate(dt_graph if use_graph else dt_eager), "unit": UNIT,
             "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
-            "launch": "one CUDA graph per step (copies, guarded step, read-back), host waits "
-                      "for each step" if graphs else "eager, host waits for each step",
+            "launch": "stream copies in, the step's kernels as one CUDA graph, stream copies "
+                      "out; host waits for each step" if use_graph
+                      else "eager calls, host waits for each step",
+            "steps_per_s_eager": rate(dt_eager), "steps_per_s_graphed_kernels": rate(dt_graph),
             "note": "inputs of both sequence modes (loop continues / loop-free) copied every "
-                    "step; outputs, flags, spans and lengths read back every step"}
-    return line, round(sum_over_ranks(K, ws) / dt_eager, 3)
+                    "step; outputs, flags, spans and lengths read back every step; the faster "
+                    "of the two launch modes"}
+    return line, rate(dt_eager)
 
 
 # ------------------------------------------------------------------ CPU oracle arm
