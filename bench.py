@@ -69,6 +69,7 @@ def parse():
                          "print its measures instead of the step benchmark")
     ap.add_argument("--eager", action="store_true",
                     help="time the steps as eager launches instead of one CUDA graph replay")
+    ap.add_argument("--oracle-sample", type=int, default=0, help=argparse.SUPPRESS)
     ap.add_argument("--profile-steps", type=int, default=0,
                     help="run this many steps untimed and exit (for ncu launch lists)")
     return ap.parse_args()
@@ -713,7 +714,7 @@ def time_oracle(w, n_seq, n_layers, steps, warm=0):
     return run(steps)
 
 
-def cpu_baseline(w, target_s=15.0):
+def cpu_baseline(w, workload, target_s=15.0):
     """oracle time for one guarded step of a bounded sample: all layers of the first
     sequences, scaled to batch steps/s"""
     n_seq = 1
@@ -724,10 +725,27 @@ def cpu_baseline(w, target_s=15.0):
     n_seq = min(n_seq, w.batch)
     frac = n_seq / w.batch
     sec = sum(times)
-    return {"value": round(frac / sec, 6), "unit": UNIT, "cores": threads, "kind": "oracle",
-            "sample": "1 guarded decode step (step 1: attention over 8193 rows, detect, budget "
-                      "prune) of %d of the %d sequences, all %d layers; value = %d/%d batch "
-                      "steps / %.2f s" % (n_seq, w.batch, w.L, n_seq, w.batch, sec)}
+    line = {"value": round(frac / sec, 6), "unit": UNIT, "cores": threads, "kind": "oracle",
+            "sample": "1 guarded decode step (step 1: attention over the prompt's rows plus the "
+                      "new one, %d..%d, detect, budget prune) of %d of the %d sequences, all %d "
+                      "layers; value = %d/%d batch steps / %.2f s"
+                      % (int(w.n0.min()) + 1, int(w.n0.max()) + 1, n_seq, w.batch, w.L, n_seq,
+                         w.batch, sec)}
+    # the same step of one sequence on one thread, in a fresh interpreter (the oracle takes its
+    # thread count when it loads)
+    try:
+        env = dict(os.environ, OMP_NUM_THREADS="1")
+        r = subprocess.run([sys.executable, os.path.abspath(__file__), "--oracle-sample", "1",
+                            "--workload", str(workload)],
+                           env=env, capture_output=True, text=True, timeout=600)
+        one = json.loads(r.stdout.strip().splitlines()[-1])
+        line["single_thread"] = {"value": round(1.0 / w.batch / one["sec"], 6), "unit": UNIT,
+                                 "cores": one["threads"],
+                                 "sample": "the same step of 1 sequence on %d thread (%.2f s), "
+                                           "scaled to batch steps" % (one["threads"], one["sec"])}
+    except Exception as e:  # a reported extra: its failure leaves the main figure
+        line["single_thread"] = {"value": None, "error": str(e)[:200]}
+    return line
 
 
 def run_reference(args, ws, rank):
@@ -787,6 +805,12 @@ def run_ablation(args, local):
 
 def main():
     args = parse()
+    if args.oracle_sample:
+        # internal: one guarded step of the first sequences on this process's threads
+        w = synth.make_workload(args.workload)
+        times, threads = time_oracle(w, args.oracle_sample, w.L, 1)
+        print(json.dumps({"sec": sum(times), "threads": threads}), flush=True)
+        return
     ws, rank, local = dist_setup()
     if args.ablation:
         if rank == 0:
@@ -803,7 +827,7 @@ def main():
     line, w = res
     if rank == 0:
         if ws == 1 and not args.no_cpu_baseline:
-            line["cpu_baseline"] = cpu_baseline(w)
+            line["cpu_baseline"] = cpu_baseline(w, args.workload)
         print(json.dumps(line), flush=True)
 
 
