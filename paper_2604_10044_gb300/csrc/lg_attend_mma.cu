@@ -1,22 +1,25 @@
 // Decode attention over a bf16 KV cache fused with the guard's per-head statistics (LoopGuard
 // Sec. 3.1, Eq. 1; statistics read by Sec. 5.2), on tensor cores.
 //
-// Persistent CTAs (one per SM) take chunks from a shared counter, each a run of consecutive rows
-// of one (layer, sequence, kv-head), sized at launch from the lengths of the call (about eight
-// chunks per CTA).  A producer warp streams 128-row K and V tiles into a 3-stage
-// shared-memory ring with 2-D tensor copies (cp.async.bulk.tensor, 128-byte swizzle, one box
-// per 64 columns) completing on mbarriers.  Each of four consumer warps owns 32 rows of a tile
-// and all g query heads of the kv-head (padded to 8):
+// Persistent CTAs (one per SM) start on chunks blockIdx.x and blockIdx.x + gridDim.x and take
+// further chunks from a shared counter, each a run of consecutive rows of one (layer,
+// sequence, kv-head), sized in the kernel from the lengths of the call (6 to 16 chunks per
+// CTA).  A producer warp streams 128-row K and V tiles into a 3-stage shared-memory ring with
+// 2-D tensor copies (cp.async.bulk.tensor, 128-byte swizzle, one box per 64 columns)
+// completing on mbarriers.  Each of four consumer warps owns 32 rows of a tile and all g query
+// heads of the kv-head (padded to 8):
 //   S^T[16 rows x 8 heads] = K[16 x d] q^T      mma.sync m16n8k16 bf16 -> fp32, A by ldmatrix
 //   online softmax in log2 units on the accumulator fragments (exact running max per head)
 //   o^T[d x 8 heads] += V^T[d x 16 rows] P^T    A by ldmatrix.trans, B = P^T by movmatrix,
 //                                               P split into bf16 hi + lo (two MMAs)
 // The suffix mass, the entropy term and the normaliser accumulate beside the softmax.  At the
-// end of a chunk the four warps merge through shared memory into one partial per head
-// {M, l, u, sigma, o[d]} and hand the chunk to one of four merger warps, which count the
-// arrivals of each (layer, sequence, kv-head) group; the arrival that completes a group merges
-// the group's chunk partials into out and the statistics while the consumers go on streaming.  Rows past the end of a sequence (ragged last tile) are masked to zero
-// weight, and their stale V rows are zeroed in shared memory before the P.V product.
+// end of a chunk each warp leaves its own {M, l, u, sigma, o[d]} per head in a shared-memory
+// ticket buffer and goes on streaming (no barrier among the consumers); one of four merger
+// warps merges the four into the chunk's partial, counts the arrivals of its (layer,
+// sequence, kv-head) group, and the arrival that completes a group merges the group's chunk
+// partials into out and the statistics.  Rows past the end of a sequence (ragged last tile)
+// are masked to zero weight, and their stale V rows are zeroed in shared memory before the
+// P.V product.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 #include <cuda_bf16.h>
@@ -39,6 +42,7 @@ constexpr int kMergerWarp0 = kConsumerWarps + 1;
 constexpr int kMergers = 4;   // merger warps; ticket k goes to merger k % kMergers
 constexpr int kThreads = (kConsumerWarps + 1 + kMergers) * 32;
 constexpr int kTickets = 2 * kMergers;  // finished chunks queued from the consumers to the mergers
+                                        // (ticket k in slot k % kTickets, owned by merger k % 4)
 constexpr int kMaxChunkRows = 4096;  // chunk rows at most (the tail of a call is about one chunk)
 constexpr int kStagedSeqs = 256;     // lengths and offsets kept in shared memory up to this batch
 
@@ -48,11 +52,32 @@ struct MmaCfg {
   static constexpr int kStageBytes = 2 * kHalves * kBoxBytes;  // K and V
   static constexpr int kStages = D == 128 ? 3 : 6;
   static constexpr int kRingBytes = kStages * kStageBytes;
-  static constexpr int kMergeBytes = kConsumerWarps * 8 * D * 4 + kConsumerWarps * 8 * 4 * 4;
+  // ticket buffers: room for one buffer of 8 heads; fewer heads fit more buffers
+  static constexpr int kMergeBytes = kConsumerWarps * 8 * (D + 8) * 4;
   static constexpr int kQBytes = 8 * D * 2;  // a stage's query rows (up to 8 heads), bf16
   static constexpr int kSmem = kRingBytes + kMergeBytes + kStages * kQBytes + 1024;  // + slack
   static constexpr int kKSteps = D / 16;
 };
+
+// One ticket buffer: every consumer warp's chunk partial of the G real heads,
+// o as [warp][head][D + 4] (the padding spreads the fragment stores over all banks), then
+// {M, l, u, sigma} as [warp][head][4].
+template <int D, int G>
+struct TicketBuf {
+  static constexpr int kOStride = D + 4;
+  static constexpr int kFloats = kConsumerWarps * G * (kOStride + 4);
+  static constexpr int kFit = MmaCfg<D>::kMergeBytes / (kFloats * 4);
+  static constexpr int kBufs = kFit >= 8 ? 8 : (kFit >= 4 ? 4 : (kFit >= 2 ? 2 : 1));
+  static_assert(kFit >= 1, "ticket buffer larger than its shared-memory budget");
+};
+
+// group arrival count: release (this chunk's partial, stored by the warp before) and acquire
+// (the other chunks' partials, read by the arrival that completes the group) at GPU scope
+__device__ __forceinline__ int arrive_acq_rel(int *p) {
+  int old;
+  asm volatile("atom.acq_rel.gpu.global.add.s32 %0, [%1], 1;" : "=r"(old) : "l"(p) : "memory");
+  return old;
+}
 
 __device__ __forceinline__ void tma_load_2d(void *smem_dst, const CUtensorMap *map, int x, int y,
                                             uint64_t *bar) {
@@ -107,8 +132,11 @@ struct ChunkId {
 };
 
 // Chunk geometry of one call, from the lengths it attends over (the host sizes the workspace
-// for max_len, which can be far above them): chunk rows a multiple of the tile, about eight
-// chunks per CTA, and never more chunks per group than the workspace holds (max_chunks).
+// for max_len, which can be far above them): chunk rows a multiple of the tile, never more
+// chunks per group than the workspace holds (max_chunks).  A CTA takes about one chunk per
+// eight of its tiles, at least 6 (a chunk end costs the consumers a hand-off) and at most 16
+// (measured: finer chunks gained nothing at the end of long passes and cost a little on the
+// way); the rows are then evened out over the chunks of the longest group.
 struct Geom {
   int rows;     // rows per chunk
   int per_grp;  // chunk ids per (layer, sequence, kv-head)
@@ -117,16 +145,25 @@ struct Geom {
 
 __device__ __forceinline__ Geom make_geom(const AttendArgs &a, int n_max, int64_t len_sum,
                                           int ctas) {
-  const int64_t rows_all = len_sum * a.H_kv * a.n_layers;
-  const int64_t target = (int64_t)ctas * 8;
-  int64_t c = (rows_all + target - 1) / target;
-  const int64_t fit = (n_max + a.max_chunks - 1) / a.max_chunks;
-  c = min(c, (int64_t)kMaxChunkRows);
-  c = max(max(c, fit), (int64_t)kTile);
+  // the chunks per CTA and the rows they imply are a heuristic: float arithmetic (the same in
+  // every CTA) keeps 64-bit divisions off the prologue
+  const float rows_all = (float)len_sum * (float)(a.H_kv * a.n_layers);
+  const float per_cta =
+      fminf(fmaxf(floorf(rows_all / (float)(kTile * 8) / (float)ctas), 6.f), 16.f);
+  const float cf = ceilf(rows_all / ((float)ctas * per_cta));
+  int c = cf >= (float)kMaxChunkRows ? kMaxChunkRows : (int)cf;
+  const unsigned nm = (unsigned)n_max;
+  const int fit = (int)((nm + (unsigned)a.max_chunks - 1u) / (unsigned)a.max_chunks);
+  c = max(max(c, fit), kTile);
   c = (c + kTile - 1) / kTile * kTile;
+  // even rows: as many chunks per group, each about n_max / per_grp rows (no more chunks, so
+  // still within max_chunks)
+  const unsigned per = max(1u, (nm + (unsigned)c - 1u) / (unsigned)c);
+  c = (int)(((nm + per - 1u) / per + kTile - 1) / kTile * kTile);
+  c = max(c, kTile);
   Geom gm;
-  gm.rows = (int)c;
-  gm.per_grp = max(1, (int)((n_max + c - 1) / c));
+  gm.rows = c;
+  gm.per_grp = max(1, (int)((nm + (unsigned)c - 1u) / (unsigned)c));
   gm.total = a.n_layers * a.batch * a.H_kv * gm.per_grp;
   return gm;
 }
@@ -147,8 +184,8 @@ __device__ __forceinline__ ChunkId decode_chunk(const AttendArgs &a, int c, int 
 //   sigma = sum f_j sigma_j, o = sum f_j o_j / l
 // out = o, stats = {M ln 2, l, ln l - u ln 2 / l, sigma / l}.  The partials were written by
 // other CTAs of this launch: read through L2.  Lane j holds chunk j's {M, l, u, sigma} (up to
-// 32 chunks; more are read again per block), and the o slices of kBlk chunks are loaded with
-// them, so a head of a group of at most kBlk chunks costs one round trip.
+// 32 chunks; more are read again per block), and the o slices of up to eight chunks are loaded
+// with them, so a head of a group of at most eight chunks costs one round trip.
 template <int D, int G>
 __device__ __forceinline__ void merge_group(const AttendArgs &a, int64_t head0, int n,
                                             int chunk_rows, int lane) {
@@ -244,9 +281,12 @@ attend_mma_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant
   __shared__ int stage_tile[C::kStages];   // tile index within that chunk
   __shared__ int stage_n[C::kStages];      // the chunk's sequence length
   __shared__ long long stage_lrow0[C::kStages];  // its first row in the logits layout
-  __shared__ __align__(8) uint64_t tfull[kTickets];   // consumer -> merger: a finished chunk
-  __shared__ __align__(8) uint64_t tempty[kTickets];  // merger -> consumer: the slot is free
-  __shared__ int t_grp[kTickets], t_n[kTickets];      // its group (-1: no more) and length
+  using TB = TicketBuf<D, G>;
+  __shared__ __align__(8) uint64_t tfull[kTickets];   // consumers -> merger: a finished chunk
+  __shared__ __align__(8) uint64_t tempty[kTickets];  // merger -> consumers: the slot is free
+  __shared__ __align__(8) uint64_t bfree[TB::kBufs];  // merger -> consumers: the buffer is read
+  __shared__ int t_grp[kTickets], t_n[kTickets], t_ch[kTickets];  // group (-1: no more), length,
+                                                                   // chunk within the group
   __shared__ int red_max[kThreads / 32];
   __shared__ long long red_sum[kThreads / 32];
   __shared__ int s_len[kStagedSeqs];         // len[b] and seq_off[b] of a batch up to kStagedSeqs
@@ -254,14 +294,16 @@ attend_mma_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant
   __shared__ int s_bad;                      // the device status at entry (one read per CTA)
   unsigned char *smem = reinterpret_cast<unsigned char *>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  float *merge_o = reinterpret_cast<float *>(smem + C::kRingBytes);  // [warps][8][D]
-  unsigned char *qbuf = smem + C::kRingBytes + C::kMergeBytes;         // [stages][8][D] bf16
-  float *merge_s = merge_o + kConsumerWarps * 8 * D;                  // [warps][8][4]
+  float *tbuf = reinterpret_cast<float *>(smem + C::kRingBytes);  // [kBufs][TB::kFloats]
+  unsigned char *qbuf = smem + C::kRingBytes + C::kMergeBytes;      // [stages][8][D] bf16
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  // the first chunk claim and the length reads below are in flight together
-  int c_first = 0;
-  if (warp == kProducerWarp && lane == 0) c_first = atomicAdd(next_chunk, 1);
+  // CTA i starts on chunk i; later chunks come from the shared counter (offset by the grid)
+  if (warp == kProducerWarp && lane == 0) {
+    // the descriptors' fetch overlaps the prologue
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmK)) : "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmV)) : "memory");
+  }
   if (threadIdx.x == 0) {
     s_bad = status_bad(a.status);
     for (int s = 0; s < C::kStages; ++s) {
@@ -269,9 +311,10 @@ attend_mma_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant
       mbar_init(&empty_bar[s], kConsumerWarps);
     }
     for (int s = 0; s < kTickets; ++s) {
-      mbar_init(&tfull[s], 1);
+      mbar_init(&tfull[s], kConsumerWarps);
       mbar_init(&tempty[s], 1);
     }
+    for (int s = 0; s < TB::kBufs; ++s) mbar_init(&bfree[s], 1);
     mbar_fence_init();
   }
   {
@@ -310,10 +353,13 @@ attend_mma_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant
 
   if (warp >= kMergerWarp0) {
     // ------------------------------------------------------------ mergers
-    // One ticket per finished chunk, dealt round-robin to the merger warps.  The consumers'
-    // partial stores are ordered before the ticket (their barrier, the mbarrier's release and
-    // acquire); the fence makes them visible to the GPU before the group's arrival count
-    // moves, and the arrival that completes the group (acquire fence after it) reads every
+    // One ticket per finished chunk, dealt round-robin to the merger warps; ticket k's warp
+    // partials are in buffer k % kBufs.  The merger folds the four into the chunk's partial
+    // {M, l, u, sigma, o} (global, read by the group's last arrival), frees the buffer, and
+    // counts the arrival.  The consumers' buffer stores are ordered before the ticket (each
+    // warp's __syncwarp and mbarrier release, the merger's acquire); the arrival count is an
+    // acquire-release atomic at GPU scope after the warp's __syncwarp, so the chunk partial is
+    // visible before the count moves, and the arrival that completes the group reads every
     // chunk partial of the group.
     for (uint32_t tk = warp - kMergerWarp0;; tk += kMergers) {
       const int slot = tk % kTickets;
@@ -321,21 +367,58 @@ attend_mma_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant
         set_status(a.status, LG_ERR_TIMEOUT);
         return;
       }
-      const int grp = t_grp[slot], n = t_n[slot];
+      const int grp = t_grp[slot], n = t_n[slot], ch = t_ch[slot];
       __syncwarp();
       if (lane == 0) mbar_arrive(&tempty[slot]);
       if (grp < 0) break;
+      const int64_t head0 = (int64_t)(grp / a.H_kv) * a.H_q + (int64_t)(grp % a.H_kv) * G;
+      {
+        const float *ob = tbuf + (size_t)(tk % TB::kBufs) * TB::kFloats;
+        const float *sb = ob + kConsumerWarps * G * TB::kOStride;
+#pragma unroll 1
+        for (int h = 0; h < G; ++h) {
+          float4 ws[kConsumerWarps];
+          float M = -INFINITY;
+#pragma unroll
+          for (int w = 0; w < kConsumerWarps; ++w) {
+            ws[w] = *reinterpret_cast<const float4 *>(sb + (w * G + h) * 4);
+            M = fmaxf(M, ws[w].x);
+          }
+          float f[kConsumerWarps], l = 0.f, u = 0.f, sg = 0.f;
+#pragma unroll
+          for (int w = 0; w < kConsumerWarps; ++w) {
+            // a warp that saw no row of this chunk has l = 0, M = -inf and no weight
+            f[w] = 0.f;
+            if (ws[w].y > 0.f) {
+              f[w] = exp2f(ws[w].x - M);
+              l += f[w] * ws[w].y;
+              u += f[w] * (ws[w].z + (ws[w].x - M) * ws[w].y);
+              sg += f[w] * ws[w].w;
+            }
+          }
+          float *pp = a.partial + ((head0 + h) * a.max_chunks + ch) * (D + 8);
+#pragma unroll
+          for (int k = 0; k < D / 32; ++k) {
+            const int e = lane + 32 * k;
+            float ov = 0.f;
+#pragma unroll
+            for (int w = 0; w < kConsumerWarps; ++w)
+              ov += f[w] * ob[(w * G + h) * TB::kOStride + e];
+            pp[8 + e] = ov;
+          }
+          if (lane == 0) *reinterpret_cast<float4 *>(pp) = make_float4(M, l, u, sg);
+        }
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&bfree[tk % TB::kBufs]);
       int last = 0;
       if (lane == 0) {
-        __threadfence();
         const int nch = (n + gm.rows - 1) / gm.rows;
-        last = atomicAdd(a.counter + 1 + grp, 1) == nch - 1;
+        last = arrive_acq_rel(a.counter + 1 + grp) == nch - 1;
       }
       last = __shfl_sync(0xffffffffu, last, 0);
-      __syncwarp();
+      __syncwarp();  // the lanes' partial reads follow lane 0's acquire
       if (last) {
-        __threadfence();
-        const int64_t head0 = (int64_t)(grp / a.H_kv) * a.H_q + (int64_t)(grp % a.H_kv) * G;
         merge_group<D, G>(a, head0, n, gm.rows, lane);
       }
     }
@@ -344,21 +427,24 @@ attend_mma_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant
 
   if (warp == kProducerWarp) {
     // ------------------------------------------------------------ producer
-    // Chunks are taken from a shared counter (ragged lengths balance across CTAs), one claim
-    // ahead so that its round trip overlaps the current chunk; each stage carries its chunk,
+    // A CTA's first two chunks are blockIdx.x and blockIdx.x + gridDim.x; later ones come from
+    // a shared counter (ragged lengths balance across CTAs), each claimed as its predecessor
+    // starts (one ahead: the claim's round trip overlaps a chunk, and a CTA near the end of the
+    // pass holds at most one chunk it has not started); each stage carries its chunk,
     // tile index, length and logits row to the consumers, and a chunk's first stage also
     // brings the chunk's query rows (one bulk copy on the same barrier).
     if (lane == 0) {
-      asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmK)) : "memory");
-      asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmV)) : "memory");
       uint32_t it = 0;
-      int c = c_first;
+      const int claimed0 = 2 * (int)gridDim.x;
+      int c = blockIdx.x;
+      bool first = true;
       while (true) {
         const bool alive = c < gm.total;
         int ntiles = 0, grow = 0, n = 0, c_next = 0;
         int64_t lrow0 = 0, head0 = 0;
         if (alive) {
-          c_next = atomicAdd(next_chunk, 1);
+          c_next = first ? (int)(blockIdx.x + gridDim.x) : claimed0 + atomicAdd(next_chunk, 1);
+          first = false;
           const ChunkId id = decode_chunk(a, c, gm.per_grp);
           n = staged ? s_len[id.b] : a.len[id.b];
           const int64_t off = staged ? s_off[id.b] : a.seq_off[id.b];
@@ -428,8 +514,8 @@ attend_mma_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant
   float o[C::kKSteps][4];
   float m2[2], l2[2], u2[2], sg2[2];
   float *logits = a.logits;
-  uint32_t tk = 0;        // tickets issued (thread 0)
-  bool handoff = true;    // false once a ticket slot was not released in time (thread 0)
+  uint32_t tk = 0;        // tickets issued (the same count in every consumer warp)
+  bool handoff = true;    // false once a buffer or ticket slot was not released in time
   for (uint32_t it = 0;; ++it) {
     const int st = it % C::kStages;
     if (!mbar_wait(&full_bar[st], (it / C::kStages) & 1)) {
@@ -585,7 +671,8 @@ attend_mma_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant
     if (lane == 0) mbar_arrive(&empty_bar[st]);
     if (t != ntiles - 1) continue;
 
-    // ---------------------------------------------------------- chunk done: merge the warps
+    // ---------------------------------------------------------- chunk done: hand it off
+    // This warp's sums over its rows (lanes of one t4 hold the rows g, g + 8 of a head pair).
 #pragma unroll
     for (int h = 0; h < 2; ++h) {
 #pragma unroll
@@ -595,77 +682,69 @@ attend_mma_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant
         sg2[h] += __shfl_xor_sync(0xffffffffu, sg2[h], off);
       }
     }
-    float *mo = merge_o + (size_t)warp * 8 * D;
-#pragma unroll
-    for (int eb = 0; eb < C::kKSteps; ++eb) {
-      const int e = eb * 16 + g;
-      mo[(2 * t4) * D + e] = o[eb][0];
-      mo[(2 * t4 + 1) * D + e] = o[eb][1];
-      mo[(2 * t4) * D + e + 8] = o[eb][2];
-      mo[(2 * t4 + 1) * D + e + 8] = o[eb][3];
+    if (!handoff) continue;
+    const int buf = tk % TB::kBufs, slot = tk % kTickets;
+    int ok = 1;
+    if (lane == 0) {
+      // the buffer's previous ticket has been read by its merger (so every warp has arrived on
+      // every ticket up to kBufs <= kTickets back, and this arrival counts toward this ticket);
+      // warp 0 also waits for the ticket slot before writing its group, length and chunk
+      if (tk >= (uint32_t)TB::kBufs && !mbar_wait(&bfree[buf], ((tk / TB::kBufs) - 1) & 1))
+        ok = 0;
+      if (ok && warp == 0) {
+        if (tk >= (uint32_t)kTickets && !mbar_wait(&tempty[slot], ((tk / kTickets) - 1) & 1)) {
+          ok = 0;
+        } else {
+          t_grp[slot] = (int)(((int64_t)id.lloc * a.batch + id.b) * a.H_kv + id.kvh);
+          t_n[slot] = n;
+          t_ch[slot] = id.ch;
+        }
+      }
+      if (!ok) set_status(a.status, LG_ERR_TIMEOUT);
     }
-    if (g == 0) {
+    if (!__shfl_sync(0xffffffffu, ok, 0)) {
+      handoff = false;
+      continue;
+    }
+    __syncwarp();  // the lanes' stores below follow lane 0's wait
+    {
+      // o^T fragments: this thread holds o[e][2 t4 + h2] for e = 16 eb + g (+8)
+      float *ob = tbuf + (size_t)buf * TB::kFloats + warp * G * TB::kOStride;
+      float *sb =
+          tbuf + (size_t)buf * TB::kFloats + kConsumerWarps * G * TB::kOStride + warp * G * 4;
 #pragma unroll
-      for (int h = 0; h < 2; ++h) {
-        float *ms = merge_s + ((size_t)warp * 8 + 2 * t4 + h) * 4;
-        ms[0] = m2[h];
-        ms[1] = l2[h];
-        ms[2] = u2[h];
-        ms[3] = sg2[h];
+      for (int h2 = 0; h2 < 2; ++h2) {
+        const int h = 2 * t4 + h2;
+        if (h < G) {
+#pragma unroll
+          for (int eb = 0; eb < C::kKSteps; ++eb) {
+            ob[h * TB::kOStride + eb * 16 + g] = o[eb][h2];
+            ob[h * TB::kOStride + eb * 16 + g + 8] = o[eb][h2 + 2];
+          }
+          if (g == 0)
+            *reinterpret_cast<float4 *>(sb + h * 4) = make_float4(m2[h2], l2[h2], u2[h2], sg2[h2]);
+        }
       }
     }
-    asm volatile("bar.sync 1, %0;" ::"n"(kConsumerWarps * 32) : "memory");
-    const int64_t pbase = ((int64_t)id.lloc * a.batch + id.b) * a.H_q + (int64_t)id.kvh * G;
-    for (int idx = threadIdx.x; idx < G * D; idx += kConsumerWarps * 32) {
-      const int h = idx / D, e = idx % D;
-      float M = -INFINITY;
-#pragma unroll
-      for (int w = 0; w < kConsumerWarps; ++w) M = fmaxf(M, merge_s[(w * 8 + h) * 4]);
-      float ov = 0.f, l = 0.f, u = 0.f, sg = 0.f;
-#pragma unroll
-      for (int w = 0; w < kConsumerWarps; ++w) {
-        const float *ms = merge_s + (w * 8 + h) * 4;
-        if (!(ms[1] > 0.f)) continue;  // warp saw no row of this chunk
-        const float f = exp2f(ms[0] - M);
-        ov += f * merge_o[((size_t)w * 8 + h) * D + e];
-        l += f * ms[1];
-        u += f * (ms[2] + (ms[0] - M) * ms[1]);
-        sg += f * ms[3];
-      }
-      float *pp = a.partial + ((pbase + h) * a.max_chunks + id.ch) * (D + 8);
-      pp[8 + e] = ov;
-      if (e == 0) {
-        pp[0] = M;
-        pp[1] = l;
-        pp[2] = u;
-        pp[3] = sg;
-      }
-    }
-    // every partial store of the chunk is done: hand the chunk to the merger warp
-    asm volatile("bar.sync 1, %0;" ::"n"(kConsumerWarps * 32) : "memory");
-    if (threadIdx.x == 0 && handoff) {
-      const int slot = tk % kTickets;
-      if (tk >= (uint32_t)kTickets && !mbar_wait(&tempty[slot], ((tk / kTickets) - 1) & 1)) {
-        set_status(a.status, LG_ERR_TIMEOUT);
-        handoff = false;
-      } else {
-        t_grp[slot] = (int)(((int64_t)id.lloc * a.batch + id.b) * a.H_kv + id.kvh);
-        t_n[slot] = n;
-        mbar_arrive(&tfull[slot]);
-        ++tk;
-      }
-    }
+    __syncwarp();
+    if (lane == 0) mbar_arrive(&tfull[slot]);
+    ++tk;
   }
-  if (threadIdx.x == 0 && handoff) {
-    // no more chunks: one last ticket for each merger
+  if (handoff && lane == 0) {
+    // no more chunks: one last ticket for each merger (no buffer).  Every warp first waits for
+    // the slot's previous ticket to be taken, so that its arrival cannot count toward a ticket
+    // another warp has not finished (end tickets follow no buffer wait)
     for (int m = 0; m < kMergers; ++m, ++tk) {
       const int slot = tk % kTickets;
       if (tk >= (uint32_t)kTickets && !mbar_wait(&tempty[slot], ((tk / kTickets) - 1) & 1)) {
         set_status(a.status, LG_ERR_TIMEOUT);
         break;
       }
-      t_grp[slot] = -1;
-      t_n[slot] = 0;
+      if (warp == 0) {
+        t_grp[slot] = -1;
+        t_n[slot] = 0;
+        t_ch[slot] = 0;
+      }
       mbar_arrive(&tfull[slot]);
     }
   }
