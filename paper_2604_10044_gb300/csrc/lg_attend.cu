@@ -70,6 +70,7 @@ __device__ __forceinline__ float2 ffma2(float2 a, float2 b, float2 c) { return _
 template <typename T, int D, int G>
 __global__ void __launch_bounds__(AttendCfg<T, D, G>::kThreads)
 attend_partial_kernel(AttendArgs a) {
+  pdl_enter();
   using C = AttendCfg<T, D, G>;
   extern __shared__ __align__(128) unsigned char smem[];
   __shared__ __align__(8) uint64_t full_bar[C::kStages];
@@ -286,6 +287,7 @@ attend_partial_kernel(AttendArgs a) {
 // statistics {m, l, H, S} in natural units.  One warp per head, eight heads per block.
 template <typename T, int D>
 __global__ void attend_combine_kernel(AttendArgs a, void *out, float *stats, float *final_ml) {
+  pdl_enter();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int64_t head = (int64_t)blockIdx.x * (blockDim.x >> 5) + warp;
   if (head >= (int64_t)a.n_layers * a.batch * a.H_q) return;
@@ -340,6 +342,7 @@ __global__ void attend_combine_kernel(AttendArgs a, void *out, float *stats, flo
 // kept by the partial pass and the merged (M, l) of every head.
 template <int G>
 __global__ void h2o_accumulate_kernel(AttendArgs a, float *h2o, const float *final_ml) {
+  pdl_enter();
   const int kvh = blockIdx.y, b = blockIdx.z % a.batch, lloc = blockIdx.z / a.batch;
   const int layer = a.layer0 + lloc;
   if (status_bad(a.status)) return;
@@ -379,21 +382,21 @@ static cudaError_t launch_typed(const AttendArgs &a, int64_t rows_total, void *o
     e = cudaFuncSetAttribute(kp, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmem);
     if (e != cudaSuccess) return e;
     dim3 grid(a.max_chunks, a.H_kv, a.n_layers * a.batch);
-    kp<<<grid, C::kThreads, C::kSmem, s>>>(a);
+    LG_TRY(launch_pdl(kp, grid, C::kThreads, C::kSmem, s, a));
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
   }
   if (Elem<T>::kDtype != LG_BF16) {
     // the tensor-core pass merges its chunk partials itself
     const int64_t heads = (int64_t)a.n_layers * a.batch * a.H_q;
-    attend_combine_kernel<T, D><<<(unsigned)((heads + 7) / 8), 256, 0, s>>>(a, out, stats,
-                                                                            final_ml);
+    LG_TRY(launch_pdl(attend_combine_kernel<T, D>, (unsigned)((heads + 7) / 8), 256, 0, s, a, out,
+                      stats, final_ml));
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
   }
   if (h2o) {
     int gx = (a.max_len + 255) / 256;
     if (gx > 64) gx = 64;
-    h2o_accumulate_kernel<G><<<dim3(gx, a.H_kv, a.n_layers * a.batch), 256, 0, s>>>(a, h2o,
-                                                                                   final_ml);
+    LG_TRY(launch_pdl(h2o_accumulate_kernel<G>, dim3(gx, a.H_kv, a.n_layers * a.batch), 256, 0, s,
+                      a, h2o, final_ml));
     e = cudaGetLastError();
   }
   return e;

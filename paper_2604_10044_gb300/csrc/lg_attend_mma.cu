@@ -304,6 +304,7 @@ attend_mma_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmK)) : "memory");
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmV)) : "memory");
   }
+  pdl_enter();  // the tensormap prefetch above reads only the kernel's parameters
   if (threadIdx.x == 0) {
     s_bad = status_bad(a.status);
     for (int s = 0; s < C::kStages; ++s) {
@@ -750,6 +751,13 @@ attend_mma_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant
   }
 }
 
+// The call's chunk and group counters to zero: a kernel rather than a memset, so that the pass
+// after it keeps its programmatic launch edge.
+__global__ void zero_counters_kernel(int *p, int n) {
+  pdl_enter();
+  for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < n; i += gridDim.x * blockDim.x) p[i] = 0;
+}
+
 // ------------------------------------------------------------------ host side
 
 namespace {
@@ -787,7 +795,7 @@ cudaError_t launch_mma_typed(const CUtensorMap &mk, const CUtensorMap &mv, const
   cudaError_t e =
       cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, MmaCfg<D>::kSmem);
   if (e != cudaSuccess) return e;
-  kern<<<grid, kThreads, MmaCfg<D>::kSmem, s>>>(mk, mv, a, counter);
+  LG_TRY(launch_pdl(kern, grid, kThreads, MmaCfg<D>::kSmem, s, mk, mv, a, counter));
   return cudaGetLastError();
 }
 
@@ -825,7 +833,12 @@ cudaError_t launch_attend_mma_partial(const AttendArgs &a, int d, int g, int64_t
   const int grid = total < sms ? total : sms;
   if (!a.counter) return cudaErrorInvalidValue;
   const size_t counters = (size_t)(1 + (int64_t)a.n_layers * a.batch * a.H_kv) * sizeof(int);
-  if ((e = cudaMemsetAsync(a.counter, 0, counters, s)) != cudaSuccess) return e;
+  {
+    const int n = (int)(counters / sizeof(int));
+    const int blocks = (n + 255) / 256 < sms ? (n + 255) / 256 : sms;
+    if ((e = launch_pdl(zero_counters_kernel, blocks, 256, 0, s, a.counter, n)) != cudaSuccess)
+      return e;
+  }
   if (d == 128) return launch_mma_d<128>(mk, mv, a, g, grid, a.counter, s);
   if (d == 64) return launch_mma_d<64>(mk, mv, a, g, grid, a.counter, s);
   return cudaErrorInvalidValue;

@@ -12,6 +12,43 @@ namespace lg {
 // A bounded wait gives up after this many nanoseconds of %globaltimer.
 constexpr uint64_t kWaitLimitNs = 2000000000ull;
 
+// Programmatic dependent launch (sm_90 and later).  Every kernel of the library is launched
+// with programmatic stream serialization (launch_pdl below), so it may be scheduled while the
+// kernel before it in the stream is still running.  Each kernel therefore starts with
+// pdl_enter(): griddepcontrol.wait returns once the kernels it depends on have completed and
+// their memory is visible (at once when there is no such kernel), so nothing of the kernel
+// touches global memory before its predecessor is done; launch_dependents then lets the
+// next kernel be scheduled early in turn, and it waits the same way.  Completion is
+// transitive: the predecessor itself passed its wait only after its own predecessor was done.
+__device__ __forceinline__ void pdl_enter() {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
+// Returns the error of a launch or call from the enclosing cudaError_t function.
+#define LG_TRY(x)                                   \
+  do {                                              \
+    const cudaError_t lg_try_e_ = (x);              \
+    if (lg_try_e_ != cudaSuccess) return lg_try_e_; \
+  } while (0)
+
+// Launch with programmatic stream serialization (see pdl_enter).
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                              cudaStream_t s, Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, args...);
+}
+
 __device__ __forceinline__ void set_status(int32_t *status, int code) {
   if (status) atomicCAS(status, 0, code);
 }

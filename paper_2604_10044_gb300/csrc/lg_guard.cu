@@ -16,6 +16,7 @@ namespace lg {
 // (Here and in append_kernel the inputs are read before the status word, so that every load
 // of a thread is in flight at once; neither kernel has a barrier after its status check.)
 __global__ void begin_step_kernel(lg_cache c) {
+  pdl_enter();
   const int b = blockIdx.x * blockDim.x + threadIdx.x;
   if (b >= c.batch) return;
   const int n = c.len[b], cap = c.cap[b];
@@ -47,6 +48,7 @@ template <typename T>
 __global__ void append_kernel(lg_cache c, int layer0, int n_layers, const uint4 *k_new,
                               const uint4 *v_new, const int32_t *pos_new, int row_blocks,
                               int lguard) {
+  pdl_enter();
   if ((int)blockIdx.x >= row_blocks) {
     const int b = blockIdx.x - row_blocks;
     const int nwords = c.H_kv * c.d / 32;
@@ -87,6 +89,7 @@ __global__ void append_kernel(lg_cache c, int layer0, int n_layers, const uint4 
 // sketches of rows [0, len[b]) of the guard layer, read from the cache
 template <typename T>
 __global__ void sketch_build_kernel(lg_cache c, int guard_layer, int max_len) {
+  pdl_enter();
   const int b = blockIdx.y;
   if (status_bad(c.dev_status)) return;
   const int n = c.len[b];
@@ -107,6 +110,7 @@ __global__ void sketch_build_kernel(lg_cache c, int guard_layer, int max_len) {
 }
 
 __global__ void state_init_kernel(int batch, lg_guard_state *state, int t_gen0) {
+  pdl_enter();
   const int b = blockIdx.x * blockDim.x + threadIdx.x;
   if (b >= batch) return;
   lg_guard_state s;
@@ -293,6 +297,7 @@ constexpr int kStatWarps = 3;  // warps that sum the statistics in fp64 (one per
 // nwords + 1 words (rows that different lanes read fall in different banks), one warp scans
 // each window row, one warp each period.
 __global__ void __launch_bounds__(kDetectThreads, 1) detect_kernel(DetectArgs a) {
+  pdl_enter();
   extern __shared__ __align__(16) uint32_t sk_s[];
   __shared__ double red_e[kStatWarps], red_l[kStatWarps];
   __shared__ int w_latest[kDetectWarps], w_nov[kDetectWarps], w_nov_tail[kDetectWarps],
@@ -620,6 +625,7 @@ struct KeepArgs {
 constexpr int kKeepThreads = 1024;
 
 __global__ void __launch_bounds__(kKeepThreads) keep_set_kernel(KeepArgs a) {
+  pdl_enter();
   const int b = blockIdx.x, tid = threadIdx.x;
   const int32_t *status = a.c.dev_status;
   const int n = a.c.len[b];
@@ -649,6 +655,7 @@ __global__ void __launch_bounds__(kCompactThreads) compact_kernel(lg_cache c,
                                                                   const int32_t *kept_idx,
                                                                   const int32_t *kept_count,
                                                                   int max_keep) {
+  pdl_enter();
   __shared__ int s_seq[kCompactSeqList], s_cnt[kCompactSeqList];
   __shared__ int s_wtot[kCompactThreads / 32];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -746,6 +753,7 @@ __global__ void __launch_bounds__(kCompactThreads) compact_kernel(lg_cache c,
 // ------------------------------------------------------------------ H2O comparator
 
 __global__ void h2o_reset_kernel(lg_cache c, int max_len) {
+  pdl_enter();
   const int lh = blockIdx.y, b = blockIdx.z;
   const int n = min(c.len[b], max_len);
   const int64_t o = (int64_t)lh * c.S_total + c.seq_off[b];
@@ -774,6 +782,7 @@ template <int kMode>
 __global__ void __launch_bounds__(kH2OThreads) evict_kernel(lg_cache c, const int32_t *budget,
                                                             const int32_t *pos_now, int max_len,
                                                             int n_sink) {
+  pdl_enter();
   __shared__ unsigned long long s_min;
   __shared__ int s_slot, s_count, s_out;
   __shared__ unsigned int hist[256];
@@ -936,6 +945,7 @@ __global__ void __launch_bounds__(kH2OThreads) evict_kernel(lg_cache c, const in
 }
 
 __global__ void h2o_len_kernel(lg_cache c, const int32_t *budget) {
+  pdl_enter();
   const int b = blockIdx.x * blockDim.x + threadIdx.x;
   if (b >= c.batch || status_bad(c.dev_status)) return;
   if (c.len[b] > budget[b]) c.len[b] = budget[b];
@@ -944,7 +954,7 @@ __global__ void h2o_len_kernel(lg_cache c, const int32_t *budget) {
 // ------------------------------------------------------------------ launchers
 
 cudaError_t launch_begin_step(const lg_cache &c, cudaStream_t s) {
-  begin_step_kernel<<<(c.batch + 127) / 128, 128, 0, s>>>(c);
+  LG_TRY(launch_pdl(begin_step_kernel, (c.batch + 127) / 128, 128, 0, s, c));
   return cudaGetLastError();
 }
 
@@ -957,13 +967,13 @@ cudaError_t launch_append(const lg_cache &c, int layer0, int n_layers, const voi
   const bool sk = c.sketch && guard_layer >= layer0 && guard_layer < layer0 + n_layers;
   const int grid = row_blocks + (sk ? c.batch : 0);
   if (c.dtype == LG_BF16) {
-    append_kernel<__nv_bfloat16><<<grid, 256, 0, s>>>(c, layer0, n_layers, (const uint4 *)k_new,
-                                                      (const uint4 *)v_new, pos_new, row_blocks,
-                                                      guard_layer - layer0);
+    LG_TRY(launch_pdl(append_kernel<__nv_bfloat16>, grid, 256, 0, s, c, layer0, n_layers,
+                      (const uint4 *)k_new, (const uint4 *)v_new, pos_new, row_blocks,
+                      guard_layer - layer0));
   } else {
-    append_kernel<float><<<grid, 256, 0, s>>>(c, layer0, n_layers, (const uint4 *)k_new,
-                                              (const uint4 *)v_new, pos_new, row_blocks,
-                                              guard_layer - layer0);
+    LG_TRY(launch_pdl(append_kernel<float>, grid, 256, 0, s, c, layer0, n_layers,
+                      (const uint4 *)k_new, (const uint4 *)v_new, pos_new, row_blocks,
+                      guard_layer - layer0));
   }
   return cudaGetLastError();
 }
@@ -976,15 +986,16 @@ cudaError_t launch_sketch_build(const lg_cache &c, int guard_layer, int max_len,
   if (gx < 1) gx = 1;
   dim3 grid(gx, c.batch);
   if (c.dtype == LG_BF16) {
-    sketch_build_kernel<__nv_bfloat16><<<grid, 256, 0, s>>>(c, guard_layer, max_len);
+    LG_TRY(launch_pdl(sketch_build_kernel<__nv_bfloat16>, grid, 256, 0, s, c, guard_layer,
+                      max_len));
   } else {
-    sketch_build_kernel<float><<<grid, 256, 0, s>>>(c, guard_layer, max_len);
+    LG_TRY(launch_pdl(sketch_build_kernel<float>, grid, 256, 0, s, c, guard_layer, max_len));
   }
   return cudaGetLastError();
 }
 
 cudaError_t launch_state_init(const lg_cache &c, lg_guard_state *state, int t_gen0, cudaStream_t s) {
-  state_init_kernel<<<(c.batch + 127) / 128, 128, 0, s>>>(c.batch, state, t_gen0);
+  LG_TRY(launch_pdl(state_init_kernel, (c.batch + 127) / 128, 128, 0, s, c.batch, state, t_gen0));
   return cudaGetLastError();
 }
 
@@ -1014,7 +1025,7 @@ cudaError_t launch_detect(const lg_cache &c, const float *stats, int H_q, lg_gua
   cudaError_t e = cudaFuncSetAttribute(detect_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)smem);
   if (e != cudaSuccess) return e;
-  detect_kernel<<<c.batch, kDetectThreads, smem, s>>>(a);
+  LG_TRY(launch_pdl(detect_kernel, c.batch, kDetectThreads, smem, s, a));
   return cudaGetLastError();
 }
 
@@ -1033,7 +1044,7 @@ cudaError_t launch_prune_compact(const lg_cache &c, const int32_t *flags, const 
   a.kept_count = kept_count;
   a.max_keep = max_keep;
   a.max_len = max_len;
-  keep_set_kernel<<<c.batch, kKeepThreads, 0, s>>>(a);
+  LG_TRY(launch_pdl(keep_set_kernel, c.batch, kKeepThreads, 0, s, a));
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   return launch_compact(c, kept_idx, kept_count, max_keep, s);
@@ -1046,7 +1057,8 @@ cudaError_t launch_compact(const lg_cache &c, const int32_t *kept_idx, const int
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   const int items = c.batch * (2 * c.L * c.H_kv + 1);
   const int grid = items < 4 * sms ? items : 4 * sms;
-  compact_kernel<<<grid, kCompactThreads, 0, s>>>(c, kept_idx, kept_count, max_keep);
+  LG_TRY(launch_pdl(compact_kernel, grid, kCompactThreads, 0, s, c, kept_idx, kept_count,
+                    max_keep));
   return cudaGetLastError();
 }
 
@@ -1054,17 +1066,17 @@ cudaError_t launch_h2o_reset(const lg_cache &c, int max_len, cudaStream_t s) {
   int gx = (max_len + 255) / 256;
   if (gx > 256) gx = 256;
   if (gx < 1) gx = 1;
-  h2o_reset_kernel<<<dim3(gx, c.L * c.H_kv, c.batch), 256, 0, s>>>(c, max_len);
+  LG_TRY(launch_pdl(h2o_reset_kernel, dim3(gx, c.L * c.H_kv, c.batch), 256, 0, s, c, max_len));
   return cudaGetLastError();
 }
 
 cudaError_t launch_h2o_evict(const lg_cache &c, const int32_t *budget, const int32_t *pos_now,
                              int max_len, cudaStream_t s) {
-  evict_kernel<kEvictH2O><<<dim3(c.L * c.H_kv, c.batch), kH2OThreads, 0, s>>>(c, budget, pos_now,
-                                                                             max_len, 0);
+  LG_TRY(launch_pdl(evict_kernel<kEvictH2O>, dim3(c.L * c.H_kv, c.batch), kH2OThreads, 0, s, c,
+                    budget, pos_now, max_len, 0));
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
-  h2o_len_kernel<<<(c.batch + 127) / 128, 128, 0, s>>>(c, budget);
+  LG_TRY(launch_pdl(h2o_len_kernel, (c.batch + 127) / 128, 128, 0, s, c, budget));
   return cudaGetLastError();
 }
 
@@ -1075,11 +1087,11 @@ namespace lg {
 cudaError_t launch_streaming_evict(const lg_cache &c, const int32_t *budget,
                                    const int32_t *pos_now, int n_sink, int max_len,
                                    cudaStream_t s) {
-  evict_kernel<kEvictStreaming><<<dim3(c.L * c.H_kv, c.batch), kH2OThreads, 0, s>>>(
-      c, budget, pos_now, max_len, n_sink);
+  LG_TRY(launch_pdl(evict_kernel<kEvictStreaming>, dim3(c.L * c.H_kv, c.batch), kH2OThreads, 0, s,
+                    c, budget, pos_now, max_len, n_sink));
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
-  h2o_len_kernel<<<(c.batch + 127) / 128, 128, 0, s>>>(c, budget);
+  LG_TRY(launch_pdl(h2o_len_kernel, (c.batch + 127) / 128, 128, 0, s, c, budget));
   return cudaGetLastError();
 }
 

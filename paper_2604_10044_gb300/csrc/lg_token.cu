@@ -66,6 +66,7 @@ __device__ __forceinline__ int block_max(int v, int *red, int lane, int warp) {
 }
 
 __global__ void __launch_bounds__(kTokThreads, 1) token_detect_kernel(TokenArgs a) {
+  pdl_enter();
   extern __shared__ __align__(16) int32_t sm[];
   __shared__ int red[kTokWarps];
   __shared__ int w_latest[kTokWarps], w_nov[kTokWarps], w_tail[kTokWarps], w_pstar[kTokWarps],
@@ -333,7 +334,7 @@ cudaError_t launch_token_detect(const lg_cache &c, const int32_t *tokens, const 
   cudaError_t e = cudaFuncSetAttribute(token_detect_kernel,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
-  token_detect_kernel<<<c.batch, kTokThreads, smem, s>>>(a);
+  LG_TRY(launch_pdl(token_detect_kernel, c.batch, kTokThreads, smem, s, a));
   return cudaGetLastError();
 }
 
