@@ -356,8 +356,10 @@ class Guard:
         self.n_layers_per_call = n_layers_per_call or cache.L
         L, b = cache.L, cache.batch
         self.state = torch.zeros((b, STATE_BYTES // 4), dtype=torch.int32, device=dev)
-        self.flags = torch.zeros(b, dtype=torch.int32, device=dev)
-        self.spans = torch.zeros((b, 2), dtype=torch.int32, device=dev)
+        # flags and spans side by side (one read-back of a step's decisions)
+        self.flags_spans = torch.zeros(3 * b, dtype=torch.int32, device=dev)
+        self.flags = self.flags_spans[:b]
+        self.spans = self.flags_spans[b:].view(b, 2)
         self.kept_idx = torch.zeros((b, self.max_keep), dtype=torch.int32, device=dev)
         self.kept_count = torch.zeros(b, dtype=torch.int32, device=dev)
         self.diag = torch.zeros((b, 8), dtype=torch.float64, device=dev)
