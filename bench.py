@@ -311,9 +311,9 @@ class GpuBench:
     # launches of this repository's kernels per step (harness + path)
     def launches_per_step(self):
         calls = math.ceil(self.w.L / self.nl)
-        # one attention kernel per call on the tensor-core path (it merges its own partials),
-        # a partial pass and a merge on the fp32 path; the H2O path adds the score update
-        attend = (1 if self.w.dtype == "bf16" else 2) + (1 if self.policy == "h2o" else 0)
+        # per call on the tensor-core path: the counter reset and the pass (it merges its own
+        # partials); a partial pass and a merge on the fp32 path; H2O adds the score update
+        attend = 2 + (1 if self.policy == "h2o" else 0)
         path = 1 + 1 + attend * calls               # begin, append (+sketch), attend
         harness = 1 + 1                             # select, advance
         if self.policy in ("h2o", "streaming"):     # evict, lengths

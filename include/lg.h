@@ -19,6 +19,12 @@
  *    owned by the caller; the library allocates nothing and keeps no global state.
  *  - Every call is asynchronous on the caller's stream; nothing synchronises except
  *    lg_read_device_status.
+ *  - Kernels are launched with programmatic stream serialization (programmatic dependent
+ *    launch): each may be scheduled while the kernel before it in the stream is still running,
+ *    and waits (griddepcontrol.wait) for that kernel to complete before it touches memory, so
+ *    stream order holds as usual.  A kernel of the caller's that follows one of the library's
+ *    on the same stream keeps full stream order unless the caller launches it with the same
+ *    attribute, in which case it must wait the same way.
  *  - Arguments are validated on the host before any launch (null or misaligned pointers,
  *    unsupported shapes, short workspaces): the call returns an error and launches nothing.
  *  - Errors only visible on the device (a length above its capacity or above the call's
