@@ -439,11 +439,13 @@ def run_gpu(args, ws, rank, local):
     # steps whose attention pass and guard are bracketed by timing events inside the timed
     # region: every EV_EVERY-th step (an event between two kernels ends their programmatic
     # launch overlap, so events on every step would slow the steps they time)
-    every = 1 if fresh else EV_EVERY
-    sampled = set(range(0, K, every))
+    # (starting at step every/2, so that the first step's one-off budget cut of every sequence,
+    # one step in K of the timed region, does not weigh as one in K/every of the sample)
+    every = 1 if fresh else min(EV_EVERY, max(1, K // 4))
+    sampled = set(range(every // 2, K, every))
     ev_note = ("every step" if every == 1 else
-               "every %dth step of the timed region (%d of %d), events around the attention "
-               "pass and the guard" % (every, len(sampled), K))
+               "every %dth step of the timed region from step %d (%d of %d), events around the "
+               "attention pass and the guard" % (every, every // 2, len(sampled), K))
     if not fresh and not args.eager:
         # the same K steps timed eagerly first (reported beside the graph figure), then
         # captured once as a CUDA graph whose single replay is the timed region; events
