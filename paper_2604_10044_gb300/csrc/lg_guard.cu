@@ -279,6 +279,11 @@ __device__ __forceinline__ double widen(float x) {
 
 constexpr int kDetectWarps = kDetectThreads / 32;
 constexpr int kStatWarps = 3;  // warps that sum the statistics in fp64 (one per SM sub-partition)
+constexpr int kStatBatch = 8;  // statistics loads a thread has in flight at once
+constexpr int kCmpWarp0 = kStatWarps + 1;  // the new-row comparisons: warps after ln n's
+constexpr int kCmpThreads = kDetectThreads - kCmpWarp0 * 32;
+constexpr int kCmpBatch = 6;  // comparison chunks a thread has in flight at once
+static_assert(kCmpThreads % 32 == 0, "comparing threads in whole warps");
 
 // One CTA per sequence, monitor state carried from call to call in dstate:
 //   lm[slot]  latest earlier row of the window (as it was when the row was examined) whose
@@ -335,13 +340,23 @@ __global__ void __launch_bounds__(kDetectThreads, 1) detect_kernel(DetectArgs a)
   // (1) sums of the entropies and suffix masses over every layer and head (fp64, one warp per
   // SM sub-partition), and ln n on the fourth sub-partition
   if (warp < kStatWarps) {
+    // kStatBatch loads in flight per thread before the first add (one round trip per batch)
     double se = 0.0, sl = 0.0;
-    for (int t = tid; t < nh; t += kStatWarps * 32) {
-      const int layer = t / a.H_q, h = t - layer * a.H_q;
-      const float4 st = __ldg(reinterpret_cast<const float4 *>(a.stats) +
-                              ((int64_t)layer * a.c.batch + b) * a.H_q + h);
-      se += widen(st.z);
-      sl += widen(st.w);
+    for (int t0 = tid; t0 < nh; t0 += kStatWarps * 32 * kStatBatch) {
+      float4 st[kStatBatch];
+#pragma unroll
+      for (int k = 0; k < kStatBatch; ++k) {
+        const int t = t0 + k * kStatWarps * 32;
+        const int layer = t / a.H_q, h = t - layer * a.H_q;
+        st[k] = t < nh ? __ldg(reinterpret_cast<const float4 *>(a.stats) +
+                               ((int64_t)layer * a.c.batch + b) * a.H_q + h)
+                       : make_float4(0.f, 0.f, 0.f, 0.f);
+      }
+#pragma unroll
+      for (int k = 0; k < kStatBatch; ++k) {
+        se += widen(st[k].z);
+        sl += widen(st[k].w);
+      }
     }
     for (int o = 16; o >= 1; o >>= 1) {
       se += __shfl_xor_sync(0xffffffffu, se, o);
@@ -356,22 +371,55 @@ __global__ void __launch_bounds__(kDetectThreads, 1) detect_kernel(DetectArgs a)
   }
 
   if (incr) {
-    // (2) the new row against the window and the periods, reduced per warp
+    // (2) the new row against the rows the window and the periods need, [jlo, i), on the
+    // warps after the statistics and ln n (so the two run side by side): chunk q of row j is
+    // read by consecutive lanes (rows are contiguous: a warp reads 512 contiguous bytes), all of
+    // a thread's loads in flight at once, the chunk popcounts summed per row into dist[] in
+    // shared memory (the staging area of the recompute path, unused here); then the latest
+    // match, the novel rows and the period runs, reduced per warp
     const int i = n - 1;
     const uint32_t *ri = sk_g + (int64_t)i * nw;
-    const int j0 = i - 1 - tid;
-    bool m0 = false;
-    int latest = -1;
-    if (j0 >= 0) {
-      m0 = hamming(ri, sk_g + (int64_t)j0 * nw, nw) <= thr;
-      if (m0 && j0 >= wlo) latest = j0;
-    }
-    if (latest < 0)
-      for (int j = j0 - kDetectThreads; j >= wlo; j -= kDetectThreads)
-        if (hamming(ri, sk_g + (int64_t)j * nw, nw) <= thr) {
-          latest = j;
-          break;
+    const int jlo = max(0, min(wlo, i - p.p_max));
+    const int m_cnt = i - jlo;
+    const int cpr = nw / 4;  // 16-byte chunks per sketch row
+    int *dist = reinterpret_cast<int *>(sk_s);
+    const int ct = tid - kCmpWarp0 * 32;  // index among the comparing threads, < 0 elsewhere
+    if (ct >= 0) {
+      if ((cpr & (cpr - 1)) == 0 && cpr <= 32) {
+        // a power-of-two number of chunks: each row's chunks sit in aligned lanes of one warp
+        const uint4 *rows4 = reinterpret_cast<const uint4 *>(sk_g + (int64_t)jlo * nw);
+        const uint4 *ri4 = reinterpret_cast<const uint4 *>(ri);
+        const int total = m_cnt * cpr;
+        // a thread's chunk index is ct mod cpr in every row (the stride is a multiple of 32)
+        const uint4 v = __ldg(ri4 + (ct & (cpr - 1)));
+        for (int base = 0; base < total; base += kCmpThreads * kCmpBatch) {
+          uint4 u[kCmpBatch];
+#pragma unroll
+          for (int k = 0; k < kCmpBatch; ++k) {
+            const int f = base + ct + k * kCmpThreads;
+            u[k] = f < total ? __ldg(rows4 + f) : make_uint4(0u, 0u, 0u, 0u);
+          }
+#pragma unroll
+          for (int k = 0; k < kCmpBatch; ++k) {
+            const int f = base + ct + k * kCmpThreads;
+            int pc = __popc(u[k].x ^ v.x) + __popc(u[k].y ^ v.y) + __popc(u[k].z ^ v.z) +
+                     __popc(u[k].w ^ v.w);
+            for (int o = cpr >> 1; o >= 1; o >>= 1) pc += __shfl_xor_sync(0xffffffffu, pc, o);
+            if (f < total && (lane & (cpr - 1)) == 0) dist[f / cpr] = pc;
+          }
         }
+      } else {
+        for (int r = ct; r < m_cnt; r += kCmpThreads)
+          dist[r] = hamming(ri, sk_g + (int64_t)(jlo + r) * nw, nw);
+      }
+    }
+    __syncthreads();
+    int latest = -1;
+    for (int j = i - 1 - tid; j >= wlo; j -= kDetectThreads)
+      if (dist[j - jlo] <= thr) {
+        latest = j;
+        break;
+      }
     // novel rows of the window other than the new one
     int nov = 0, nov_tail = 0;
     for (int r = wlo + tid; r < i; r += kDetectThreads) {
@@ -386,7 +434,7 @@ __global__ void __launch_bounds__(kDetectThreads, 1) detect_kernel(DetectArgs a)
       const int P = p.p_min + pi;
       const int cap = max(p.m_rep * P, p.l_min);
       const int j = i - P;
-      const bool m = j >= 0 && (P == tid + 1 ? m0 : hamming(ri, sk_g + (int64_t)j * nw, nw) <= thr);
+      const bool m = j >= 0 && dist[j - jlo] <= thr;
       const int r = m ? min(run[pi] + 1, cap) : 0;
       run[pi] = r;
       if (pstar == 0x7fffffff && n >= cap + P && r >= cap) pstar = P;
