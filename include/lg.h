@@ -172,7 +172,10 @@ LG_API lg_status lg_sketch_build(const lg_cache *c, const lg_guard_params *p, in
    stats: device [n_layers][batch][H_q][4] fp32.  Query head h reads kv-head h / (H_q/H_kv).
    accumulate_h2o: also add sum over the GQA group of a_i to h2o[l][kvh][slot] (c->h2o).
    max_len: host bound on every len[b] (sizes the grid; a longer sequence is an error).
-   ws: device workspace of at least lg_workspace_size(...) bytes, 256-byte aligned. */
+   ws: device workspace of at least lg_workspace_size(...) bytes, 256-byte aligned.  On the bf16
+   path successive calls with one workspace walk the cache in alternating directions (one word
+   of ws keeps the direction), so that a call starts on the rows the previous call read last,
+   which may still be in L2; no result depends on the direction. */
 LG_API lg_status lg_decode_attend(const lg_cache *c, int layer0, int n_layers, const void *q, int H_q,
                            float scale, void *out, float *stats, int suffix_w,
                            int accumulate_h2o, int max_len, void *ws, size_t ws_bytes,
@@ -316,8 +319,10 @@ LG_API lg_status lg_h2o_evict(const lg_cache *c, const int32_t *budget, const in
    - The first call on each device looks up the array's device address (cudaGetSymbolAddress,
      with that device current); make that first call before any stream capture.
    - Every call on a device shares the one array, and it keeps the last call's contents (no
-     clearing is needed: every scratch byte read is written earlier in the same call).  Calls
-     that overlap on the GPU (different streams without ordering) race on it: order them. */
+     clearing is needed: every scratch byte read is written earlier in the same call, except
+     one word whose low bit picks the direction in which the call walks the cache, which never
+     changes a result).  Calls that overlap on the GPU (different streams without ordering)
+     race on it: order them. */
 LG_API lg_status lg_decode_attend_noalloc(const lg_cache *c, int layer0, int n_layers,
                                           const void *q, int H_q, float scale, void *out,
                                           float *stats, int suffix_w, int accumulate_h2o,

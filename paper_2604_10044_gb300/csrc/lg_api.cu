@@ -82,7 +82,8 @@ AttendLayout attend_layout(const lg_cache *c, int H_q, int n_layers, int max_len
   L.logits_bytes =
       h2o ? round256((size_t)n_layers * c->H_kv * c->S_total * (H_q / c->H_kv) * sizeof(float))
           : 0;
-  L.counter_bytes = round256((size_t)(1 + (int64_t)n_layers * c->batch * c->H_kv) * sizeof(int));
+  // chunk counter, one arrival counter per group, and the pass-direction word
+  L.counter_bytes = round256((size_t)(2 + (int64_t)n_layers * c->batch * c->H_kv) * sizeof(int));
   L.total = L.partial_bytes + L.final_bytes + L.logits_bytes + L.counter_bytes;
   return L;
 }

@@ -292,6 +292,7 @@ attend_mma_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant
   __shared__ int s_len[kStagedSeqs];         // len[b] and seq_off[b] of a batch up to kStagedSeqs
   __shared__ long long s_off[kStagedSeqs];
   __shared__ int s_bad;                      // the device status at entry (one read per CTA)
+  __shared__ int s_rev;                      // this call walks its chunks from the last one
   unsigned char *smem = reinterpret_cast<unsigned char *>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   float *tbuf = reinterpret_cast<float *>(smem + C::kRingBytes);  // [kBufs][TB::kFloats]
@@ -307,6 +308,7 @@ attend_mma_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant
   pdl_enter();  // the tensormap prefetch above reads only the kernel's parameters
   if (threadIdx.x == 0) {
     s_bad = status_bad(a.status);
+    s_rev = a.counter[1 + a.n_layers * a.batch * a.H_kv] & 1;
     for (int s = 0; s < C::kStages; ++s) {
       mbar_init(&full_bar[s], 1);
       mbar_init(&empty_bar[s], kConsumerWarps);
@@ -437,16 +439,20 @@ attend_mma_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant
     if (lane == 0) {
       uint32_t it = 0;
       const int claimed0 = 2 * (int)gridDim.x;
+      const bool rev = s_rev != 0;
       int c = blockIdx.x;
       bool first = true;
       while (true) {
         const bool alive = c < gm.total;
+        // the chunk this claim stands for: every other call walks the chunks from the last,
+        // so that it starts on the rows the previous call read last (still in L2)
+        const int cm = rev ? gm.total - 1 - c : c;
         int ntiles = 0, grow = 0, n = 0, c_next = 0;
         int64_t lrow0 = 0, head0 = 0;
         if (alive) {
           c_next = first ? (int)(blockIdx.x + gridDim.x) : claimed0 + atomicAdd(next_chunk, 1);
           first = false;
-          const ChunkId id = decode_chunk(a, c, gm.per_grp);
+          const ChunkId id = decode_chunk(a, cm, gm.per_grp);
           n = staged ? s_len[id.b] : a.len[id.b];
           const int64_t off = staged ? s_off[id.b] : a.seq_off[id.b];
           const int row0 = id.ch * gm.rows;
@@ -477,7 +483,7 @@ attend_mma_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant
             set_status(a.status, LG_ERR_TIMEOUT);
             return;
           }
-          stage_chunk[st] = alive ? c : -1;
+          stage_chunk[st] = alive ? cm : -1;
           stage_tile[st] = t;
           stage_n[st] = n;
           stage_lrow0[st] = lrow0;
@@ -751,11 +757,13 @@ attend_mma_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant
   }
 }
 
-// The call's chunk and group counters to zero: a kernel rather than a memset, so that the pass
-// after it keeps its programmatic launch edge.
+// The call's chunk and group counters to zero (a kernel rather than a memset, so that the pass
+// after it keeps its programmatic launch edge), and the word after them flipped: its low bit
+// is the direction of this call's pass (any start value will do; it only alternates).
 __global__ void zero_counters_kernel(int *p, int n) {
   pdl_enter();
   for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < n; i += gridDim.x * blockDim.x) p[i] = 0;
+  if (blockIdx.x == 0 && threadIdx.x == 0) p[n] ^= 1;
 }
 
 // ------------------------------------------------------------------ host side

@@ -48,8 +48,9 @@ extern "C" lg_status lg_decode_attend_noalloc(const lg_cache *c, int layer0, int
   void *ws = nullptr;
   lg_status st = scratch_for_current_device(&ws);
   if (st != LG_OK) return st;
-  // every byte of scratch the kernels read is written earlier in the same call, so the
-  // contents left by a previous call need no clearing
+  // every byte of scratch the kernels read is written earlier in the same call (but the
+  // pass-direction word, whose value never changes a result), so the contents left by a
+  // previous call need no clearing
   return lg_decode_attend(c, layer0, n_layers, q, H_q, scale, out, stats, suffix_w,
                           accumulate_h2o, max_len, ws, (size_t)LG_NOALLOC_SCRATCH_BYTES, s);
 }
