@@ -141,9 +141,21 @@ def test_paper_shaped_guard(cuda):
     dict(W=400, p_min=3, p_max=40, m_rep=2, l_min=16, stall_len=6, K=1),
     # a narrow window, all three votes, a short cooldown and warmup
     dict(W=100, p_max=60, K=3, theta_lift=1.5, cooldown=8, t_min=10, retrig_window=20),
+    # a window wider than the detect CTA (512 threads): several rounds of comparisons and of
+    # the latest-match scan
+    dict(W=700, p_max=100),
 ])
 def test_nondefault_guard_params(cuda, over):
     """the same pipeline under other monitor constants: both sides take the same parameters"""
     w = synth.make_workload(2, L=2, batch=4, n=1200, budget=768, steps=40, tail=(300, 500),
                             periods=(8, 40))
     run_loopguard(w, cuda, params=over)
+
+
+def test_sketch_rows_of_six_chunks(cuda):
+    """6 kv-heads of d = 128: a sketch row of 24 words is 6 16-byte chunks, not a power of two,
+    so the loop-onset test compares the new row a row per thread instead of a chunk per lane"""
+    w = synth.make_workload(2, L=2, batch=4, n=1200, budget=768, steps=40, tail=(300, 500),
+                            periods=(8, 40), H_q=12, H_kv=6)
+    c = run_loopguard(w, cuda)
+    assert c["triggers"] >= 1 and c["prunes"] >= 4
