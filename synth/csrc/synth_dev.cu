@@ -7,6 +7,29 @@
 
 namespace {
 
+// The per-step harness kernels (selection of each sequence's inputs, advance) sit between the
+// guard's kernels, which are launched with programmatic stream serialization; they are launched
+// the same way and wait (griddepcontrol.wait) for the kernel before them before touching memory.
+__device__ __forceinline__ void pdl_enter() {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, cudaStream_t s,
+                       Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, args...);
+}
+
 __device__ __forceinline__ void store(const syn_workload &w, void *out, int64_t i, float v) {
   if (w.dtype == SYN_BF16)
     ((uint16_t *)out)[i] = syn_bf16_bits(v);
@@ -67,6 +90,7 @@ __global__ void step_kv_kernel(syn_workload w, const syn_seq *seqs, int batch,
 // After a step: a sequence whose guard intervened turns loop-free from the next token on, and
 // every sequence moves to its next position.
 __global__ void advance_kernel(syn_seq *seqs, int batch, const int32_t *flags, int64_t *pos) {
+  pdl_enter();
   int b = blockIdx.x * blockDim.x + threadIdx.x;
   if (b >= batch) return;
   if (flags && flags[b] && seqs[b].fresh_from == SYN_NEVER) seqs[b].fresh_from = (int)pos[b] + 1;
@@ -78,6 +102,7 @@ __global__ void advance_kernel(syn_seq *seqs, int batch, const int32_t *flags, i
 __global__ void select_kernel(const syn_seq *seqs, int batch, const int64_t *pos, int L,
                               int64_t rowlen_bytes, const char *loop_buf, const char *fresh_buf,
                               char *out) {
+  pdl_enter();
   int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;  // 16-byte chunk index
   int64_t chunks = rowlen_bytes / 16;
   int64_t total = (int64_t)L * batch * chunks;
@@ -96,6 +121,7 @@ struct Sel3 {
 };
 
 __global__ void select3_kernel(const syn_seq *seqs, int batch, const int64_t *pos, int L, Sel3 s) {
+  pdl_enter();
   int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   for (int k = 0; k < 3; ++k) {
     const int64_t total = (int64_t)L * batch * s.chunks[k];
@@ -115,6 +141,7 @@ __global__ void select_tokens_kernel(const syn_seq *seqs, int batch, const int64
                                      const int32_t *tok_loop, const int32_t *tok_fresh,
                                      const float *pm_loop, const float *pm_fresh, int32_t *tok,
                                      float *pm) {
+  pdl_enter();
   const int b = blockIdx.x * blockDim.x + threadIdx.x;
   if (b >= batch) return;
   const bool fresh = pos[b] >= seqs[b].fresh_from;
@@ -139,9 +166,10 @@ int syn_dev_select3(const syn_seq *seqs_dev, int batch, const int64_t *pos_dev, 
     s.chunks[k] = rowlen_bytes[k] / 16;
     total += (int64_t)L * batch * s.chunks[k];
   }
-  select3_kernel<<<(unsigned)((total + 255) / 256), 256, 0, stream>>>(seqs_dev, batch, pos_dev, L,
-                                                                      s);
-  return cudaGetLastError() == cudaSuccess ? 0 : 2;
+  return launch_pdl(select3_kernel, dim3((unsigned)((total + 255) / 256)), dim3(256), stream,
+                    seqs_dev, batch, pos_dev, L, s) == cudaSuccess
+             ? 0
+             : 2;
 }
 
 int syn_dev_fill_cache(const syn_workload *w, const syn_seq *seqs_dev, int batch,
@@ -170,8 +198,10 @@ int syn_dev_step(const syn_workload *w, const syn_seq *seqs_dev, int batch, cons
 
 int syn_dev_advance(syn_seq *seqs_dev, int batch, const int32_t *flags_dev, int64_t *pos_dev,
                     cudaStream_t stream) {
-  advance_kernel<<<(batch + 127) / 128, 128, 0, stream>>>(seqs_dev, batch, flags_dev, pos_dev);
-  return cudaGetLastError() == cudaSuccess ? 0 : 2;
+  return launch_pdl(advance_kernel, dim3((batch + 127) / 128), dim3(128), stream, seqs_dev,
+                    batch, flags_dev, pos_dev) == cudaSuccess
+             ? 0
+             : 2;
 }
 
 int syn_dev_select(const syn_seq *seqs_dev, int batch, const int64_t *pos_dev, int L,
@@ -179,18 +209,21 @@ int syn_dev_select(const syn_seq *seqs_dev, int batch, const int64_t *pos_dev, i
                    cudaStream_t stream) {
   if (rowlen_bytes % 16) return 1;
   int64_t total = (int64_t)L * batch * (rowlen_bytes / 16);
-  select_kernel<<<(unsigned)((total + 255) / 256), 256, 0, stream>>>(
-      seqs_dev, batch, pos_dev, L, rowlen_bytes, (const char *)loop_buf, (const char *)fresh_buf,
-      (char *)out);
-  return cudaGetLastError() == cudaSuccess ? 0 : 2;
+  return launch_pdl(select_kernel, dim3((unsigned)((total + 255) / 256)), dim3(256), stream,
+                    seqs_dev, batch, pos_dev, L, rowlen_bytes, (const char *)loop_buf,
+                    (const char *)fresh_buf, (char *)out) == cudaSuccess
+             ? 0
+             : 2;
 }
 
 int syn_dev_select_tokens(const syn_seq *seqs_dev, int batch, const int64_t *pos_dev,
                           const int32_t *tok_loop, const int32_t *tok_fresh, const float *pm_loop,
                           const float *pm_fresh, int32_t *tok, float *pm, cudaStream_t stream) {
-  select_tokens_kernel<<<(batch + 127) / 128, 128, 0, stream>>>(
-      seqs_dev, batch, pos_dev, tok_loop, tok_fresh, pm_loop, pm_fresh, tok, pm);
-  return cudaGetLastError() == cudaSuccess ? 0 : 2;
+  return launch_pdl(select_tokens_kernel, dim3((batch + 127) / 128), dim3(128), stream,
+                    seqs_dev, batch, pos_dev, tok_loop, tok_fresh, pm_loop, pm_fresh, tok,
+                    pm) == cudaSuccess
+             ? 0
+             : 2;
 }
 
 }  // extern "C"
