@@ -57,3 +57,32 @@ def test_attend_empty_and_boundary_lengths(cuda, dtype):
                 tag = "layer %d seq %d (n=%d) kv-head %d" % (layer, b, n, kvh)
                 assert_close(o[layer, b, hs], o_ref, rt, ra, tag + " out")
                 assert_close(st[layer, b, hs], s_ref, *STAT_TOL, what=tag + " stats")
+
+
+def test_pass_direction_changes_no_result(cuda):
+    """successive lg_decode_attend calls with one workspace walk the cache in opposite
+    directions; the same inputs give bit-identical outputs and statistics, with the H2O score
+    accumulation both off and on (ragged lengths, several chunks per group)"""
+    w = synth.make_workload(4, L=2, batch=5, len_range=(40, 5000), budget_max=8192, steps=1,
+                            onset_max=1, periods=(4, 8))
+    K, V = synth.host_cache(w)
+    for h2o in (0, 1):
+        cache = lg.Cache.from_host(w, K, V, cuda, policy="h2o" if h2o else "loopguard")
+        max_len = int(w.n0.max())
+        if h2o:
+            lg.lg_h2o_reset(cache, max_len)
+        q, _, _ = synth.host_step(w, w.n0.astype(np.int64))
+        qd = lg.host_to_device(q, cuda, "bf16")
+        ws = torch.empty(lg.lg_workspace_size(cache, w.H_q, w.L, max_len, h2o) // 4 + 64,
+                         dtype=torch.float32, device=cuda)
+        runs = []
+        for _ in range(2):
+            out = torch.zeros((w.L, w.batch, w.H_q, w.d), dtype=torch.bfloat16, device=cuda)
+            stats = torch.zeros((w.L, w.batch, w.H_q, 4), dtype=torch.float32, device=cuda)
+            lg.lg_decode_attend(cache, 0, w.L, qd, w.H_q, 1.0 / np.sqrt(w.d), out, stats, 64,
+                                h2o, max_len, ws)
+            torch.cuda.synchronize()
+            assert lg.lg_read_device_status(cache) == 0
+            runs.append((out.cpu(), stats.cpu()))
+        assert torch.equal(runs[0][0], runs[1][0]), h2o
+        assert torch.equal(runs[0][1], runs[1][1]), h2o
