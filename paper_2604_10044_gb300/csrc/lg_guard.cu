@@ -383,6 +383,10 @@ __global__ void __launch_bounds__(kDetectThreads, 1) detect_kernel(DetectArgs a)
     const int m_cnt = i - jlo;
     const int cpr = nw / 4;  // 16-byte chunks per sketch row
     int *dist = reinterpret_cast<int *>(sk_s);
+    // the monitor state this thread reads after the comparisons, requested before them
+    const int r0 = wlo + tid;
+    const int lm0 = r0 < i ? lm[r0] : 0;
+    const int run0 = tid < np ? run[tid] : 0;
     const int ct = tid - kCmpWarp0 * 32;  // index among the comparing threads, < 0 elsewhere
     if (ct >= 0) {
       if ((cpr & (cpr - 1)) == 0 && cpr <= 32) {
@@ -422,8 +426,8 @@ __global__ void __launch_bounds__(kDetectThreads, 1) detect_kernel(DetectArgs a)
       }
     // novel rows of the window other than the new one
     int nov = 0, nov_tail = 0;
-    for (int r = wlo + tid; r < i; r += kDetectThreads) {
-      const int novel = lm[r] < wlo;
+    for (int r = r0; r < i; r += kDetectThreads) {
+      const int novel = (r == r0 ? lm0 : lm[r]) < wlo;
       nov += novel;
       if (r >= n - p.stall_len) nov_tail += novel;
     }
@@ -435,7 +439,7 @@ __global__ void __launch_bounds__(kDetectThreads, 1) detect_kernel(DetectArgs a)
       const int cap = max(p.m_rep * P, p.l_min);
       const int j = i - P;
       const bool m = j >= 0 && dist[j - jlo] <= thr;
-      const int r = m ? min(run[pi] + 1, cap) : 0;
+      const int r = m ? min((pi == tid ? run0 : run[pi]) + 1, cap) : 0;
       run[pi] = r;
       if (pstar == 0x7fffffff && n >= cap + P && r >= cap) pstar = P;
     }
