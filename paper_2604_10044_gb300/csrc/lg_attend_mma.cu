@@ -138,9 +138,11 @@ struct ChunkId {
 // (measured: finer chunks gained nothing at the end of long passes and cost a little on the
 // way); the rows are then evened out over the chunks of the longest group.
 struct Geom {
-  int rows;     // rows per chunk
-  int per_grp;  // chunk ids per (layer, sequence, kv-head)
-  int total;    // chunk ids of the call
+  int rows;        // rows per chunk
+  int per_grp;     // chunk ids per (layer, sequence, kv-head)
+  int total;       // chunk ids of the call
+  int groups;      // (layer, sequence, kv-head) groups of the call
+  bool long_pass;  // the last chunks of the groups are short and claimed last; no reversal
 };
 
 __device__ __forceinline__ Geom make_geom(const AttendArgs &a, int n_max, int64_t len_sum,
@@ -162,16 +164,34 @@ __device__ __forceinline__ Geom make_geom(const AttendArgs &a, int n_max, int64_
   c = (int)(((nm + per - 1u) / per + kTile - 1) / kTile * kTile);
   c = max(c, kTile);
   Geom gm;
+  // a long pass (64 tiles a CTA or more) ends on short chunks: each group's last chunk is
+  // about a quarter of the others (rows n_max / (per - 3/4), as many chunks per group), and
+  // decode_chunk hands out every group's last chunk after all the others
+  gm.long_pass = rows_all >= 64.f * (float)kTile * (float)ctas && per >= 2;
+  if (gm.long_pass) {
+    const float cl = ceilf((float)nm / ((float)per - 0.75f));
+    c = max(c, ((int)cl + kTile - 1) / kTile * kTile);
+  }
   gm.rows = c;
   gm.per_grp = max(1, (int)((nm + (unsigned)c - 1u) / (unsigned)c));
-  gm.total = a.n_layers * a.batch * a.H_kv * gm.per_grp;
+  gm.groups = a.n_layers * a.batch * a.H_kv;
+  gm.total = gm.groups * gm.per_grp;
   return gm;
 }
 
-__device__ __forceinline__ ChunkId decode_chunk(const AttendArgs &a, int c, int per_grp) {
+// Chunk id -> (layer, sequence, kv-head, chunk): the groups' chunks but the last come first
+// (per_grp - 1 of each group, group-major), then every group's last chunk.
+__device__ __forceinline__ ChunkId decode_chunk(const AttendArgs &a, int c, const Geom &gm) {
   ChunkId id;
-  id.ch = c % per_grp;
-  int r = c / per_grp;
+  const int nb = gm.per_grp - 1;
+  int r;
+  if (c < gm.groups * nb) {
+    id.ch = c % nb;
+    r = c / nb;
+  } else {
+    id.ch = nb;
+    r = c - gm.groups * nb;
+  }
   id.kvh = r % a.H_kv;
   r /= a.H_kv;
   id.b = r % a.batch;
@@ -444,15 +464,16 @@ attend_mma_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant
       bool first = true;
       while (true) {
         const bool alive = c < gm.total;
-        // the chunk this claim stands for: every other call walks the chunks from the last,
-        // so that it starts on the rows the previous call read last (still in L2)
-        const int cm = rev ? gm.total - 1 - c : c;
+        // the chunk this claim stands for: a short pass walks the chunks from the last on
+        // every other call, so that it starts on the rows the previous call read last (still
+        // in L2); a long pass keeps its order (its short last chunks stay at the end)
+        const int cm = rev && !gm.long_pass ? gm.total - 1 - c : c;
         int ntiles = 0, grow = 0, n = 0, c_next = 0;
         int64_t lrow0 = 0, head0 = 0;
         if (alive) {
           c_next = first ? (int)(blockIdx.x + gridDim.x) : claimed0 + atomicAdd(next_chunk, 1);
           first = false;
-          const ChunkId id = decode_chunk(a, cm, gm.per_grp);
+          const ChunkId id = decode_chunk(a, cm, gm);
           n = staged ? s_len[id.b] : a.len[id.b];
           const int64_t off = staged ? s_off[id.b] : a.seq_off[id.b];
           const int row0 = id.ch * gm.rows;
@@ -534,7 +555,7 @@ attend_mma_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant
     const int t = stage_tile[st];
     if (t == 0) {
       // first tile of a chunk: its geometry, the q^T fragments, fresh softmax state
-      id = decode_chunk(a, c, gm.per_grp);
+      id = decode_chunk(a, c, gm);
       n = stage_n[st];
       row0 = id.ch * gm.rows;
       rows = min(gm.rows, n - row0);
