@@ -43,7 +43,8 @@ __device__ __forceinline__ uint32_t sketch_word(const void *row_base, int64_t he
 
 // Blocks [0, row_blocks): one thread per 16-byte chunk of a new row, written to slot
 // len[b] - 1.  Blocks [row_blocks, row_blocks + batch) when the guard layer is in the call:
-// the sketch of that layer's new V row (read from v_new [n_layers][b][H_kv][d]).
+// the sketch of that layer's new V row (read from v_new [n_layers][b][H_kv][d]), a warp per
+// word: lane j reads element 32w + j and the ballot of the sign bits is word w.
 template <typename T>
 __global__ void append_kernel(lg_cache c, int layer0, int n_layers, const uint4 *k_new,
                               const uint4 *v_new, const int32_t *pos_new, int row_blocks,
@@ -51,13 +52,18 @@ __global__ void append_kernel(lg_cache c, int layer0, int n_layers, const uint4 
   pdl_enter();
   if ((int)blockIdx.x >= row_blocks) {
     const int b = blockIdx.x - row_blocks;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int nwords = c.H_kv * c.d / 32;
     const int slot = c.len[b] - 1;
     const int64_t off = c.seq_off[b];
-    if (status_bad(c.dev_status) || slot < 0) return;
+    // one status read per warp, so that every lane of the ballot takes the same branch
+    const int bad = __shfl_sync(0xffffffffu, lane == 0 ? (int)status_bad(c.dev_status) : 0, 0);
+    if (bad || slot < 0) return;
     const T *row = (const T *)v_new + ((int64_t)lguard * c.batch + b) * c.H_kv * c.d;
-    for (int w = threadIdx.x; w < nwords; w += blockDim.x)
-      c.sketch[(off + slot) * nwords + w] = sketch_word<T>(row, c.d, c.d, w);
+    for (int w = warp; w < nwords; w += blockDim.x >> 5) {
+      const uint32_t word = __ballot_sync(0xffffffffu, Elem<T>::sign(row, w * 32 + lane) != 0u);
+      if (lane == 0) c.sketch[(off + slot) * nwords + w] = word;
+    }
     return;
   }
   const int cpr = c.d * (int)sizeof(T) / 16;
