@@ -257,7 +257,43 @@ class GpuBench:
         self.cache.status.zero_()
         torch.cuda.synchronize()
 
+    def use_stage(self, on=True):
+        """read every step's inputs from one fixed device slab (filled by the caller before each
+        step, as a serving loop fills its input buffers) instead of the step's own slab, so that
+        one captured graph serves every step; the slab packs both input variants and, for the
+        token-level detector, both token and p_max variants as raw bytes"""
+        torch, w = self.torch, self.w
+        self.stage = None
+        if not on:
+            return
+        L, b, d = w.L, w.batch, w.d
+        nq, nk = L * b * w.H_q * d, L * b * w.H_kv * d
+        inp_bytes = self.inp[0].numel() * self.inp.element_size()
+        tok_bytes = 16 * b if self.detector == "token" else 0
+        self.stage = torch.empty(inp_bytes + tok_bytes, dtype=torch.uint8, device=self.dev)
+        sin = self.stage[:inp_bytes].view(self.inp.dtype)
+        cut = lambda o, n, h: sin[o:o + n].view(L, b, h, d)
+        self.st_A = (cut(0, nq, w.H_q), cut(2 * nq, nk, w.H_kv), cut(2 * nq + 2 * nk, nk, w.H_kv))
+        self.st_B = (cut(nq, nq, w.H_q), cut(2 * nq + nk, nk, w.H_kv),
+                     cut(2 * nq + 3 * nk, nk, w.H_kv))
+        if tok_bytes:
+            ti = self.stage[inp_bytes:inp_bytes + 8 * b].view(torch.int32)
+            tp = self.stage[inp_bytes + 8 * b:].view(torch.float32)
+            self.st_tok = (ti[:b], ti[b:], tp[:b], tp[b:])
+
+    def stage_host(self, K):
+        """the K steps' staged inputs in pinned host memory, [K][stage bytes]"""
+        torch = self.torch
+        rows = [self.inp[:K].cpu().view(torch.uint8).reshape(K, -1)]
+        if self.detector == "token":
+            rows += [torch.cat([self.tokA[:K], self.tokB[:K]], 1).cpu().view(torch.uint8),
+                     torch.cat([self.pmA[:K], self.pmB[:K]], 1).cpu().view(torch.uint8)]
+        return torch.cat(rows, 1).contiguous().pin_memory()
+
     def select_inputs(self, t):
+        if getattr(self, "stage", None) is not None:
+            self.sel(self.st_A, self.st_B, self.s)
+            return
         self.sel((self.qA[t], self.kA[t], self.vA[t]), (self.qB[t], self.kB[t], self.vB[t]),
                  self.s)
 
@@ -283,8 +319,12 @@ class GpuBench:
         token = guard_path and self.detector == "token"
         if token:
             # the caller's generated token and top-1 probability, then the token-level monitor
-            synth.dev_select_tokens(w, self.seqs_d, self.pos_d, self.tokA[t], self.tokB[t],
-                                    self.pmA[t], self.pmB[t], self.tok, self.pm, self.s)
+            if getattr(self, "stage", None) is not None:
+                tl, tf, pl, pf = self.st_tok
+            else:
+                tl, tf, pl, pf = self.tokA[t], self.tokB[t], self.pmA[t], self.pmB[t]
+            synth.dev_select_tokens(w, self.seqs_d, self.pos_d, tl, tf, pl, pf, self.tok,
+                                    self.pm, self.s)
             lg.lg_token_detect(c, self.tok, self.pm, g.state, p, self.tp, g.flags, g.spans,
                                None, self.tstate, g.kept_idx, g.kept_count, self.s)
         elif guard_path and not split:
@@ -609,21 +649,17 @@ def run_gpu(args, ws, rank, local):
 
 def run_e2e(bench, K, ws, graphs=True):
     """the same steps through the C ABI with host buffers: every step copies its inputs from
-    pinned host memory, runs the guarded step and reads the outputs back (attention output,
-    flags, spans, lengths), and the host waits for them before the next step.  graphs: each
-    step's copies, calls and read-back are captured once as a CUDA graph (as a serving loop
-    captures its decode step) and replayed in the timed loop; else they are launched eagerly.
-    Returns (line dict, eager steps/s or None)."""
+    pinned host memory into the step's input slab on the device (one copy), runs the guarded
+    step and reads the outputs back (attention output, flags, spans, lengths), and the host
+    waits for them before the next step.  graphs: the step's calls and the gathering of its
+    results are captured once as one CUDA graph over the fixed slab (as a serving loop
+    captures its decode step) and replayed every step, the copies around it stream copies;
+    else the calls are launched eagerly.  Returns (line dict, eager steps/s)."""
     torch = bench.torch
     w = bench.w
-    # both input variants of every step in pinned host memory (filled before timing), one
-    # slab per step
-    pairs = [(bench.inp, bench.inp[:K].cpu().pin_memory())]
-    if bench.detector == "token":
-        # the generated token ids and top-1 probabilities of the step, both variants
-        for dev_t in (bench.tokA, bench.tokB, bench.pmA, bench.pmB):
-            pairs.append((dev_t, dev_t[:K].cpu().pin_memory()))
     g = bench.guard
+    bench.use_stage(True)
+    stage_h = bench.stage_host(K)  # both input variants of every step, filled before timing
     out_h = torch.empty(g.out.shape, dtype=g.out.dtype).pin_memory()
     fs_h = torch.empty(3 * w.batch, dtype=torch.int32).pin_memory()
     len_h = torch.empty(w.batch, dtype=torch.int32).pin_memory()
@@ -642,9 +678,7 @@ def run_e2e(bench, K, ws, graphs=True):
         pack_len.copy_(bench.cache.len)
 
     def copy_in(t):
-        # H2D: this step's input variants into the device slots the harness reads
-        for dst, src in pairs:
-            dst[t].copy_(src[t], non_blocking=True)
+        bench.stage.copy_(stage_h[t], non_blocking=True)
 
     def copy_out():
         out_h.copy_(g.out, non_blocking=True)
@@ -667,29 +701,27 @@ def run_e2e(bench, K, ws, graphs=True):
         return max_over_ranks(time.perf_counter() - t0, ws)
 
     dt_eager = timed(enqueue)
-    dt = dt_graph = None
+    dt_graph = None
     if graphs:
-        # the step's kernels as one graph per step; the host copies stay stream copies (as
-        # graph nodes, copies from pinned host memory ran several times slower on this system)
-        step_graphs = []
-        for t in range(K):
-            gr = torch.cuda.CUDAGraph()
-            with torch.cuda.graph(gr, stream=bench.stream, capture_error_mode="thread_local"):
-                bench.step(t)
-                pack()
-            step_graphs.append(gr)
-        # one untimed replay of every graph first: the first launch of a graph uploads it
+        # one graph for every step: it reads the fixed input slab (the copies into it and out
+        # of the gathered results stay stream copies; as graph nodes, copies from pinned host
+        # memory ran several times slower on this system)
+        gr = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(gr, stream=bench.stream, capture_error_mode="thread_local"):
+            bench.step(0)
+            pack()
         bench.reset()
-        for gr in step_graphs:
-            gr.replay()
+        copy_in(0)
+        gr.replay()  # untimed: the first launch of a graph uploads it
         torch.cuda.synchronize()
 
         def graphed(t):
             copy_in(t)
-            step_graphs[t].replay()
+            gr.replay()
             pack_h.copy_(pack_d, non_blocking=True)
         dt_graph = timed(graphed)
-    h2d = sum(h[0].numel() * h.element_size() for _, h in pairs)
+    bench.use_stage(False)
+    h2d = stage_h[0].numel()
     d2h = out_h.numel() * out_h.element_size() + (fs_h.numel() + len_h.numel()) * 4
     rate = lambda d: round(sum_over_ranks(K, ws) / d, 3) if d else None
     # the faster of the two ways a serving loop can drive the calls (both reported)
@@ -697,7 +729,8 @@ def run_e2e(bench, K, ws, graphs=True):
     line = {"value": rate(dt_graph if use_graph else dt_eager), "unit": UNIT,
             "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
             "launch": "a stream copy in, the step's kernels and the gathering of its results as "
-                      "one CUDA graph, a stream copy out; host waits for each step" if use_graph
+                      "one CUDA graph (the same for every step), a stream copy out; host waits "
+                      "for each step" if use_graph
                       else "eager calls, host waits for each step",
             "steps_per_s_eager": rate(dt_eager), "steps_per_s_graphed_kernels": rate(dt_graph),
             "note": "inputs of both sequence modes (loop continues / loop-free) copied every "
