@@ -271,21 +271,11 @@ __device__ __forceinline__ int hamming(const uint32_t *x, const uint32_t *y, int
   return dist;
 }
 
-// fp32 -> fp64 by moving the bits (IEEE-754 binary32 into binary64: exponent rebiased by
-// 1023 - 127 = 896, mantissa shifted up by 29), exact; normal numbers and zeros stay on the
-// integer pipe, subnormals, infinities and NaNs take the conversion instruction.
-__device__ __forceinline__ double widen(float x) {
-  const uint32_t u = __float_as_uint(x);
-  const uint32_t e = (u >> 23) & 0xffu, m = u & 0x7fffffu, sgn = u & 0x80000000u;
-  if (e - 1u < 254u)
-    return __hiloint2double((int)(sgn | ((e + 896u) << 20) | (m >> 3)), (int)(u << 29));
-  if (e == 0u && m == 0u) return __hiloint2double((int)sgn, 0);
-  return (double)x;
-}
-
 constexpr int kDetectWarps = kDetectThreads / 32;
 constexpr int kStatWarps = 3;  // warps that sum the statistics in fp64 (one per SM sub-partition)
 constexpr int kStatBatch = 8;  // statistics loads a thread has in flight at once
+constexpr float kFixScale = 1099511627776.0f;  // 2^40: statistics summed in 2^-40 units
+constexpr double kFixUnit = 1.0 / 1099511627776.0;
 constexpr int kCmpWarp0 = kStatWarps + 1;  // the new-row comparisons: warps after ln n's
 constexpr int kCmpThreads = kDetectThreads - kCmpWarp0 * 32;
 constexpr int kCmpBatch = 6;  // comparison chunks a thread has in flight at once
@@ -310,7 +300,8 @@ static_assert(kCmpThreads % 32 == 0, "comparing threads in whole warps");
 __global__ void __launch_bounds__(kDetectThreads, 1) detect_kernel(DetectArgs a) {
   pdl_enter();
   extern __shared__ __align__(16) uint32_t sk_s[];
-  __shared__ double red_e[kStatWarps], red_l[kStatWarps];
+  __shared__ long long red_e[kStatWarps], red_l[kStatWarps];  // fixed point, 2^-40 units
+  __shared__ int red_ok[kStatWarps];                          // every statistic finite
   __shared__ int w_latest[kDetectWarps], w_nov[kDetectWarps], w_nov_tail[kDetectWarps],
       w_pstar[kDetectWarps];
   __shared__ double s_logn;
@@ -343,11 +334,15 @@ __global__ void __launch_bounds__(kDetectThreads, 1) detect_kernel(DetectArgs a)
   const bool incr = n >= 1 && synced + 1 == n;
   const int nh = a.c.L * a.H_q;
 
-  // (1) sums of the entropies and suffix masses over every layer and head (fp64, one warp per
-  // SM sub-partition), and ln n on the fourth sub-partition
+  // (1) sums of the entropies and suffix masses over every layer and head, one warp per SM
+  // sub-partition, and ln n on the fourth.  The sums are exact in 64-bit fixed point (units of
+  // 2^-40: a value loses at most 2^-40 when it is scaled and truncated, and values up to 2^23
+  // fit), on the integer pipes rather than GB300's slow fp64 pipe; a non-finite statistic
+  // makes its sum NaN.
   if (warp < kStatWarps) {
     // kStatBatch loads in flight per thread before the first add (one round trip per batch)
-    double se = 0.0, sl = 0.0;
+    long long se = 0, sl = 0;
+    int finite = 1;
     for (int t0 = tid; t0 < nh; t0 += kStatWarps * 32 * kStatBatch) {
       float4 st[kStatBatch];
 #pragma unroll
@@ -360,17 +355,20 @@ __global__ void __launch_bounds__(kDetectThreads, 1) detect_kernel(DetectArgs a)
       }
 #pragma unroll
       for (int k = 0; k < kStatBatch; ++k) {
-        se += widen(st[k].z);
-        sl += widen(st[k].w);
+        finite &= isfinite(st[k].z) && isfinite(st[k].w);
+        se += __float2ll_rz(st[k].z * kFixScale);
+        sl += __float2ll_rz(st[k].w * kFixScale);
       }
     }
     for (int o = 16; o >= 1; o >>= 1) {
       se += __shfl_xor_sync(0xffffffffu, se, o);
       sl += __shfl_xor_sync(0xffffffffu, sl, o);
     }
+    finite = __all_sync(0xffffffffu, finite);
     if (lane == 0) {
       red_e[warp] = se;
       red_l[warp] = sl;
+      red_ok[warp] = finite;
     }
   } else if (warp == kStatWarps && lane == 0) {
     s_logn = n >= 2 ? log((double)n) : 1.0;
@@ -546,15 +544,25 @@ __global__ void __launch_bounds__(kDetectThreads, 1) detect_kernel(DetectArgs a)
   if (lane == 0 && warp < 4 && n >= 1) {
     if (warp == 0) {
       // vote 2: mean of H / ln n over every layer and head
-      double e_sum = 0.0;
-      for (int k = 0; k < kStatWarps; ++k) e_sum += red_e[k];
+      long long e_fix = 0;
+      int ok = 1;
+      for (int k = 0; k < kStatWarps; ++k) {
+        e_fix += red_e[k];
+        ok &= red_ok[k];
+      }
+      const double e_sum = ok ? (double)e_fix * kFixUnit : (double)NAN;
       const double ebar = n >= 2 ? e_sum / ((double)nh * s_logn) : 1.0;
       s_sig[1] = ebar < p.theta_ent;
       if (a.diag) a.diag[8 * b] = ebar;
     } else if (warp == 1) {
       // vote 3: mean of S * n / W_s over every layer and head
-      double l_sum = 0.0;
-      for (int k = 0; k < kStatWarps; ++k) l_sum += red_l[k];
+      long long l_fix = 0;
+      int ok = 1;
+      for (int k = 0; k < kStatWarps; ++k) {
+        l_fix += red_l[k];
+        ok &= red_ok[k];
+      }
+      const double l_sum = ok ? (double)l_fix * kFixUnit : (double)NAN;
       const double lbar = l_sum * (double)n / ((double)Ws * (double)nh);
       s_sig[2] = lbar >= p.theta_lift;
       if (a.diag) a.diag[8 * b + 1] = lbar;
