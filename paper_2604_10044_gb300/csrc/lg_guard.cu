@@ -333,6 +333,11 @@ __global__ void __launch_bounds__(kDetectThreads, 1) detect_kernel(DetectArgs a)
   int32_t *lm = a.dstate + (int64_t)a.c.batch * (np + 2) + off;
   const bool incr = n >= 1 && synced + 1 == n;
   const int nh = a.c.L * a.H_q;
+  // the monitor state the incremental step reads after its comparisons (a window row's latest
+  // match, a period's run), requested now, before the statistics warps start their sums
+  const int r0 = wlo + tid;
+  const int lm0 = incr && r0 < n - 1 ? lm[r0] : 0;
+  const int run0 = incr && tid < np ? run[tid] : 0;
 
   // (1) sums of the entropies and suffix masses over every layer and head, one warp per SM
   // sub-partition, and ln n on the fourth.  The sums are exact in 64-bit fixed point (units of
@@ -387,10 +392,6 @@ __global__ void __launch_bounds__(kDetectThreads, 1) detect_kernel(DetectArgs a)
     const int m_cnt = i - jlo;
     const int cpr = nw / 4;  // 16-byte chunks per sketch row
     int *dist = reinterpret_cast<int *>(sk_s);
-    // the monitor state this thread reads after the comparisons, requested before them
-    const int r0 = wlo + tid;
-    const int lm0 = r0 < i ? lm[r0] : 0;
-    const int run0 = tid < np ? run[tid] : 0;
     const int ct = tid - kCmpWarp0 * 32;  // index among the comparing threads, < 0 elsewhere
     if (ct >= 0) {
       if ((cpr & (cpr - 1)) == 0 && cpr <= 32) {
