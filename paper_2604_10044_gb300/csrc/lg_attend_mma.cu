@@ -205,86 +205,112 @@ __device__ __forceinline__ ChunkId decode_chunk(const AttendArgs &a, int c, cons
 // out = o, stats = {M ln 2, l, ln l - u ln 2 / l, sigma / l}.  The partials were written by
 // other CTAs of this launch: read through L2.  Lane j holds chunk j's {M, l, u, sigma} (up to
 // 32 chunks; more are read again per block), and the o slices of up to eight chunks are loaded
-// with them, so a head of a group of at most eight chunks costs one round trip.
-template <int D, int G>
-__device__ __forceinline__ void merge_group(const AttendArgs &a, int64_t head0, int n,
-                                            int chunk_rows, int lane) {
+// with them; heads go two at a time (an even G of 4 or more), so a group of at most eight
+// chunks costs one round trip per pair of heads.
+template <int D, int H>
+__device__ __forceinline__ void merge_heads(const AttendArgs &a, int64_t head_first, int nch,
+                                            int lane) {
   constexpr int EPL = D / 32;
   constexpr int kBlk = 8;
-  const int nch = (n + chunk_rows - 1) / chunk_rows;
-  for (int h = 0; h < G; ++h) {
-    const int64_t head = head0 + h;
-    const float *pp = a.partial + head * a.max_chunks * (D + 8);
-    float ob[kBlk][EPL];
+  const float *pp[H];
+  float ob[H][kBlk][EPL];
+  float4 sl[H];
+#pragma unroll
+  for (int hh = 0; hh < H; ++hh) {
+    pp[hh] = a.partial + (head_first + hh) * a.max_chunks * (D + 8);
 #pragma unroll
     for (int jj = 0; jj < kBlk; ++jj)
 #pragma unroll
       for (int k = 0; k < EPL; ++k)
-        ob[jj][k] = jj < nch ? __ldcg(pp + (int64_t)jj * (D + 8) + 8 + lane + 32 * k) : 0.f;
-    float4 sl = make_float4(-INFINITY, 0.f, 0.f, 0.f);  // this lane's chunk (j = lane)
-    if (lane < nch) sl = __ldcg(reinterpret_cast<const float4 *>(pp + (int64_t)lane * (D + 8)));
-    float M = sl.x;
-    for (int j = lane + 32; j < nch; j += 32) M = fmaxf(M, __ldcg(pp + (int64_t)j * (D + 8)));
+        ob[hh][jj][k] =
+            jj < nch ? __ldcg(pp[hh] + (int64_t)jj * (D + 8) + 8 + lane + 32 * k) : 0.f;
+    sl[hh] = make_float4(-INFINITY, 0.f, 0.f, 0.f);  // this lane's chunk (j = lane)
+    if (lane < nch)
+      sl[hh] = __ldcg(reinterpret_cast<const float4 *>(pp[hh] + (int64_t)lane * (D + 8)));
+  }
+  float M[H], l[H], u[H], sg[H], acc[H][EPL];
 #pragma unroll
-    for (int o = 16; o >= 1; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
-    float l = 0.f, u = 0.f, sg = 0.f, acc[EPL];
+  for (int hh = 0; hh < H; ++hh) {
+    M[hh] = sl[hh].x;
+    for (int j = lane + 32; j < nch; j += 32)
+      M[hh] = fmaxf(M[hh], __ldcg(pp[hh] + (int64_t)j * (D + 8)));
 #pragma unroll
-    for (int k = 0; k < EPL; ++k) acc[k] = 0.f;
-    for (int j0 = 0; j0 < nch; j0 += kBlk) {
+    for (int o = 16; o >= 1; o >>= 1) M[hh] = fmaxf(M[hh], __shfl_xor_sync(0xffffffffu, M[hh], o));
+    l[hh] = u[hh] = sg[hh] = 0.f;
+#pragma unroll
+    for (int k = 0; k < EPL; ++k) acc[hh][k] = 0.f;
+  }
+  for (int j0 = 0; j0 < nch; j0 += kBlk) {
+#pragma unroll
+    for (int hh = 0; hh < H; ++hh) {
       if (j0 > 0) {
 #pragma unroll
         for (int jj = 0; jj < kBlk; ++jj)
 #pragma unroll
           for (int k = 0; k < EPL; ++k)
-            ob[jj][k] = j0 + jj < nch
-                            ? __ldcg(pp + (int64_t)(j0 + jj) * (D + 8) + 8 + lane + 32 * k)
-                            : 0.f;
+            ob[hh][jj][k] = j0 + jj < nch
+                                ? __ldcg(pp[hh] + (int64_t)(j0 + jj) * (D + 8) + 8 + lane + 32 * k)
+                                : 0.f;
       }
       // weights of this block's chunks: lane jj < kBlk takes chunk j0 + jj (held by lane
       // j0 + jj when that is below 32, read again otherwise)
       const int j = j0 + lane;
-      float4 sv = make_float4(__shfl_sync(0xffffffffu, sl.x, j & 31),
-                              __shfl_sync(0xffffffffu, sl.y, j & 31),
-                              __shfl_sync(0xffffffffu, sl.z, j & 31),
-                              __shfl_sync(0xffffffffu, sl.w, j & 31));
+      float4 sv = make_float4(__shfl_sync(0xffffffffu, sl[hh].x, j & 31),
+                              __shfl_sync(0xffffffffu, sl[hh].y, j & 31),
+                              __shfl_sync(0xffffffffu, sl[hh].z, j & 31),
+                              __shfl_sync(0xffffffffu, sl[hh].w, j & 31));
       float f = 0.f;
       if (lane < kBlk && j < nch) {
-        if (j >= 32) sv = __ldcg(reinterpret_cast<const float4 *>(pp + (int64_t)j * (D + 8)));
-        f = exp2f(sv.x - M);
-        l += f * sv.y;
-        u += f * (sv.z + (sv.x - M) * sv.y);
-        sg += f * sv.w;
+        if (j >= 32) sv = __ldcg(reinterpret_cast<const float4 *>(pp[hh] + (int64_t)j * (D + 8)));
+        f = exp2f(sv.x - M[hh]);
+        l[hh] += f * sv.y;
+        u[hh] += f * (sv.z + (sv.x - M[hh]) * sv.y);
+        sg[hh] += f * sv.w;
       }
 #pragma unroll
       for (int jj = 0; jj < kBlk; ++jj) {
         const float fj = __shfl_sync(0xffffffffu, f, jj);
 #pragma unroll
-        for (int k = 0; k < EPL; ++k) acc[k] += fj * ob[jj][k];
-      }
-    }
-#pragma unroll
-    for (int o = 16; o >= 1; o >>= 1) {
-      l += __shfl_xor_sync(0xffffffffu, l, o);
-      u += __shfl_xor_sync(0xffffffffu, u, o);
-      sg += __shfl_xor_sync(0xffffffffu, sg, o);
-    }
-    const float inv_l = 1.f / l;
-    __nv_bfloat16 *out = reinterpret_cast<__nv_bfloat16 *>(a.out) + head * D;
-#pragma unroll
-    for (int k = 0; k < EPL; ++k) out[lane + 32 * k] = __float2bfloat16_rn(acc[k] * inv_l);
-    if (lane == 0) {
-      constexpr float kLn2 = 0.69314718055994530942f;
-      float *st = a.stats + head * 4;
-      st[0] = M * kLn2;
-      st[1] = l;
-      st[2] = logf(l) - u * kLn2 * inv_l;
-      st[3] = sg * inv_l;
-      if (a.final_ml) {
-        a.final_ml[head * 2] = M;
-        a.final_ml[head * 2 + 1] = l;
+        for (int k = 0; k < EPL; ++k) acc[hh][k] += fj * ob[hh][jj][k];
       }
     }
   }
+#pragma unroll
+  for (int hh = 0; hh < H; ++hh) {
+#pragma unroll
+    for (int o = 16; o >= 1; o >>= 1) {
+      l[hh] += __shfl_xor_sync(0xffffffffu, l[hh], o);
+      u[hh] += __shfl_xor_sync(0xffffffffu, u[hh], o);
+      sg[hh] += __shfl_xor_sync(0xffffffffu, sg[hh], o);
+    }
+    const int64_t head = head_first + hh;
+    const float inv_l = 1.f / l[hh];
+    __nv_bfloat16 *out = reinterpret_cast<__nv_bfloat16 *>(a.out) + head * D;
+#pragma unroll
+    for (int k = 0; k < EPL; ++k) out[lane + 32 * k] = __float2bfloat16_rn(acc[hh][k] * inv_l);
+    if (lane == 0) {
+      constexpr float kLn2 = 0.69314718055994530942f;
+      float *st = a.stats + head * 4;
+      st[0] = M[hh] * kLn2;
+      st[1] = l[hh];
+      st[2] = logf(l[hh]) - u[hh] * kLn2 * inv_l;
+      st[3] = sg[hh] * inv_l;
+      if (a.final_ml) {
+        a.final_ml[head * 2] = M[hh];
+        a.final_ml[head * 2 + 1] = l[hh];
+      }
+    }
+  }
+}
+
+template <int D, int G>
+__device__ __forceinline__ void merge_group(const AttendArgs &a, int64_t head0, int n,
+                                            int chunk_rows, int lane) {
+  const int nch = (n + chunk_rows - 1) / chunk_rows;
+  // pairs of heads for an even G of 4 or more (measured: at G = 2 the pair is slower)
+  constexpr int H = G % 2 == 0 && G >= 4 ? 2 : 1;
+#pragma unroll 1
+  for (int h = 0; h < G; h += H) merge_heads<D, H>(a, head0 + h, nch, lane);
 }
 
 }  // namespace
