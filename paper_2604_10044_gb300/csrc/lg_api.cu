@@ -48,9 +48,10 @@ lg_status check_token_params(const lg_guard_params *p, const lg_token_params *tp
   return LG_OK;
 }
 
-// rows per chunk (one work item: one CTA of the fp32 path, one loop trip of a persistent CTA
-// of the bf16 path): a multiple of the staging tile, about eight chunks per SM of a 152-SM
-// GB300 for the bf16 path and twelve CTAs per SM for the fp32 path, at most 4096 rows
+// rows per chunk of the fp32 path (one work item: one CTA), a multiple of the staging tile,
+// twelve CTAs per SM of a 152-SM GB300, at most 2048 rows; for the bf16 path it only sizes the
+// workspace (the kernel picks its own chunk rows from the call's lengths, never more chunks
+// per group than the workspace holds): about eight chunks per SM, at most 4096 rows
 int attend_chunk_rows(const lg_cache *c, int n_layers, int max_len) {
   const int tile = lg::attend_tile_rows(c->dtype, c->d);
   const int64_t rows = (int64_t)max_len * c->batch * c->H_kv * n_layers;

@@ -272,7 +272,7 @@ __device__ __forceinline__ int hamming(const uint32_t *x, const uint32_t *y, int
 }
 
 constexpr int kDetectWarps = kDetectThreads / 32;
-constexpr int kStatWarps = 3;  // warps that sum the statistics in fp64 (one per SM sub-partition)
+constexpr int kStatWarps = 3;  // warps that sum the statistics (one per SM sub-partition)
 constexpr int kStatBatch = 8;  // statistics loads a thread has in flight at once
 constexpr float kFixScale = 1099511627776.0f;  // 2^40: statistics summed in 2^-40 units
 constexpr double kFixUnit = 1.0 / 1099511627776.0;
@@ -288,11 +288,13 @@ static_assert(kCmpThreads % 32 == 0, "comparing threads in whole warps");
 //   run[P]    trailing rows (up to the test length) that match the row P earlier.
 //   synced    the length seen by the previous call.
 // When the length grew by exactly one row since the previous call, only the new row i = n-1 is
-// examined: thread t compares it with rows i-1-t, i-1-t-T, ... of the window (T threads) and
-// stops at its first match; the comparison with row i-1-t is also period P = t+1's, so the
-// runs cost nothing more when p_min = 1.  Everything the call reads is loaded up front and the
-// CTA meets at two barriers, the first after every warp has reduced its share (latest match,
-// novel rows, shortest verified period, fp64 statistic sums).  Otherwise (first call, after a
+// examined: the warps after the statistics warps compare it with every row the window and the
+// periods need (the window comparisons double as the period comparisons), a row's 16-byte
+// chunks on consecutive lanes, the distances in shared memory; beside them three warps sum the
+// statistics in 64-bit fixed point.  Then thread t takes window row i-1-t (and i-1-t-T, ...)
+// for the latest match and period P = t+1's run, and the CTA meets at a barrier after every
+// warp has reduced its share (latest match, novel rows, shortest verified period).  Otherwise
+// (first call, after a
 // prune or any other change of the cache) the window and the runs are recomputed: the
 // sketches of the last smem_rows rows are staged in shared memory with a row stride of
 // nwords + 1 words (rows that different lanes read fall in different banks), one warp scans
