@@ -790,6 +790,7 @@ def cpu_baseline(w, workload, target_s=15.0):
     frac = n_seq / w.batch
     sec = sum(times)
     line = {"value": round(frac / sec, 6), "unit": UNIT, "cores": threads, "kind": "oracle",
+            "affinity_cores": len(os.sched_getaffinity(0)),
             "sample": "1 guarded decode step (step 1: attention over the prompt's rows plus the "
                       "new one, %d..%d, detect, budget prune) of %d of the %d sequences, all %d "
                       "layers; value = %d/%d batch steps / %.2f s"
