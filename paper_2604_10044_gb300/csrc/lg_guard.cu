@@ -276,6 +276,31 @@ constexpr int kStatWarps = 3;  // warps that sum the statistics (one per SM sub-
 constexpr int kStatBatch = 8;  // statistics loads a thread has in flight at once
 constexpr float kFixScale = 1099511627776.0f;  // 2^40: statistics summed in 2^-40 units
 constexpr double kFixUnit = 1.0 / 1099511627776.0;
+constexpr long long kFixNever = -0x7fffffffffffffffll - 1;  // "x < bound" never holds
+constexpr long long kFixAlways = 0x7fffffffffffffffll;       // "x >= bound" never holds
+
+// For a count k >= 0 and t formed exactly in fp64 (a float threshold times a count below 2^29):
+// k < t exactly when k < count_bound(t).  For 0 <= k <= m < 2^29 this is also the decision on
+// the fp64 quotient, k / m < theta: with theta = M 2^-e (M < 2^24), k / m is either theta or at
+// least 1 / (m 2^e) away from it, more than half an ulp of theta, so rounding the quotient cannot
+// carry it across theta.  NaN or t <= 0: never.
+__device__ __forceinline__ int count_bound(double t) {
+  if (!(t > 0.0)) return 0;
+  return t > 1073741824.0 ? (1 << 30) : (int)ceil(t);
+}
+
+// For an integer sum x in units of 2^-40 (|x| < 2^62): x 2^-40 < t exactly when x < bound and
+// x 2^-40 >= t exactly when x >= bound, bound = fix_bound(t) (the scaling by 2^40 is exact);
+// a NaN bound takes nan_bound, so that the comparison it feeds fails as the quotient's would.
+__device__ __forceinline__ long long fix_bound(double t, long long nan_bound) {
+  if (t != t) return nan_bound;
+  const double x = t * 1099511627776.0;
+  const double lim = 4611686018427387904.0;  // 2^62
+  if (x >= lim) return 1ll << 62;
+  if (x <= -lim) return -(1ll << 62);
+  return (long long)ceil(x);
+}
+
 constexpr int kCmpWarp0 = kStatWarps + 1;  // the new-row comparisons: warps after ln n's
 constexpr int kCmpThreads = kDetectThreads - kCmpWarp0 * 32;
 constexpr int kCmpBatch = 6;  // comparison chunks a thread has in flight at once
@@ -293,10 +318,11 @@ static_assert(kCmpThreads % 32 == 0, "comparing threads in whole warps");
 // chunks on consecutive lanes, the distances in shared memory; beside them three warps sum the
 // statistics in 64-bit fixed point.  Then thread t takes window row i-1-t (and i-1-t-T, ...)
 // for the latest match and period P = t+1's run, and the CTA meets at a barrier after every
-// warp has reduced its share (latest match, novel rows, shortest verified period).  Otherwise
-// (first call, after a
-// prune or any other change of the cache) the window and the runs are recomputed: the
-// sketches of the last smem_rows rows are staged in shared memory with a row stride of
+// warp has reduced its share (latest match, novel rows, shortest verified period); thread 0 then
+// takes the votes as integer comparisons against bounds that the ln n warp formed beside the
+// sums (no fp64 division after the comparisons) and updates the guard state.  Otherwise (first
+// call, after a prune or any other change of the cache) the window and the runs are recomputed:
+// the sketches of the last smem_rows rows are staged in shared memory with a row stride of
 // nwords + 1 words (rows that different lanes read fall in different banks), one warp scans
 // each window row, one warp each period.
 __global__ void __launch_bounds__(kDetectThreads, 1) detect_kernel(DetectArgs a) {
@@ -307,7 +333,8 @@ __global__ void __launch_bounds__(kDetectThreads, 1) detect_kernel(DetectArgs a)
   __shared__ int w_latest[kDetectWarps], w_nov[kDetectWarps], w_nov_tail[kDetectWarps],
       w_pstar[kDetectWarps];
   __shared__ double s_logn;
-  __shared__ int s_sig[4];  // vote 1, vote 2, vote 3, stall
+  __shared__ long long s_bound_ent, s_bound_lift;  // vote bounds in 2^-40 units, see (1)
+  __shared__ int s_bound_ttr, s_bound_stall;         // vote bounds on row counts
   __shared__ int s_novel, s_novel_tail, s_pstar, s_mismatch, s_trig, s_span_lo, s_span_hi,
       s_level;
   const int b = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -378,7 +405,20 @@ __global__ void __launch_bounds__(kDetectThreads, 1) detect_kernel(DetectArgs a)
       red_ok[warp] = finite;
     }
   } else if (warp == kStatWarps && lane == 0) {
-    s_logn = n >= 2 ? log((double)n) : 1.0;
+    // ln n and the bounds of the votes, so that (3) compares counts and fixed-point sums:
+    //   vote 1  novel / w < theta_ttr               <=>  novel < count_bound(theta_ttr w)
+    //   stall   tail / stall_len < theta_nov         <=>  tail < count_bound(theta_nov stall_len)
+    //   vote 2  sum H / (L H_q ln n) < theta_ent     <=>  e_fix < fix_bound(theta_ent L H_q ln n)
+    //   vote 3  sum S n / (W_s L H_q) >= theta_lift  <=>  l_fix >= fix_bound(theta_lift W_s L H_q / n)
+    const double logn = n >= 2 ? log((double)n) : 1.0;
+    const int n1 = max(n, 1);
+    s_logn = logn;
+    s_bound_ttr = count_bound((double)p.theta_ttr * (double)w);
+    s_bound_stall = count_bound((double)p.theta_nov * (double)p.stall_len);
+    s_bound_ent = fix_bound((double)p.theta_ent * (double)nh * logn, kFixNever);
+    s_bound_lift = fix_bound((double)p.theta_lift * (double)min(p.suffix_w, n1) * (double)nh /
+                                 (double)n1,
+                             kFixAlways);
   }
 
   if (incr) {
@@ -539,79 +579,78 @@ __global__ void __launch_bounds__(kDetectThreads, 1) detect_kernel(DetectArgs a)
       const int span_len = max(p.m_rep * P, p.l_min);
       if (n >= span_len + P && run[pi] >= span_len) atomicMin(&s_pstar, P);
     }
+    __syncthreads();
   }
-  __syncthreads();
-
-  // (3) the votes and the stall gate, one quotient per warp (different sub-partitions)
-  const int Ws = min(p.suffix_w, n);
-  if (lane == 0 && warp < 4 && n >= 1) {
-    if (warp == 0) {
-      // vote 2: mean of H / ln n over every layer and head
-      long long e_fix = 0;
-      int ok = 1;
+  // (3) the votes, the stall gate and the trigger, on thread 0: integer comparisons against the
+  // bounds formed in (1), then the guard state's update.  The recompute path's counts arrive by
+  // shared-memory atomics (its own barrier above); the incremental path's are thread 0's own.
+  if (tid == 0) {
+    int trig = 0, sig1 = 0, sig2 = 0, sig3 = 0, stall = 0;
+    const bool tailrep = s_pstar != 0x7fffffff;
+    long long e_fix = 0, l_fix = 0;
+    int ok = 1;
+    if (n >= 1) {
       for (int k = 0; k < kStatWarps; ++k) {
         e_fix += red_e[k];
-        ok &= red_ok[k];
-      }
-      const double e_sum = ok ? (double)e_fix * kFixUnit : (double)NAN;
-      const double ebar = n >= 2 ? e_sum / ((double)nh * s_logn) : 1.0;
-      s_sig[1] = ebar < p.theta_ent;
-      if (a.diag) a.diag[8 * b] = ebar;
-    } else if (warp == 1) {
-      // vote 3: mean of S * n / W_s over every layer and head
-      long long l_fix = 0;
-      int ok = 1;
-      for (int k = 0; k < kStatWarps; ++k) {
         l_fix += red_l[k];
         ok &= red_ok[k];
       }
+      sig1 = s_novel < s_bound_ttr;
+      sig2 = n >= 2 ? ok && e_fix < s_bound_ent : 1.0 < (double)p.theta_ent;
+      sig3 = ok && l_fix >= s_bound_lift;
+      stall = w >= p.stall_len && p.stall_len > 0 && s_novel_tail < s_bound_stall;
+      trig = st_a.x >= p.t_min && st_a.y == 0 && sig1 + sig2 + sig3 >= p.K && (stall || tailrep);
+    }
+    if (a.diag && n >= 1) {
+      // the quotients themselves (tests and diagnostics only): mean H / ln n, mean S n / W_s,
+      // novel-row fraction
+      double *dg = a.diag + 8 * b;
+      const double e_sum = ok ? (double)e_fix * kFixUnit : (double)NAN;
       const double l_sum = ok ? (double)l_fix * kFixUnit : (double)NAN;
-      const double lbar = l_sum * (double)n / ((double)Ws * (double)nh);
-      s_sig[2] = lbar >= p.theta_lift;
-      if (a.diag) a.diag[8 * b + 1] = lbar;
-    } else if (warp == 2) {
-      // vote 1: novel-row fraction of the window
-      const double ttr = (double)s_novel / (double)w;
-      s_sig[0] = ttr < p.theta_ttr;
-      if (a.diag) a.diag[8 * b + 2] = ttr;
-    } else {
-      s_sig[3] = w >= p.stall_len && p.stall_len > 0 &&
-                 (double)s_novel_tail / (double)p.stall_len < p.theta_nov;
+      dg[0] = n >= 2 ? e_sum / ((double)nh * s_logn) : 1.0;
+      dg[1] = l_sum * (double)n / ((double)min(p.suffix_w, n) * (double)nh);
+      dg[2] = (double)s_novel / (double)w;
+      dg[3] = sig1;
+      dg[4] = sig2;
+      dg[5] = sig3;
+      dg[6] = stall;
+      dg[7] = tailrep ? s_pstar : 0;
     }
-  }
-  __syncthreads();
-
-  // (4) gates and the trigger
-  if (tid == 0) {
-    int trig = 0;
-    if (n >= 1) {
-      const int sig1 = s_sig[0], sig2 = s_sig[1], sig3 = s_sig[2], stall = s_sig[3];
-      const int warn = sig1 + sig2 + sig3 >= p.K;
-      const int tailrep = s_pstar != 0x7fffffff;
-      trig = st_a.x >= p.t_min && st_a.y == 0 && warn && (stall || tailrep);
-      if (a.diag) {
-        double *dg = a.diag + 8 * b;
-        dg[3] = sig1;
-        dg[4] = sig2;
-        dg[5] = sig3;
-        dg[6] = stall;
-        dg[7] = tailrep ? s_pstar : 0;
-      }
+    // state: x = t_gen, y = cd, z = level, w = last_trig; st_b.x = n_int
+    if (trig) {
+      const bool quick = st_a.x - st_a.w <= p.retrig_window;
+      st_a.z = quick ? min(st_a.z + 1, p.level_max) : 0;
+      st_a.w = st_a.x;
+      st_a.y = p.cooldown;
+      st_b.x += 1;
+    } else if (st_a.y > 0) {
+      st_a.y -= 1;
     }
+    st_a.x += 1;
+    reinterpret_cast<int4 *>(a.state + b)[0] = st_a;
+    reinterpret_cast<int4 *>(a.state + b)[1] = st_b;
+    ds[0] = n;
+    a.flags[b] = trig;
+    if (!(trig && tailrep)) {
+      a.spans[2 * b] = 0;
+      a.spans[2 * b + 1] = 0;
+      s_span_lo = 0;
+      s_span_hi = 0;
+    }
+    s_level = st_a.z;
     s_trig = trig;
     s_mismatch = -1;
   }
   __syncthreads();
 
-  // (5) span: extend the verified tail back while rows keep matching the row P* earlier
+  // (4) span: extend the verified tail back while rows keep matching the row P* earlier
   const int trig = s_trig;
   const int Pstar = s_pstar;
   const int R = B / 2;
-  int s = 0;
   if (trig && Pstar != 0x7fffffff) {
     const int span_len = max(p.m_rep * Pstar, p.l_min);
     const int lo_ext = max(Pstar, n - R);
-    s = n - span_len;
+    int s = n - span_len;
     if (s < lo_ext) {
       s = lo_ext;
     } else {
@@ -627,40 +666,25 @@ __global__ void __launch_bounds__(kDetectThreads, 1) detect_kernel(DetectArgs a)
       if (s_mismatch >= 0) s = s_mismatch + 1;
       else s = lo_ext;
     }
-  }
-  if (tid == 0) {
-    int lo = 0, hi = 0;
-    if (trig && Pstar != 0x7fffffff) {
-      lo = max(max(s - Pstar, n - R), 0);
-      hi = n;
+    if (tid == 0) {
+      const int lo = max(max(s - Pstar, n - R), 0);
+      a.spans[2 * b] = lo;
+      a.spans[2 * b + 1] = n;
+      s_span_lo = lo;
+      s_span_hi = n;
     }
-    a.flags[b] = trig;
-    a.spans[2 * b] = lo;
-    a.spans[2 * b + 1] = hi;
-    // x = t_gen, y = cd, z = level, w = last_trig; st_b.x = n_int
-    if (trig) {
-      const bool quick = st_a.x - st_a.w <= p.retrig_window;
-      st_a.z = quick ? min(st_a.z + 1, p.level_max) : 0;
-      st_a.w = st_a.x;
-      st_a.y = p.cooldown;
-      st_b.x += 1;
-    } else if (st_a.y > 0) {
-      st_a.y -= 1;
-    }
-    st_a.x += 1;
-    reinterpret_cast<int4 *>(a.state + b)[0] = st_a;
-    reinterpret_cast<int4 *>(a.state + b)[1] = st_b;
-    ds[0] = n;
-    s_span_lo = lo;
-    s_span_hi = hi;
-    s_level = st_a.z;
   }
   if (a.kept_idx) {
-    // (6) the retained set of this sequence from the decision just taken
-    __syncthreads();
-    const int code = write_keep(a.c, b, n, B, trig, s_span_lo, s_span_hi, s_level, p,
-                                a.kept_idx, a.kept_count, a.max_keep, a.max_len, tid,
-                                kDetectThreads);
+    // (5) the retained set of this sequence from the decision just taken; a sequence that
+    // neither triggered nor outgrew its budget only marks "no prune"
+    int code = 0;
+    if (trig || n > B) {
+      __syncthreads();  // thread 0's span and level
+      code = write_keep(a.c, b, n, B, trig, s_span_lo, s_span_hi, s_level, p, a.kept_idx,
+                        a.kept_count, a.max_keep, a.max_len, tid, kDetectThreads);
+    } else if (tid == 0) {
+      a.kept_count[b] = -1;
+    }
     if (code && tid == 0) set_status(a.c.dev_status, code);
   }
 }
