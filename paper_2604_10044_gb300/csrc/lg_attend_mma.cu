@@ -3,7 +3,7 @@
 //
 // Persistent CTAs (one per SM) start on chunks blockIdx.x and blockIdx.x + gridDim.x and take
 // further chunks from a shared counter, each a run of consecutive rows of one (layer,
-// sequence, kv-head), sized in the kernel from the lengths of the call (6 to 16 chunks per
+// sequence, kv-head), sized in the kernel from the lengths of the call (4 to 16 chunks per
 // CTA).  A producer warp streams 128-row K and V tiles into a 3-stage shared-memory ring with
 // 2-D tensor copies (cp.async.bulk.tensor, 128-byte swizzle, one box per 64 columns)
 // completing on mbarriers.  Each of four consumer warps owns 32 rows of a tile and all g query
@@ -151,7 +151,7 @@ __device__ __forceinline__ Geom make_geom(const AttendArgs &a, int n_max, int64_
   // every CTA) keeps 64-bit divisions off the prologue
   const float rows_all = (float)len_sum * (float)(a.H_kv * a.n_layers);
   const float per_cta =
-      fminf(fmaxf(floorf(rows_all / (float)(kTile * 8) / (float)ctas), 6.f), 16.f);
+      fminf(fmaxf(floorf(rows_all / (float)(kTile * 8) / (float)ctas), 4.f), 16.f);
   const float cf = ceilf(rows_all / ((float)ctas * per_cta));
   int c = cf >= (float)kMaxChunkRows ? kMaxChunkRows : (int)cf;
   const unsigned nm = (unsigned)n_max;
