@@ -199,11 +199,9 @@ LG_API lg_status lg_decode_attend(const lg_cache *c, int layer0, int n_layers, c
    [batch] (1 = trigger);
    spans: device [batch][2] ([0,0) when empty).
    diag: nullable device [batch][8] fp64, per sequence {mean normalised entropy, mean suffix
-   lift, novel fraction, vote 1, vote 2, vote 3, Stall, P* (0 = no tail repetition)}.  The
-   votes compare exact counts and 64-bit fixed-point sums with bounds formed once per call
-   rather than the quotients: vote 1 and Stall are exactly the quotient decisions; a mean
-   within a few fp64 ulps of theta_ent or theta_lift can land on the other side than the
-   reported quotient.
+   lift, novel fraction, vote 1, vote 2, vote 3, Stall, P* (0 = no tail repetition)}.  Each
+   vote is the fp64 quotient's decision against its threshold (the kernel compares counts and
+   fixed-point sums with bounds and divides only next to a threshold).
    dstate: device, lg_detect_state_size bytes, zero-filled before the first call on a cache and
    after any change of W or of the period range.  It carries the monitor from call to call (for
    each slot the latest earlier matching row, for each period the trailing matching run), so a

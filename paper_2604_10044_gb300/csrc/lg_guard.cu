@@ -276,29 +276,71 @@ constexpr int kStatWarps = 3;  // warps that sum the statistics (one per SM sub-
 constexpr int kStatBatch = 8;  // statistics loads a thread has in flight at once
 constexpr float kFixScale = 1099511627776.0f;  // 2^40: statistics summed in 2^-40 units
 constexpr double kFixUnit = 1.0 / 1099511627776.0;
-constexpr long long kFixNever = -0x7fffffffffffffffll - 1;  // "x < bound" never holds
-constexpr long long kFixAlways = 0x7fffffffffffffffll;       // "x >= bound" never holds
-
-// For a count k >= 0 and t formed exactly in fp64 (a float threshold times a count below 2^29):
-// k < t exactly when k < count_bound(t).  For 0 <= k <= m < 2^29 this is also the decision on
-// the fp64 quotient, k / m < theta: with theta = M 2^-e (M < 2^24), k / m is either theta or at
-// least 1 / (m 2^e) away from it, more than half an ulp of theta, so rounding the quotient cannot
-// carry it across theta.  NaN or t <= 0: never.
-__device__ __forceinline__ int count_bound(double t) {
-  if (!(t > 0.0)) return 0;
-  return t > 1073741824.0 ? (1 << 30) : (int)ceil(t);
+// The votes are the decisions of fp64 quotients against fp64 thresholds (vote 1: novel / w <
+// theta_ttr; Stall: tail / stall_len < theta_nov; vote 2: sum H / (L H_q ln n) < theta_ent;
+// vote 3: sum S n / (W_s L H_q) >= theta_lift).  Bounds formed beside the sums decide them
+// without a division except next to the threshold, where the quotient itself is taken, so every
+// vote is exactly the quotient's decision.
+//
+// Count votes, k / m < theta for 0 <= k <= m < 2^29: from t = RN(theta m), whose rounding error
+// is below 2^-23 while |t| < 2^30, a = ceil(t - 2^-20) and z = floor(t + 2^-20) (count_bounds).
+// A count k < a lies below theta m by more than 2^-20 - 2^-23, so k / m lies below theta by more
+// than the quotient's rounding (2^-53 for k <= m); likewise k > z lies above.  Only a count
+// within 2^-20 of theta m (an exact tie, in practice) divides.
+__device__ __forceinline__ int2 count_bounds(double t) {
+  if (t != t) return make_int2(0, -1);  // NaN: every count is "above" (the vote fails)
+  const double d = 0.00000095367431640625;  // 2^-20
+  const double lo = fmin(fmax(t - d, -1.0), 1073741824.0);
+  const double hi = fmin(fmax(t + d, -1.0), 1073741824.0);
+  return make_int2((int)ceil(lo), (int)floor(hi));
 }
 
-// For an integer sum x in units of 2^-40 (|x| < 2^62): x 2^-40 < t exactly when x < bound and
-// x 2^-40 >= t exactly when x >= bound, bound = fix_bound(t) (the scaling by 2^40 is exact);
-// a NaN bound takes nan_bound, so that the comparison it feeds fails as the quotient's would.
-__device__ __forceinline__ long long fix_bound(double t, long long nan_bound) {
-  if (t != t) return nan_bound;
-  const double x = t * 1099511627776.0;
-  const double lim = 4611686018427387904.0;  // 2^62
-  if (x >= lim) return 1ll << 62;
-  if (x <= -lim) return -(1ll << 62);
-  return (long long)ceil(x);
+// The quotients themselves, out of line: they run only next to a threshold, and a call keeps
+// the compiler from evaluating their fp64 divisions on the common path.
+__device__ __noinline__ int count_quotient_below(int k, int m, double theta) {
+  return (double)k / (double)m < theta;
+}
+
+// RN(RN(RN(x 2^-40) mul) / RN(den_a den_b)) against theta: below it, or at least it (at_least)
+__device__ __noinline__ int sum_quotient_vote(long long x, int mul, double den_a, double den_b,
+                                              double theta, int at_least) {
+  const double q = (double)x * kFixUnit * (double)mul / (den_a * den_b);
+  return at_least ? q >= theta : q < theta;
+}
+
+__device__ __forceinline__ bool count_vote(int k, int2 az, int m, double theta) {
+  if (k < az.x) return true;
+  if (k > az.y) return false;
+  return count_quotient_below(k, m, theta);
+}
+
+// Sum votes on a fixed-point sum x (units of 2^-40) against t, the threshold times the quotient's
+// divisor: b = ceil(RN(t) 2^40), and a margin within which the rounded quotient may land on
+// either side of theta (each side carries a few fp64 roundings, relative 2^-50 at most; the
+// margin is 2^-45 of b, plus 4).  x < b - margin is below, x > b + margin above; in between, and
+// for a NaN or out-of-range t (margin < 0), the quotient decides.
+struct FixBound {
+  long long b, margin;
+};
+
+__device__ __forceinline__ FixBound fix_bound(double t) {
+  FixBound f;
+  if (!(fabs(t) < 4194304.0)) {  // NaN, or |t| 2^40 >= 2^62
+    f.b = 0;
+    f.margin = -1;
+    return f;
+  }
+  f.b = (long long)ceil(t * 1099511627776.0);  // the scaling by 2^40 is exact
+  f.margin = ((f.b < 0 ? -f.b : f.b) >> 45) + 4;
+  return f;
+}
+
+// -1: x 2^-40 is below t, +1: above, 0: too close to tell (take the quotient)
+__device__ __forceinline__ int fix_side(long long x, const FixBound &f) {
+  if (f.margin < 0) return 0;
+  if (x < f.b - f.margin) return -1;
+  if (x > f.b + f.margin) return 1;
+  return 0;
 }
 
 constexpr int kCmpWarp0 = kStatWarps + 1;  // the new-row comparisons: warps after ln n's
@@ -319,8 +361,8 @@ static_assert(kCmpThreads % 32 == 0, "comparing threads in whole warps");
 // statistics in 64-bit fixed point.  Then thread t takes window row i-1-t (and i-1-t-T, ...)
 // for the latest match and period P = t+1's run, and the CTA meets at a barrier after every
 // warp has reduced its share (latest match, novel rows, shortest verified period); thread 0 then
-// takes the votes as integer comparisons against bounds that the ln n warp formed beside the
-// sums (no fp64 division after the comparisons) and updates the guard state.  Otherwise (first
+// takes the votes against bounds that the ln n warp formed beside the sums (a division only next
+// to a threshold) and updates the guard state.  Otherwise (first
 // call, after a prune or any other change of the cache) the window and the runs are recomputed:
 // the sketches of the last smem_rows rows are staged in shared memory with a row stride of
 // nwords + 1 words (rows that different lanes read fall in different banks), one warp scans
@@ -333,8 +375,8 @@ __global__ void __launch_bounds__(kDetectThreads, 1) detect_kernel(DetectArgs a)
   __shared__ int w_latest[kDetectWarps], w_nov[kDetectWarps], w_nov_tail[kDetectWarps],
       w_pstar[kDetectWarps];
   __shared__ double s_logn;
-  __shared__ long long s_bound_ent, s_bound_lift;  // vote bounds in 2^-40 units, see (1)
-  __shared__ int s_bound_ttr, s_bound_stall;         // vote bounds on row counts
+  __shared__ FixBound s_bound_ent, s_bound_lift;  // sum-vote bounds, 2^-40 units, see (1)
+  __shared__ int2 s_bound_ttr, s_bound_stall;       // count-vote bounds
   __shared__ int s_novel, s_novel_tail, s_pstar, s_mismatch, s_trig, s_span_lo, s_span_hi,
       s_level;
   const int b = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -405,20 +447,16 @@ __global__ void __launch_bounds__(kDetectThreads, 1) detect_kernel(DetectArgs a)
       red_ok[warp] = finite;
     }
   } else if (warp == kStatWarps && lane == 0) {
-    // ln n and the bounds of the votes, so that (3) compares counts and fixed-point sums:
-    //   vote 1  novel / w < theta_ttr               <=>  novel < count_bound(theta_ttr w)
-    //   stall   tail / stall_len < theta_nov         <=>  tail < count_bound(theta_nov stall_len)
-    //   vote 2  sum H / (L H_q ln n) < theta_ent     <=>  e_fix < fix_bound(theta_ent L H_q ln n)
-    //   vote 3  sum S n / (W_s L H_q) >= theta_lift  <=>  l_fix >= fix_bound(theta_lift W_s L H_q / n)
+    // ln n and the bounds of the votes (see count_vote and fix_side): novel rows against
+    // theta_ttr w, the stall test's tail against theta_nov stall_len, the entropy sum against
+    // theta_ent L H_q ln n, the suffix-mass sum against theta_lift W_s L H_q / n
     const double logn = n >= 2 ? log((double)n) : 1.0;
     const int n1 = max(n, 1);
     s_logn = logn;
-    s_bound_ttr = count_bound((double)p.theta_ttr * (double)w);
-    s_bound_stall = count_bound((double)p.theta_nov * (double)p.stall_len);
-    s_bound_ent = fix_bound((double)p.theta_ent * (double)nh * logn, kFixNever);
-    s_bound_lift = fix_bound((double)p.theta_lift * (double)min(p.suffix_w, n1) * (double)nh /
-                                 (double)n1,
-                             kFixAlways);
+    s_bound_ttr = count_bounds(p.theta_ttr * (double)w);
+    s_bound_stall = count_bounds(p.theta_nov * (double)p.stall_len);
+    s_bound_ent = fix_bound(p.theta_ent * (double)nh * logn);
+    s_bound_lift = fix_bound(p.theta_lift * (double)min(p.suffix_w, n1) * (double)nh / (double)n1);
   }
 
   if (incr) {
@@ -581,8 +619,8 @@ __global__ void __launch_bounds__(kDetectThreads, 1) detect_kernel(DetectArgs a)
     }
     __syncthreads();
   }
-  // (3) the votes, the stall gate and the trigger, on thread 0: integer comparisons against the
-  // bounds formed in (1), then the guard state's update.  The recompute path's counts arrive by
+  // (3) the votes, the stall gate and the trigger, on thread 0, against the bounds formed in (1)
+  // (count_vote, fix_side), then the guard state's update.  The recompute path's counts arrive by
   // shared-memory atomics (its own barrier above); the incremental path's are thread 0's own.
   if (tid == 0) {
     int trig = 0, sig1 = 0, sig2 = 0, sig3 = 0, stall = 0;
@@ -595,10 +633,21 @@ __global__ void __launch_bounds__(kDetectThreads, 1) detect_kernel(DetectArgs a)
         l_fix += red_l[k];
         ok &= red_ok[k];
       }
-      sig1 = s_novel < s_bound_ttr;
-      sig2 = n >= 2 ? ok && e_fix < s_bound_ent : 1.0 < (double)p.theta_ent;
-      sig3 = ok && l_fix >= s_bound_lift;
-      stall = w >= p.stall_len && p.stall_len > 0 && s_novel_tail < s_bound_stall;
+      sig1 = count_vote(s_novel, s_bound_ttr, w, p.theta_ttr);
+      stall = w >= p.stall_len && p.stall_len > 0 &&
+              count_vote(s_novel_tail, s_bound_stall, p.stall_len, p.theta_nov);
+      if (n < 2) {
+        sig2 = 1.0 < p.theta_ent;  // the mean is taken as 1 below two rows
+      } else if (ok) {
+        const int side = fix_side(e_fix, s_bound_ent);
+        sig2 = side ? side < 0 : sum_quotient_vote(e_fix, 1, (double)nh, s_logn, p.theta_ent, 0);
+      }
+      if (ok) {
+        const int side = fix_side(l_fix, s_bound_lift);
+        sig3 = side ? side > 0
+                    : sum_quotient_vote(l_fix, n, (double)min(p.suffix_w, n), (double)nh,
+                                        p.theta_lift, 1);
+      }
       trig = st_a.x >= p.t_min && st_a.y == 0 && sig1 + sig2 + sig3 >= p.K && (stall || tailrep);
     }
     if (a.diag && n >= 1) {
