@@ -23,6 +23,7 @@ import os
 import statistics
 import subprocess
 import sys
+import tempfile
 import time
 
 ROOT = os.path.dirname(os.path.abspath(__file__))
@@ -131,8 +132,10 @@ class Clocks:
               "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
 
     def __init__(self, gpu_index, enabled=True):
+        """the raw samples go to $LG_CLOCKS_DIR (default: the system temporary directory)"""
         self.proc = None
-        self.path = os.path.join(ROOT, "gpurun_out", "clocks_bench_%d.csv" % gpu_index)
+        self.path = os.path.join(os.environ.get("LG_CLOCKS_DIR") or tempfile.gettempdir(),
+                                 "clocks_bench_%d.csv" % gpu_index)
         if not enabled:
             return
         os.makedirs(os.path.dirname(self.path), exist_ok=True)
