@@ -211,3 +211,86 @@ def test_short_sequences():
     sk = np.zeros((1, 8), dtype=np.uint32)
     flag, span, diag = oracle.detect(_stats_for(1.0, 1.0, 1, 2, 2, 2)[:, :, :], sk, 256, prm, st)
     assert flag == 0 and span == (0, 0) and diag["ttr"] == 1.0
+
+
+# --------------------------------------------------------------------------- threshold boundaries
+
+def test_entropy_vote_normalises_by_ln_n():
+    """stats with H = c ln n in every head give a mean normalised entropy of exactly c (up to
+    rounding), for any n: the divisor is ln n (Sec. 5.2's concentration signal restated)"""
+    rng = np.random.default_rng(12)
+    for n in (2, 100, 4096):
+        sk = _sketches(rng, n, 4)
+        for c in (0.3, 0.9):
+            _, _, diag = oracle.detect(_stats_for(c, 1.0, 2, 3, n, min(64, n)), sk, 8192,
+                                       oracle.params(), oracle.new_state())
+            assert diag["ebar"] == pytest.approx(c, rel=1e-12), (n, c)
+
+
+def test_votes_are_strict_at_their_thresholds():
+    """vote 1 fires for a novel fraction below theta_ttr, not at it; vote 2 for a mean
+    normalised entropy below theta_ent, not at it (Eq. 8)"""
+    rng = np.random.default_rng(13)
+    base = _sketches(rng, 2, 4)
+    sk = np.stack([base[i % 2] for i in range(10)])      # rows 0 and 1 novel, the rest repeats
+    prm = oracle.params(W=10, stall_len=4)
+    _, _, diag = oracle.detect(_stats_for(0.9, 1.0, 1, 2, 10, 10), sk, 4096, prm,
+                               oracle.new_state())
+    assert diag["ttr"] == 0.2 and diag["sig1"] == 0      # 2 / 10 == theta_ttr: no vote
+    sk1 = np.stack([base[0]] * 10)
+    _, _, diag = oracle.detect(_stats_for(0.9, 1.0, 1, 2, 10, 10), sk1, 4096, prm,
+                               oracle.new_state())
+    assert diag["ttr"] == 0.1 and diag["sig1"] == 1
+    # the entropy vote at exactly theta_ent: take theta_ent from the oracle's own mean
+    stats = _stats_for(0.6, 1.0, 2, 3, 300, 64)
+    sk300 = _sketches(rng, 300, 4)
+    _, _, d0 = oracle.detect(stats, sk300, 4096, oracle.params(), oracle.new_state())
+    e = d0["ebar"]
+    _, _, d1 = oracle.detect(stats, sk300, 4096, oracle.params(theta_ent=e), oracle.new_state())
+    assert d1["sig2"] == 0
+    _, _, d2 = oracle.detect(stats, sk300, 4096, oracle.params(theta_ent=float(np.nextafter(e, 2.0))),
+                             oracle.new_state())
+    assert d2["sig2"] == 1
+
+
+def test_stall_counts_the_first_row_of_its_tail():
+    """Stall looks at the last theta_stall = 4 rows: one novel row among them (the earliest,
+    n - 4) gives a novel fraction of 1/4 >= theta_nov, so no stall; with it repeated too, stall"""
+    rng = np.random.default_rng(14)
+    sk = _sketches(rng, 20, 4)
+    sk[17:20] = sk[0:3]                                  # rows 17..19 repeat earlier rows
+    prm = oracle.params(W=20, stall_len=4)
+    _, _, diag = oracle.detect(_stats_for(0.9, 1.0, 1, 2, 20, 20), sk, 4096, prm,
+                               oracle.new_state())
+    assert diag["stall"] == 0                            # row 16 is novel
+    sk[16] = sk[5]
+    _, _, diag = oracle.detect(_stats_for(0.9, 1.0, 1, 2, 20, 20), sk, 4096, prm,
+                               oracle.new_state())
+    assert diag["stall"] == 1
+
+
+def test_tail_repetition_needs_l_min_rows():
+    """TailRep checks the last max(m_rep P, l_min) rows (App. B.2 debounce): a period-4 repeat
+    over the last 20 rows is not enough with l_min = 32 (m_rep P = 12), over the last 40 it is"""
+    rng = np.random.default_rng(15)
+    prm = oracle.params(m_rep=3, l_min=32, p_min=1, p_max=16)
+    for tail, P in ((20, 0), (40, 4)):
+        n = 100
+        sk = _sketches(rng, n, 4, 4, n - tail)
+        _, _, diag = oracle.detect(_stats_for(0.9, 1.0, 1, 2, n, 64), sk, 4096, prm,
+                                   oracle.new_state())
+        assert int(diag["P"]) == P, tail
+
+
+def test_retrigger_exactly_at_the_window_escalates():
+    """a trigger exactly retrig_window = 64 steps after the previous one counts as 'shortly
+    after' (Sec. 5.3) and raises the level; one step later it resets the level"""
+    rng = np.random.default_rng(16)
+    n = 300
+    sk = _sketches(rng, n, 8, 5, 40)
+    stats = _stats_for(0.5, 3.0, 1, 4, n, 64)
+    for gap, level in ((64, 2), (65, 0)):
+        st = oracle.new_state(t_gen=200)
+        st.level, st.last_trig = 1, 200 - gap
+        f, _, _ = oracle.detect(stats, sk, 4096, oracle.params(), st)
+        assert f == 1 and st.level == level, gap

@@ -154,3 +154,40 @@ def test_streaming_select_brute_force(seed):
     assert kept.tolist() == expect and len(kept) == B
     x = oracle.streaming_oldest(pos, 4)
     assert pos[x] == 4                       # positions 0..n-1 are all present
+
+
+def test_budget_event_prunes_at_level_zero():
+    """a budget event (no trigger) keeps B/4 recent rows whatever level the guard is at; only a
+    trigger prunes at the progressive level (Sec. 5.3)"""
+    prm = oracle.params()
+    base = oracle.keep_set(8193, 4096, 0, (0, 0), 0, prm)
+    for level in (1, 2, 3):
+        assert np.array_equal(oracle.keep_set(8193, 4096, 0, (0, 0), level, prm), base)
+    assert len(oracle.keep_set(8193, 4096, 1, (0, 0), 2, prm)) < len(base)
+
+
+def test_h2o_scores_add_every_head_of_the_group():
+    """four query heads of one kv-head, each attending almost only to its own key row: the
+    accumulated score of each of those rows is about 1, every other row about 0 (the score sums
+    the attention the row receives from every head of its group)"""
+    import synth
+    w = synth.make_workload(2, L=1, batch=1, n=64, budget=64, steps=1, H_q=4, H_kv=1,
+                            tail=(20, 24), periods=(8, 8))
+    n = int(w.n0[0])
+    rng = np.random.default_rng(17)
+    Kf = (rng.standard_normal((w.L, w.H_kv, w.S_total, w.d)) * 0.01).astype(np.float32)
+    qf = np.zeros((w.L, w.batch, w.H_q, w.d), dtype=np.float32)
+    rows = [3, 13, 23, 33]
+    for h, r in enumerate(rows):
+        Kf[0, 0, r, 32 * h:32 * (h + 1)] = 1.0
+        qf[0, 0, h, 32 * h:32 * (h + 1)] = 4.0
+    Vf = rng.standard_normal((w.L, w.H_kv, w.S_total, w.d)).astype(np.float32)
+    from test_oracle_attention import bf16_bits
+    g = oracle.OracleGuard(w, bf16_bits(Kf), bf16_bits(Vf), policy="h2o")
+    g.attend(bf16_bits(qf))
+    sc = g.h2o[0, 0, :n]
+    for r in rows:
+        assert 0.99 < sc[r] < 1.0, r
+    others = np.delete(sc, rows)
+    assert others.max() < 0.01
+    assert sc.sum() == pytest.approx(w.g, rel=1e-12)

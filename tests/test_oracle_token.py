@@ -201,3 +201,41 @@ def test_span_follows_a_contiguous_kept_tail():
         f, span, dg = oracle.token_detect(y[:t + 1], pm[t], n, prm, tp, st, ts, kept=kept)
     assert f == 1 and span == (n - L_star, n)
     assert ts.appended == 400 + 50
+
+
+# --------------------------------------------------------------------------- threshold boundaries
+
+def _last_diag(tokens, pmax, prm, tp):
+    st, ts = oracle.new_state(0), oracle.new_token_state()
+    dg = None
+    for t in range(len(tokens)):
+        _, _, dg = oracle.token_detect(tokens[:t + 1], pmax, 4000 + t + 1, prm, tp, st, ts)
+    return dg
+
+
+def test_token_votes_are_strict_at_their_thresholds():
+    """W = 25, CR evaluated every token: the period-2 window 1 2 1 2 ... 1 of 25 tokens parses
+    into 3 phrases, CR = 3/25 = theta_cr = 0.12, so the redundancy vote does not fire (strictly
+    below); the window 1 2 3 4 5 1 1 ... 1 has 5 distinct of 25 tokens, TTR = 0.2 = theta_ttr,
+    so the diversity vote does not fire either"""
+    prm = oracle.params(W=25, t_min=10_000)
+    tp = oracle.token_params(cr_every=1)
+    dg = _last_diag((np.arange(25) % 2 + 1).astype(np.int32), 0.5, prm, tp)
+    assert dg["cr"] == 3 / 25 and dg["sig2"] == 0
+    assert dg["sig1"] == 1                                # TTR 2/25 < 0.2
+    dg = _last_diag(np.array([1, 2, 3, 4, 5] + [1] * 20, dtype=np.int32), 0.5, prm, tp)
+    assert dg["ttr"] == 5 / 25 and dg["sig1"] == 0
+
+
+def test_streak_vote_fires_at_theta_streak():
+    """the confidence vote fires once the streak reaches theta_streak = 6 steps (Eq. 8: >=)"""
+    prm = oracle.params(t_min=10_000)
+    tp = oracle.token_params()
+    toks = (np.arange(200) + 7).astype(np.int32)
+    pm = np.full(200, 0.95)
+    st, ts = oracle.new_state(0), oracle.new_token_state()
+    seen = []
+    for t in range(8):
+        _, _, dg = oracle.token_detect(toks[:t + 1], pm[t], 4000 + t + 1, prm, tp, st, ts)
+        seen.append((int(dg["streak"]), int(dg["sig3"])))
+    assert seen[4] == (5, 0) and seen[5] == (6, 1) and seen[6] == (7, 1)
