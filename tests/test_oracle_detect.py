@@ -294,3 +294,37 @@ def test_retrigger_exactly_at_the_window_escalates():
         st.level, st.last_trig = 1, 200 - gap
         f, _, _ = oracle.detect(stats, sk, 4096, oracle.params(), st)
         assert f == 1 and st.level == level, gap
+
+
+def test_lift_of_a_cache_shorter_than_the_suffix():
+    """W_s = min(64, n): with n = 40 rows the suffix is the whole cache, S = 1 and the lift is
+    exactly 1 (uniform attention's value), not 40 / 64"""
+    rng = np.random.default_rng(18)
+    n = 40
+    stats = np.zeros((1, 2, 4))
+    stats[..., 2] = 0.5 * math.log(n)
+    stats[..., 3] = 1.0
+    _, _, diag = oracle.detect(stats, _sketches(rng, n, 4), 4096, oracle.params(),
+                               oracle.new_state())
+    assert diag["lbar"] == 1.0
+
+
+def test_stall_with_a_window_of_exactly_theta_stall_rows():
+    """the stall test runs once the window holds theta_stall rows (w >= theta_stall): four
+    identical rows have one novel row, 1/4 < theta_nov = 0.5"""
+    sk = np.zeros((4, 4), dtype=np.uint32)
+    prm = oracle.params(W=4, stall_len=4, theta_nov=0.5)
+    _, _, diag = oracle.detect(_stats_for(0.9, 1.0, 1, 2, 4, 4), sk, 4096, prm,
+                               oracle.new_state())
+    assert diag["stall"] == 1
+
+
+def test_tail_repetition_at_the_shortest_cache_that_can_show_it():
+    """a period P is testable once n >= max(m_rep P, l_min) + P: a cache of exactly 12 + 4 rows
+    repeating with period 4 (m_rep 3, l_min 6) reports P = 4"""
+    rng = np.random.default_rng(19)
+    sk = _sketches(rng, 16, 4, 4, 4)
+    prm = oracle.params(m_rep=3, l_min=6, p_min=4, p_max=8)
+    _, _, diag = oracle.detect(_stats_for(0.9, 1.0, 1, 2, 16, 16), sk, 4096, prm,
+                               oracle.new_state())
+    assert int(diag["P"]) == 4

@@ -191,3 +191,10 @@ def test_h2o_scores_add_every_head_of_the_group():
     others = np.delete(sc, rows)
     assert others.max() < 0.01
     assert sc.sum() == pytest.approx(w.g, rel=1e-12)
+
+
+def test_a_cache_exactly_at_its_budget_is_not_pruned():
+    """Sec. 5.3 prunes on a trigger or when the cache outgrows B: n == B keeps every row"""
+    prm = oracle.params()
+    assert np.array_equal(oracle.keep_set(4096, 4096, 0, (0, 0), 0, prm), np.arange(4096))
+    assert len(oracle.keep_set(4097, 4096, 0, (0, 0), 0, prm)) < 4096

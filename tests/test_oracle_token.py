@@ -24,6 +24,8 @@ import oracle
     ([1, 2, 3, 1, 2, 4, 1, 2, 3], 6),  # 1 | 2 | 3 | ref(1 2) | 4 | ref(1 2 3)
     # a b r a c a d a b r a: a | b | r | a | c | a | d | ref(a b r a)
     ([1, 2, 3, 1, 4, 1, 5, 1, 2, 3, 1], 8),
+    # the longest earlier match wins, not the first: 1 | 2 | 9 | ref(1 2) | 3 | ref(1 2 3)
+    ([1, 2, 9, 1, 2, 3, 1, 2, 3], 6),
 ])
 def test_lz77_hand_worked(x, phrases):
     assert oracle.lz77_phrases(x) == phrases
@@ -239,3 +241,17 @@ def test_streak_vote_fires_at_theta_streak():
         _, _, dg = oracle.token_detect(toks[:t + 1], pm[t], 4000 + t + 1, prm, tp, st, ts)
         seen.append((int(dg["streak"]), int(dg["sig3"])))
     assert seen[4] == (5, 0) and seen[5] == (6, 1) and seen[6] == (7, 1)
+
+
+def test_span_reaches_back_no_further_than_the_kept_history():
+    """the span extends back over tokens the monitor still holds (the last hist tokens): with
+    hist = 64 the loop's span is exactly those 64 tokens, with the default 512 it is the whole
+    loop (its L* tokens, first period included)"""
+    H, P = 300, 8
+    L_star = math.floor(256 + P - 51.2) + 1
+    y = _healthy_then_loop(H, P, L_star)
+    pm = np.where(np.arange(len(y)) >= H, 0.95, 0.5)
+    for hist, length in ((64, 64), (512, L_star)):
+        ev, _, _ = _run(y, pm, prm=oracle.params(), tp=oracle.token_params(hist=hist))
+        t, span, dg, n = ev[0]
+        assert span[1] - span[0] == length, (hist, span)
