@@ -436,12 +436,39 @@ def traffic_from_profile(kernel_src_hash):
     return d
 
 
+def code_only(src):
+    """C/C++/CUDA source without its comments, runs of white space as one space: an edit of a
+    comment or of the layout leaves it unchanged, any edit of the code does not"""
+    out, i, n = [], 0, len(src)
+    while i < n:
+        c = src[i]
+        if c == '"' or c == "'":                      # a literal, copied whole
+            j = i + 1
+            while j < n and src[j] != c:
+                j += 2 if src[j] == "\\" else 1
+            out.append(src[i:j + 1])
+            i = j + 1
+        elif src.startswith("//", i):
+            j = src.find("\n", i)
+            i = n if j < 0 else j
+        elif src.startswith("/*", i):
+            j = src.find("*/", i + 2)
+            out.append(" ")
+            i = n if j < 0 else j + 2
+        else:
+            out.append(c)
+            i += 1
+    return " ".join("".join(out).split())
+
+
 def source_hash():
+    """sha256 of the attention kernel's code (comments and layout excluded): the committed
+    DRAM-traffic summary holds the value for the code it was captured on"""
     import hashlib
     h = hashlib.sha256()
     for f in ("lg_attend_mma.cu", "lg_common.cuh"):
-        with open(os.path.join(ROOT, "paper_2604_10044_gb300", "csrc", f), "rb") as fh:
-            h.update(fh.read())
+        with open(os.path.join(ROOT, "paper_2604_10044_gb300", "csrc", f)) as fh:
+            h.update(code_only(fh.read()).encode())
     return h.hexdigest()
 
 

@@ -134,9 +134,10 @@ struct ChunkId {
 // Chunk geometry of one call, from the lengths it attends over (the host sizes the workspace
 // for max_len, which can be far above them): chunk rows a multiple of the tile, never more
 // chunks per group than the workspace holds (max_chunks).  A CTA takes about one chunk per
-// eight of its tiles, at least 6 (a chunk end costs the consumers a hand-off) and at most 16
-// (measured: finer chunks gained nothing at the end of long passes and cost a little on the
-// way); the rows are then evened out over the chunks of the longest group.
+// eight of its tiles, at least 4 (a chunk end costs the consumers a hand-off, and a short pass
+// with fewer, longer chunks measured faster) and at most 16 (measured: finer chunks gained
+// nothing at the end of long passes and cost a little on the way); the rows are then evened
+// out over the chunks of the longest group.
 struct Geom {
   int rows;        // rows per chunk
   int per_grp;     // chunk ids per (layer, sequence, kv-head)
