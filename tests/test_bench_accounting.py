@@ -45,3 +45,11 @@ def test_traffic_summary_is_gated_on_the_kernel_source():
     assert 0.8 * 512 < d["dram_bytes_per_row"] < 1.1 * 512
     got = bench.traffic_from_profile(d["source_sha256"])
     assert got is not None and got["dram_bytes_per_row"] == d["dram_bytes_per_row"]
+
+
+def test_traffic_gate_ignores_comments_not_code():
+    src = 'int a = 1;  // rows\n/* chunks\n   per CTA */\nconst char *s = "// kept";\n'
+    same = 'int a = 1;\nconst char *s = "// kept";  /* a new comment */\n'
+    assert bench.code_only(src) == bench.code_only(same)
+    assert bench.code_only(src) != bench.code_only(src.replace("a = 1", "a = 2"))
+    assert '"// kept"' in bench.code_only(src)
