@@ -288,7 +288,6 @@ class OracleGuard:
         self.cap = w.cap.astype(np.int32)
         self.off = w.seq_off.astype(np.int64)
         self.nwords = w.H_kv * w.d // 32
-        self.thr = int(math.floor(self.prm.tau_ham * self.nwords * 32))
         self.sk = np.zeros((w.S_total, self.nwords), dtype=np.uint32)
         for b in range(w.batch):
             for i in range(int(self.len[b])):

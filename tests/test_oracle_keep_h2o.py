@@ -112,8 +112,9 @@ def test_h2o_select_brute_force(seed):
 
 
 def test_h2o_path_keeps_budget_and_mass():
-    """whole-step H2O comparator on a tiny workload: length <= B after every step and the
-    scores of every (layer, kv-head) stream sum to g * (steps seen) minus the evicted mass"""
+    """whole-step H2O comparator on a tiny workload: length <= B after every step, distinct
+    positions in every (layer, kv-head) stream, the B/2 most recent positions all present (the
+    scores' bookkeeping: tests/test_oracle_guard_steps.py)"""
     import synth
     w = synth.make_workload(2, L=2, batch=3, n=200, budget=128, steps=6, H_q=4, H_kv=2,
                             tail=(60, 80), periods=(5, 9))
