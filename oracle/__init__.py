@@ -42,7 +42,7 @@ class State(ctypes.Structure):
                 ("pad", ctypes.c_int32 * 3)]
 
 
-# Paper constants (App. B.2, Sec. 6.1) and the build's readings where it is silent.
+# Paper constants (App. B.2, Sec. 6.1) and, where the paper is silent, the readings taken here.
 DEFAULTS = dict(W=256, K=2, t_min=64, cooldown=32, n_anchor=32, stall_len=4, p_min=1, p_max=128,
                 l_min=32, m_rep=3, suffix_w=64, guard_layer=0, level_max=3, retrig_window=64,
                 headroom=64, theta_ttr=0.2, theta_nov=0.02, theta_ent=0.7, theta_lift=2.0,
@@ -62,7 +62,7 @@ class TokenState(ctypes.Structure):
                 ("appended", ctypes.c_int32), ("pad", ctypes.c_int32), ("cr", ctypes.c_double)]
 
 
-# App. B.2 thresholds of the token-level monitor; cr_every and hist are the build's readings.
+# App. B.2 thresholds of the token-level monitor; the paper fixes neither cr_every nor hist.
 TOKEN_DEFAULTS = dict(cr_every=16, theta_streak=6, hist=512, theta_cr=0.12, theta_conf=0.9)
 
 

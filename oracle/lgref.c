@@ -22,7 +22,7 @@
  * lgref_token_detect follows it on those inputs.  A decode path that carries
  * only K/V caches and attention has neither, so lgref_detect restates each
  * signal over attention statistics and sign sketches of the guard layer's V
- * rows.  Where the paper is silent the constants are this build's choice, stated
+ * rows.  Where the paper is silent the constants are chosen here, stated
  * beside each function; tests/test_oracle_*.py pin every function.
  */
 #include "lgref.h"

@@ -4,7 +4,7 @@ interventions come before the loop begins.  Harness only: no attention, detectio
 arithmetic lives here; the caller runs the guard (the GPU path or the oracle) and reports each
 step's decisions back.
 
-Model (the build's reading; the paper's data and models are not available):
+Model (a reading of the paper's setting; its data and models are not available):
   - healthy text: token ids drawn Zipf(1.1) over a 50 000-token vocabulary (so a 256-token
     window repeats tokens, TTR well below 1), top-1 probability uniform in [0.2, 0.8), with
     benign confident runs (a run of 4..12 steps with p_max in [0.9, 1) starts with
