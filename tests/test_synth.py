@@ -77,3 +77,34 @@ def test_workload_shapes(i):
         assert w.n0.min() >= 1024 and w.n0.max() <= 65536
         assert np.array_equal(w.budget, np.minimum(w.n0 + 256, 16384))
     assert np.all(w.cap >= np.maximum(w.n0, w.budget) + 1)
+
+
+def test_paper_shaped_workload():
+    """workload 6: the Qwen3-1.7B shape, one 3853-token prompt, B = 1024, T_max = 2500, a loop
+    whose onset is 800-1300 generated tokens in, with a period of 16-64"""
+    w = synth.make_workload(6)
+    assert (w.L, w.H_q, w.H_kv, w.d, w.dtype, w.batch) == (28, 16, 8, 128, "bf16", 1)
+    assert w.n0.tolist() == [3853] and w.budget.tolist() == [1024] and w.steps == 2500
+    s = w.seqs[0]
+    assert s["looping"] == 1 and 800 <= s["start"] - 3853 <= 1300 and 16 <= s["period"] <= 64
+
+
+@pytest.mark.parametrize("i", [2, 3, 4, 5])
+def test_loop_plans_follow_the_recipe(i):
+    """the planted loops of each full-size workload: periods, tails, starts and onsets drawn from
+    the stated ranges (workload 2: P 16-128, tail 1024-3072; 3: P 8-64, start in
+    [3n/4, n - 4P]; 4: P 16-64, onset 0-200 steps after the prompt; 5: P 32, tail 16384)"""
+    w = synth.make_workload(i)
+    for b in np.flatnonzero(w.seqs["looping"]):
+        s, n = w.seqs[b], int(w.n0[b])
+        P, start = int(s["period"]), int(s["start"])
+        if i == 2:
+            assert 16 <= P <= 128 and 1024 <= n - start <= 3072
+        elif i == 3:
+            assert 8 <= P <= 64 and 3 * n // 4 <= start <= max(3 * n // 4, n - 4 * P)
+        elif i == 4:
+            assert 16 <= P <= 64 and 0 <= start - n <= 200
+        else:
+            assert P == 32 and n - start == 16384
+    if i == 3:
+        assert w.n_sink == 4 and w.sink_factor == 8.0
