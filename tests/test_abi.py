@@ -63,3 +63,15 @@ def test_host_validation_rejects_before_launch():
     assert L.lg_detect_state_size(ctypes.byref(c), ctypes.byref(p)) == 4 * (130 + c.S_total)
     ws = L.lg_workspace_size(ctypes.byref(c), 32, 1, 1000, 0)
     assert ws > 0 and ws % 256 == 0
+
+
+def test_every_status_code_has_its_own_message():
+    """each lg_status value lg.h declares maps to a distinct message; anything else is unknown"""
+    src = open(os.path.join(ROOT, "include", "lg.h")).read()
+    block = src[src.index("typedef enum {"):src.index("} lg_status;")]
+    codes = [int(v) for v in re.findall(r"LG_\w+ = (\d+)", block)]
+    assert codes == list(range(len(codes)))
+    msgs = [lg.lg_status_string(c) for c in codes]
+    assert len(set(msgs)) == len(codes) and "unknown status" not in msgs
+    assert lg.lg_status_string(len(codes)) == "unknown status"
+    assert lg.lg_status_string(-1) == "unknown status"
