@@ -43,12 +43,12 @@ LG_VOTE_FN LG_VOTE_INLINE int2 count_bounds(double t) {
 
 // The quotients themselves, out of line: they run only next to a threshold, and a call keeps
 // the compiler from evaluating their fp64 divisions on the common path.
-LG_VOTE_FN LG_VOTE_NOINLINE int count_quotient_below(int k, int m, double theta) {
+static LG_VOTE_FN LG_VOTE_NOINLINE int count_quotient_below(int k, int m, double theta) {
   return (double)k / (double)m < theta;
 }
 
 // RN(RN(RN(x 2^-40) mul) / RN(den_a den_b)) against theta: below it, or at least it (at_least)
-LG_VOTE_FN LG_VOTE_NOINLINE int sum_quotient_vote(long long x, int mul, double den_a, double den_b,
+static LG_VOTE_FN LG_VOTE_NOINLINE int sum_quotient_vote(long long x, int mul, double den_a, double den_b,
                                               double theta, int at_least) {
   const double q = (double)x * kFixUnit * (double)mul / (den_a * den_b);
   return at_least ? q >= theta : q < theta;
