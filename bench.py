@@ -1,20 +1,24 @@
 #!/usr/bin/env python3
 """Benchmark of the LoopGuard decode path on GB300: guarded decode steps/s.
 
-Workload (default): the Llama-3-8B-shaped decode batch -- 32 layers, 32 query / 8 KV heads,
-head_dim 128, bf16, 8 sequences, cache length 8192, budget 4096, half the sequences carrying a
-planted periodic tail.  Synthetic seeded inputs (the paper's LoopBench prompts and model
-weights are not available); the cache (4.3-8.6 GB) is far larger than L2.
+Workload (default): the bandwidth sweep, the largest of the five -- 32 layers, 64 query / 8 KV
+heads, head_dim 128, bf16, 16 sequences of 131072 cached tokens (275 GB of K/V), budget 32768,
+half the sequences carrying a planted period-32 tail of 16384 tokens.  Synthetic seeded inputs
+(the paper's LoopBench prompts and model weights are not available); every step reads tens of
+GB of K/V, far more than the 129 MB L2.  --workload 1..6 selects the others (2 = the
+Llama-3-8B-shaped decode batch, 6 = the paper's own setting).
 
 One step = one guarded decode step of the whole batch through the C ABI, every kernel of
-the path included: reserve the slot, append the new K/V rows of all 32 layers (+ sketch),
+the path included: reserve the slot, append the new K/V rows of all layers (+ sketch),
 decode attention over the cache fused with the per-head statistics (Eq. 1), the loop-onset
 test (Eq. 8, Eq. 9), the retained set and in-place compaction (Eq. 10, Eq. 11).  A harness
 kernel selects each sequence's next inputs (loop continuation, or loop-free after the guard
 intervened) from buffers generated before timing.  The timed steps start from the freshly
-generated cache, so step 1 carries the budget event of every sequence (8193 -> 4032 rows).
+generated cache, so step 1 carries the budget event of every sequence (131073 -> 32704 rows
+on the default workload) and the later steps read the retained rows.
 
-Prints one JSON line.  --impl reference times the CPU oracle instead (bounded sample).
+Prints one JSON line.  --impl reference times the CPU oracle instead, on a bounded sample of
+the same timed run (the same sample as the GPU line's cpu_baseline).
 """
 import argparse
 import json
@@ -37,15 +41,20 @@ METRIC = "guarded decode steps/s (attend+stats, detect, prune/compact) and achie
 UNIT = "steps/s"
 L2_BYTES = 129e6
 EV_EVERY = 8  # timing events on every 8th timed step
+DEFAULT_STEPS = 400
+DEFAULT_STEPS_W5 = 20   # about 0.25 s of GPU time from the fresh 275 GB cache
+ORACLE_TARGET_S = 20.0  # CPU seconds of the oracle's timed sample (both oracle figures)
 
 
 def parse():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=400)
+    ap.add_argument("--steps", type=int, default=0,
+                    help="timed steps (default: %d on the bandwidth sweep, %d on the others)"
+                         % (DEFAULT_STEPS_W5, DEFAULT_STEPS))
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
-    ap.add_argument("--workload", type=int, default=2)
+    ap.add_argument("--workload", type=int, default=5)
     ap.add_argument("--layers-per-call", type=int, default=0,
                     help="layers per lg_decode_attend call (0 = all layers in one call)")
     ap.add_argument("--no-e2e", action="store_true")
@@ -71,10 +80,12 @@ def parse():
                          "print its measures instead of the step benchmark")
     ap.add_argument("--eager", action="store_true",
                     help="time the steps as eager launches instead of one CUDA graph replay")
-    ap.add_argument("--oracle-sample", type=int, default=0, help=argparse.SUPPRESS)
     ap.add_argument("--profile-steps", type=int, default=0,
                     help="run this many steps untimed and exit (for ncu launch lists)")
-    return ap.parse_args()
+    args = ap.parse_args()
+    if not args.steps:
+        args.steps = DEFAULT_STEPS_W5 if args.workload == 5 else DEFAULT_STEPS
+    return args
 
 
 def peaks():
@@ -84,6 +95,61 @@ def peaks():
             d = json.load(f)
         return float(d["hbm_gbs"]), "measured"
     return 6800.0, "fallback"
+
+
+def read_peak(dev, gib=4, reps=10):
+    """read-only HBM bandwidth of this GPU, measured in this run: the best of `reps` timed
+    passes of a streaming read (synth.dev_read_stream: 16-byte evict-first loads, no stores)
+    over gib GiB, alternating between two such buffers so that no pass starts on rows the
+    previous one left in L2; CUDA events on the launching stream.  Returns GB/s."""
+    import torch
+    n = gib << 30
+    bufs = [torch.zeros(n, dtype=torch.uint8, device=dev) for _ in range(2)]
+    sink = torch.zeros(1, dtype=torch.int32, device=dev)
+    st = torch.cuda.current_stream(dev)
+    ctas = 4 * torch.cuda.get_device_properties(dev).multi_processor_count
+    synth.dev_read_stream(bufs[1], sink, ctas, st.cuda_stream)  # warm-up (loads the kernel)
+    best = float("inf")
+    for r in range(reps):
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(st)
+        synth.dev_read_stream(bufs[r % 2], sink, ctas, st.cuda_stream)
+        b.record(st)
+        b.synchronize()
+        best = min(best, a.elapsed_time(b))
+    del bufs
+    torch.cuda.empty_cache()
+    return n / (best * 1e-3) / 1e9
+
+
+def l2_note(w):
+    """the K/V bytes a step reads against the 129 MB L2, from the workload's shape alone (the
+    same words in both arms): the first step reads every cached row; once the cache is within
+    budget a step reads at least the anchors and the sparse lattice of each sequence
+    (T_keep - B/4 rows, T_keep = B - min(64, B/4)) and at most its budget"""
+    row = 2 * w.L * w.H_kv * w.d * w.esize  # K+V of one cached token over all layers
+    first = row * int(np.sum(w.n0.astype(np.int64) + 1))
+    tk = w.budget - np.minimum(64, w.budget // 4)
+    lo = row * int(np.sum(np.where(w.n0 > w.budget, tk - w.budget // 4, w.n0)))
+    hi = row * int(np.sum(np.minimum(w.n0.astype(np.int64) + 1, w.budget + 1)))
+    if lo > L2_BYTES:
+        return ("inputs larger than L2: the first step reads %.1f GB of K/V, later steps "
+                "%.1f-%.1f GB (cache %.1f GB per GPU)" % (first / 1e9, lo / 1e9, hi / 1e9,
+                                                         w.kv_bytes() / 1e9))
+    return ("no flush between steps: a step within budget reads %.0f-%.0f MB of K/V, near or "
+            "below the 129 MB L2, so bandwidth figures include L2 hits (cache %.0f MB per GPU)"
+            % (lo / 1e6, hi / 1e6, w.kv_bytes() / 1e6))
+
+
+def run_config(w, args, ws):
+    """the config dict of both arms' lines (the workload and what the timed steps are)"""
+    return dict(w.describe(), decode_steps=args.steps, l2=l2_note(w), policy=args.policy,
+                timed_steps="each from a fresh cache" if args.fresh_each_step
+                else "consecutive decode steps from a fresh cache",
+                detector="token ids and p_max (lg_token_detect)"
+                if args.detector == "token" else "attention statistics and V-row sketches",
+                parallelism="dp%d (independent batches, no collective)" % ws,
+                tokens_per_step=w.batch * ws)
 
 
 # ------------------------------------------------------------------ distributed plumbing
@@ -472,16 +538,24 @@ def source_hash():
     return h.hexdigest()
 
 
+def gpu_workload(args, rank=0):
+    """the GPU arm's workload: rank r > 0 draws its own batch (seed 1000 + r); the capacity
+    covers every step of the run under any policy (the full cache never evicts)"""
+    over = {"steps": max(args.steps, args.warmup, args.profile_steps, 1)}
+    if rank:
+        over["seed"] = 1000 + rank
+    if args.batch:
+        over["batch"] = args.batch
+    return synth.make_workload(args.workload, **over)
+
+
 def run_gpu(args, ws, rank, local):
     import torch
     assert torch.cuda.is_available(), "the gb300 arm needs a CUDA device"
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
-    over = {} if rank == 0 else {"seed": 1000 + rank}
-    if args.batch:
-        over["batch"] = args.batch
-    w = synth.make_workload(args.workload, **over)
     K, W = args.steps, args.warmup
+    w = gpu_workload(args, rank)
     if args.profile_steps:
         # untimed steps inside an NVTX range "steps" (ncu --nvtx-include "steps/")
         bench = GpuBench(w, dev, args.profile_steps, args.layers_per_call, args.policy,
@@ -493,6 +567,8 @@ def run_gpu(args, ws, rank, local):
         torch.cuda.synchronize()
         torch.cuda.nvtx.range_pop()
         return None
+    # the read-only bandwidth denominator, measured before the cache takes the memory
+    rpeak = read_peak(dev)
     fresh = args.fresh_each_step
     # every launch of the run goes to one side stream (stream capture needs a non-default one)
     side = torch.cuda.Stream(device=dev)
@@ -592,7 +668,6 @@ def run_gpu(args, ws, rank, local):
     # algorithmic bytes of the same trajectory (deterministic replay, not the timed region)
     lens, kept, prune_ms = bench.replay_log(K, fresh)
     a_bytes, c_bytes, c_ms = [], [], []
-    triggers = 0
     for t in range(K):
         n_rows = lens[t].cpu().numpy() + 1
         a_bytes.append(attend_bytes(w, n_rows, args.policy == "h2o"))
@@ -612,53 +687,54 @@ def run_gpu(args, ws, rank, local):
         e2e, e2e_eager = run_e2e(bench, K, ws, graphs=not args.eager)
 
     value = sum_over_ranks(K, ws) / (ms * 1e-3)
-    # the K/V bytes a step reads against the 129 MB L2 (no flush between steps)
     step_read = sum(a_bytes) / max(1, len(a_bytes))
-    if step_read > L2_BYTES:
-        l2_note = ("inputs larger than L2: each step reads %.2f GB of K/V (cache %.1f GB per GPU)"
-                   % (step_read / 1e9, w.kv_bytes() / 1e9))
-    else:
-        l2_note = ("each step reads %.0f MB of K/V, less than the 129 MB L2 (cache %.1f GB per GPU, "
-                   "no flush between steps): bandwidth figures include L2 hits"
-                   % (step_read / 1e6, w.kv_bytes() / 1e9))
     path_l, harness_l = bench.launches_per_step()
+    # DRAM bytes of one attention launch of the sampled steps, from the committed capture of
+    # this workload on the current kernel code (scaled by the rows a launch reads: the sampled
+    # steps' lengths differ from the captured launch's by a few rows); else null
     prof = traffic_from_profile(source_hash())
-    traffic = None
-    if prof and bench.nl == w.L:
-        # DRAM bytes of one launch: per-row bytes of the captured (smaller) launch scaled by
-        # the K/V rows one launch of this run reads on average
-        rows_per_launch = sum(int(np.sum(l.cpu().numpy() + 1)) for l in lens) / K * w.L * w.H_kv
-        traffic = int(prof["dram_bytes_per_row"] * rows_per_launch)
+    traffic, traffic_note = None, "no DRAM capture of this workload on the current kernel code"
+    sampled_rows = [w.L * w.H_kv * int(np.sum(lens[t].cpu().numpy() + 1)) for t in sampled]
+    if (prof and bench.nl == w.L and prof.get("workload") == args.workload
+            and prof.get("batch") == w.batch and args.policy == "loopguard"):
+        rows = sum(sampled_rows) / len(sampled_rows)
+        traffic = int(prof["dram_bytes"] * rows / prof["rows"])
+        traffic_note = ("ncu dram__bytes_read.sum + dram__bytes_write.sum of the attention launch "
+                        "of %s (profiles/attend_mma_traffic.txt), scaled by %.6f for the rows "
+                        "of the sampled steps" % (prof["launch"], rows / prof["rows"]))
     line = {
         "metric": METRIC, "value": round(value, 3), "unit": UNIT, "n_gpus": ws, "steps": K,
         "warmup": W, "ms_per_step": round(ms / K, 4), "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": w.dtype, "data": "synthetic",
-        "config": dict(w.describe(), decode_steps=K, l2=l2_note, policy=args.policy,
-                       timed_steps="each from a fresh cache" if fresh
-                       else "consecutive decode steps from a fresh cache",
-                       launch="eager" if graph is None else
-                       "one CUDA graph replay of the K steps (captured before timing)",
-                       layers_per_attend_call=bench.nl,
-                       detector="token ids and p_max (lg_token_detect)"
-                       if args.detector == "token" else "attention statistics and V-row sketches",
-                       parallelism="dp%d (independent batches, "
-                       "no collective)" % ws, tokens_per_step=w.batch * ws),
+        "config": run_config(w, args, ws),
+        "launch": {"mode": "eager" if graph is None else
+                   "one CUDA graph replay of the K steps (captured before timing)",
+                   "layers_per_attend_call": bench.nl},
+        "kv_read_GB_per_step": round(step_read / 1e9, 3),
         "roofline": {"bound": "hbm", "achieved": round(attend_gbs, 1), "peak": hbm_peak,
                      "unit": "GB/s", "frac": round(attend_gbs / hbm_peak, 4),
-                     "traffic": traffic,
+                     "traffic": traffic, "traffic_note": traffic_note,
+                     "alg_bytes_per_launch": int(sum(a_bytes[t] for t in sampled) / len(sampled)),
                      "kernel": "lg_decode_attend (tensor-core pass with its split-K merge), all "
                                "%d layers per call" % w.L if bench.nl == w.L
                                else "lg_decode_attend",
-                     "peak_kind": peak_kind + " copy bandwidth"},
+                     "peak_kind": peak_kind + " copy bandwidth (MEASURED_PEAKS.json)",
+                     "read_peak": round(rpeak, 1),
+                     "frac_of_read_peak": round(attend_gbs / rpeak, 4),
+                     "read_peak_kind": "read-only streaming pass over 4 GiB, measured in this "
+                                       "run (best of 10, CUDA events)"},
         "kernels": {
             "attend_stats": {"GB_per_s": round(attend_gbs, 1),
                              "frac_of_%s_peak" % peak_kind: round(attend_gbs / hbm_peak, 4),
                              "frac_of_8TBs_nominal": round(attend_gbs / 8000.0, 4),
+                             "frac_of_read_peak": round(attend_gbs / rpeak, 4),
                              "ms_per_step": round(sum(attend_ms) / len(sampled), 4),
                              "timed_steps": ev_note},
             "prune_compact": {"GB_per_s": round(compact_gbs, 1) if compact_gbs else None,
                               "frac_of_%s_peak" % peak_kind:
                                   round(compact_gbs / hbm_peak, 4) if compact_gbs else None,
+                              "frac_of_8TBs_nominal":
+                                  round(compact_gbs / 8000.0, 4) if compact_gbs else None,
                               "events": len(c_ms),
                               "ms_per_event": round(sum(c_ms) / len(c_ms), 4) if c_ms else None,
                               "moved_bytes_per_event": int(sum(c_bytes) / len(c_bytes))
@@ -781,16 +857,17 @@ def oracle_sample_workload(w, n_seq):
     return sub
 
 
-def time_oracle(w, n_seq, n_layers, steps, warm=0):
+def time_oracle(w, n_seq, n_layers, steps, warm=0, policy="loopguard"):
     """the oracle (as it stands) running `steps` guarded decode steps of the first n_seq
-    sequences restricted to the first n_layers layers; returns (seconds per step, threads)"""
+    sequences restricted to the first n_layers layers, from a fresh cache (after `warm`
+    warm-up steps, themselves from a fresh cache); returns (seconds per step, threads)"""
     import oracle
     sub = oracle_sample_workload(w, n_seq)
     sub.L = n_layers
     K, V = synth.host_cache(sub)
 
     def run(n):
-        g = oracle.OracleGuard(sub, K.copy(), V.copy())
+        g = oracle.OracleGuard(sub, K.copy(), V.copy(), policy=policy)
         seqs = sub.seqs.copy()
         pos = sub.n0.astype(np.int64)
         times = []
@@ -799,75 +876,67 @@ def time_oracle(w, n_seq, n_layers, steps, warm=0):
             t0 = time.perf_counter()
             r = g.step(q, kn, vn, pos)
             times.append(time.perf_counter() - t0)
-            synth.note_interventions(seqs, pos, r["flags"])
+            if policy == "loopguard":
+                synth.note_interventions(seqs, pos, r["flags"])
             pos = pos + 1
-        return times, g.threads
+        return times, getattr(g, "threads", 1)
 
     if warm:
         run(warm)          # warm-up steps; the timed steps start again from the fresh cache
     return run(steps)
 
 
-def cpu_baseline(w, workload, target_s=15.0):
-    """oracle time for one guarded step of a bounded sample: all layers of the first
-    sequences, scaled to batch steps/s"""
-    n_seq = 1
-    times, threads = time_oracle(w, n_seq, w.L, 1)
-    while sum(times) < target_s / 4 and n_seq < w.batch:
-        n_seq *= 2
-        times, threads = time_oracle(w, min(n_seq, w.batch), w.L, 1)
-    n_seq = min(n_seq, w.batch)
-    frac = n_seq / w.batch
+def oracle_sample(w, K, W, policy="loopguard", target_s=ORACLE_TARGET_S):
+    """The oracle on a bounded sample of the GPU arm's timed run: sequence 0 of the batch and its
+    first n_layers layers, W warm-up steps, then the same K consecutive guarded decode steps from
+    a fresh cache (the first carries the budget cut, as on the GPU).  n_layers is sized from a
+    one-layer calibration run so that the K timed steps take about target_s.  Both oracle figures
+    of bench.py (the GPU line's cpu_baseline and the --impl reference line) are this sample.
+    Returns a dict: value (batch steps/s, the sample scaled by sequences and layers), the
+    measured seconds, the scale and a description."""
+    cal = min(K, 3)
+    t_cal, _ = time_oracle(w, 1, 1, cal, policy=policy)
+    per_layer = t_cal[0] + (K - 1) * (float(np.mean(t_cal[1:])) if cal > 1 else t_cal[0])
+    n_layers = int(max(1, min(w.L, target_s // max(per_layer, 1e-6))))
+    times, threads = time_oracle(w, 1, n_layers, K, warm=W, policy=policy)
     sec = sum(times)
-    line = {"value": round(frac / sec, 6), "unit": UNIT, "cores": threads, "kind": "oracle",
-            "affinity_cores": len(os.sched_getaffinity(0)),
-            "sample": "1 guarded decode step (step 1: attention over the prompt's rows plus the "
-                      "new one, %d..%d, detect, budget prune) of %d of the %d sequences, all %d "
-                      "layers; value = %d/%d batch steps / %.2f s"
-                      % (int(w.n0.min()) + 1, int(w.n0.max()) + 1, n_seq, w.batch, w.L, n_seq,
-                         w.batch, sec)}
-    # the same step of one sequence on one thread, in a fresh interpreter (the oracle takes its
-    # thread count when it loads)
-    try:
-        env = dict(os.environ, OMP_NUM_THREADS="1")
-        r = subprocess.run([sys.executable, os.path.abspath(__file__), "--oracle-sample", "1",
-                            "--workload", str(workload)],
-                           env=env, capture_output=True, text=True, timeout=600)
-        one = json.loads(r.stdout.strip().splitlines()[-1])
-        line["single_thread"] = {"value": round(1.0 / w.batch / one["sec"], 6), "unit": UNIT,
-                                 "cores": one["threads"],
-                                 "sample": "the same step of 1 sequence on %d thread (%.2f s), "
-                                           "scaled to batch steps" % (one["threads"], one["sec"])}
-    except Exception as e:  # a reported extra: its failure leaves the main figure
-        line["single_thread"] = {"value": None, "error": str(e)[:200]}
-    return line
+    scale = (1.0 / w.batch) * (n_layers / w.L)   # batch steps per sampled step
+    return {"value": K * scale / sec, "sec": sec, "steps": K, "scale": scale,
+            "threads": threads, "n_layers": n_layers,
+            "sample": "%d guarded decode steps from a fresh cache (after %d warm-up step(s)), the "
+                      "same trajectory as the GPU arm's timed steps, of sequence 0 of %d and its "
+                      "layers 0..%d of %d; value = steps x %.6f batch steps per sampled step / "
+                      "%.2f s" % (K, W, w.batch, n_layers - 1, w.L, scale, sec)}
+
+
+def cpu_baseline(w, args):
+    """the oracle on the host cores: the bounded sample of oracle_sample, as batch steps/s"""
+    o = oracle_sample(w, args.steps, args.warmup, args.policy)
+    return {"value": round(o["value"], 6), "unit": UNIT, "cores": o["threads"],
+            "kind": "oracle", "affinity_cores": len(os.sched_getaffinity(0)),
+            "sample": o["sample"], "sample_scale": o["scale"],
+            "ms_per_sample_step": round(o["sec"] / o["steps"] * 1e3, 3)}
 
 
 def run_reference(args, ws, rank):
-    """--impl reference: the CPU oracle on the host cores, K timed steps after W warm-up steps,
-    each step a bounded sample of the workload (the first sequence, the first layers)"""
+    """--impl reference: the CPU oracle on the host cores, on the same bounded sample of the
+    same timed run as the GPU line's cpu_baseline (oracle_sample): W warm-up steps, then K
+    timed steps from a fresh cache.  ms_per_step is the measured time of one sampled step;
+    value = sample_scale x 1000 / ms_per_step batch steps/s."""
     if rank != 0:
         return
-    w = synth.make_workload(args.workload)
     K, W = args.steps, args.warmup
-    # size the sample so that the whole run stays within about two minutes
-    per_step_budget = 120.0 / max(1, K + W)
-    t1, _ = time_oracle(w, 1, 1, 1)
-    n_layers = int(max(1, min(w.L, per_step_budget / max(t1[0], 1e-6))))
-    times, threads = time_oracle(w, 1, n_layers, K, warm=W)
-    sec = sum(times)
-    frac = (1.0 / w.batch) * (n_layers / w.L)
-    value = K * frac / sec
+    w = synth.make_workload(args.workload, steps=max(K, W, 1))
+    o = oracle_sample(w, K, W, args.policy)
+    value = o["value"]
     line = {"impl": "reference", "metric": METRIC, "value": round(value, 6), "unit": UNIT,
-            "n_gpus": ws, "steps": K, "warmup": W, "ms_per_step": round(1e3 / value, 3),
+            "n_gpus": ws, "steps": K, "warmup": W,
+            "ms_per_step": round(o["sec"] / K * 1e3, 3), "sample_scale": o["scale"],
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
-            "data": "synthetic", "config": dict(w.describe(), decode_steps=args.steps),
-            "cpu_baseline": {"value": round(value, 6), "unit": UNIT, "cores": threads,
-                             "kind": "oracle",
-                             "sample": "each step: the oracle's guarded decode step of sequence "
-                                       "0 of %d, layers 0..%d of %d; value scaled by %.5f "
-                                       "batch steps per sample step" % (
-                                           w.batch, n_layers - 1, w.L, frac)},
+            "data": "synthetic", "config": run_config(w, args, ws),
+            "cpu_baseline": {"value": round(value, 6), "unit": UNIT, "cores": o["threads"],
+                             "kind": "oracle", "affinity_cores": len(os.sched_getaffinity(0)),
+                             "sample": o["sample"], "sample_scale": o["scale"]},
             "e2e": {"value": round(value, 6), "unit": UNIT, "h2d_bytes_per_step": 0,
                     "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
@@ -900,12 +969,6 @@ def run_ablation(args, local):
 
 def main():
     args = parse()
-    if args.oracle_sample:
-        # internal: one guarded step of the first sequences on this process's threads
-        w = synth.make_workload(args.workload)
-        times, threads = time_oracle(w, args.oracle_sample, w.L, 1)
-        print(json.dumps({"sec": sum(times), "threads": threads}), flush=True)
-        return
     ws, rank, local = dist_setup()
     if args.ablation:
         if rank == 0:
@@ -922,7 +985,7 @@ def main():
     line, w = res
     if rank == 0:
         if ws == 1 and not args.no_cpu_baseline:
-            line["cpu_baseline"] = cpu_baseline(w, args.workload)
+            line["cpu_baseline"] = cpu_baseline(w, args)
         print(json.dumps(line), flush=True)
 
 

@@ -3,8 +3,11 @@
 // Sec. 6.1).
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
+#include <limits.h>
 #include <math.h>
 #include <stdint.h>
+
+#include <atomic>
 
 #include "lg_common.cuh"
 #include "lg_internal.h"
@@ -723,9 +726,17 @@ constexpr int kCompactSeqList = 1024;  // pruned sequences listed in shared memo
 // Stream (sequence b, one of 2*L*H_kv K/V streams or the sketch stream): slot j <- row kept[j]
 // for j >= j0, tiles in ascending order; CTAs take (sequence, stream) items of the pruned
 // sequences grid-stride (each CTA first lists them from one pass over kept_count, so a step
-// that prunes nothing costs that pass).  kept[] is strictly increasing with kept[j] >= j,
-// so a tile reads only rows at or above its own first slot: once every load of the tile is
-// performed (the barrier) its stores cannot clobber a row another tile still needs.
+// that prunes nothing costs that pass).  kept[] is strictly increasing with kept[j] >= j, so
+// no tile reads a slot an earlier tile wrote; the only hazard is a store to slot s racing a
+// load of row s = kept[j] (j <= s) that another thread has not performed yet.  A barrier
+// orders every load issued before it ahead of every store after it, so a tile needs one only
+// when a load issued since the last barrier may read a slot the tile writes: the loads since
+// then read rows >= kept[first index loaded since then] (kept is increasing), and the tile
+// writes [t0, t1).  Dense stretches (a short removed span) pay a barrier per tile; the sparse
+// lattice of a budget cut and the rows above a long removed span go barrier-free for many
+// tiles at a time (a barrier only where t1 catches up with the pending rows).  A per-tile
+// test alone (kept[t0] >= t1) would not do: without a barrier a fast warp may already store
+// the next tile's slots while a slow warp still loads this tile's rows there.
 __global__ void __launch_bounds__(kCompactThreads) compact_kernel(lg_cache c,
                                                                   const int32_t *kept_idx,
                                                                   const int32_t *kept_count,
@@ -807,10 +818,17 @@ __global__ void __launch_bounds__(kCompactThreads) compact_kernel(lg_cache c,
       }
     };
     if (j0 < cnt) load_tile(cur, j0);
+    // lowest row read by the loads issued since the last barrier (none yet: those of tile j0)
+    int pend_row = j0 < cnt ? kept[j0] : INT_MAX;
     for (int t0 = j0; t0 < cnt; t0 += rows_per_tile) {
       const int t1 = t0 + rows_per_tile;
       if (t1 < cnt) load_tile(nxt, t1);
-      __syncthreads();
+      // kept[] is read-only here, so every thread takes the same branch
+      if (pend_row < min(t1, cnt)) {
+        __syncthreads();
+        const int jn = t1 + rows_per_tile;  // the first tile loaded after this barrier
+        pend_row = jn < cnt ? kept[jn] : INT_MAX;
+      }
 #pragma unroll
       for (int k = 0; k < kCompactChunks; ++k) {
         const int ci = k * kCompactThreads + tid;
@@ -1127,11 +1145,24 @@ cudaError_t launch_prune_compact(const lg_cache &c, const int32_t *flags, const 
 
 cudaError_t launch_compact(const lg_cache &c, const int32_t *kept_idx, const int32_t *kept_count,
                            int max_keep, cudaStream_t s) {
-  int dev = 0, sms = 152;
-  if (cudaGetDevice(&dev) == cudaSuccess)
+  // one wave of resident CTAs (items are handed out grid-stride, so a second wave would start
+  // its items late); the residency per SM is looked up once per device
+  constexpr int kMaxDev = 64;
+  static std::atomic<int> resident[kMaxDev];  // CTAs per GPU, 0 = not looked up yet
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0) dev = 0;
+  int ctas = dev < kMaxDev ? resident[dev].load(std::memory_order_relaxed) : 0;
+  if (ctas <= 0) {
+    int sms = 152, per_sm = 1;
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, compact_kernel, kCompactThreads,
+                                                      0) != cudaSuccess || per_sm < 1)
+      per_sm = 1;
+    ctas = sms * per_sm;
+    if (dev < kMaxDev) resident[dev].store(ctas, std::memory_order_relaxed);
+  }
   const int items = c.batch * (2 * c.L * c.H_kv + 1);
-  const int grid = items < 4 * sms ? items : 4 * sms;
+  const int grid = items < ctas ? items : ctas;
   LG_TRY(launch_pdl(compact_kernel, grid, kCompactThreads, 0, s, c, kept_idx, kept_count,
                     max_keep));
   return cudaGetLastError();

@@ -374,8 +374,10 @@ def dev_lib():
         lib.syn_dev_select.argtypes = [vp, i32, vp, i32, i64, vp, vp, vp, vp]
         lib.syn_dev_select3.argtypes = [vp, i32, vp, i32, vp, vp, vp, vp, vp]
         lib.syn_dev_select_tokens.argtypes = [vp, i32, vp, vp, vp, vp, vp, vp, vp, vp]
+        lib.syn_dev_read_stream.argtypes = [vp, i64, vp, i32, vp]
         for f in (lib.syn_dev_fill_cache, lib.syn_dev_step, lib.syn_dev_advance,
-                  lib.syn_dev_select, lib.syn_dev_select3, lib.syn_dev_select_tokens):
+                  lib.syn_dev_select, lib.syn_dev_select3, lib.syn_dev_select_tokens,
+                  lib.syn_dev_read_stream):
             f.restype = ctypes.c_int
         _dev = lib
     return _dev
@@ -427,6 +429,13 @@ def dev_select_tokens(w: Workload, seqs_dev, pos_dev, tok_loop, tok_fresh, pm_lo
                                            pm_loop.data_ptr(), pm_fresh.data_ptr(),
                                            tok.data_ptr(), pm.data_ptr(), stream),
            "syn_dev_select_tokens")
+
+
+def dev_read_stream(buf, sink, ctas: int, stream):
+    """one read-only pass over the bytes of device tensor buf (harness: the read-only bandwidth
+    denominator of bench.py); sink is a one-word int32 device tensor"""
+    _check(dev_lib().syn_dev_read_stream(buf.data_ptr(), buf.numel() * buf.element_size(),
+                                         sink.data_ptr(), ctas, stream), "syn_dev_read_stream")
 
 
 TOKEN_VOCAB = 50_000

@@ -149,6 +149,31 @@ __global__ void select_tokens_kernel(const syn_seq *seqs, int batch, const int64
   pm[b] = fresh ? pm_fresh[b] : pm_loop[b];
 }
 
+
+// Read-only streaming pass (harness, not part of the generator's recipe): every 16-byte word of
+// the buffer is loaded once with an evict-first hint and folded by XOR into one word per warp,
+// so the loads cannot be dropped.  bench.py times it as the read-only bandwidth denominator
+// beside the copy peak (a decode pass reads its K/V and writes next to nothing).  Grid-stride,
+// eight independent 16-byte loads in flight per thread.
+__global__ void __launch_bounds__(256) read_stream_kernel(const uint4 *p, int64_t n16,
+                                                          unsigned *sink) {
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  unsigned acc = 0;
+  for (; i + 7 * stride < n16; i += 8 * stride) {
+    uint4 v[8];
+#pragma unroll
+    for (int k = 0; k < 8; ++k) v[k] = __ldcs(p + i + k * stride);
+#pragma unroll
+    for (int k = 0; k < 8; ++k) acc ^= v[k].x ^ v[k].y ^ v[k].z ^ v[k].w;
+  }
+  for (; i < n16; i += stride) {
+    const uint4 v = __ldcs(p + i);
+    acc ^= v.x ^ v.y ^ v.z ^ v.w;
+  }
+  acc = __reduce_xor_sync(0xffffffffu, acc);
+  if ((threadIdx.x & 31) == 0) atomicXor(sink, acc);
+}
 }  // namespace
 
 extern "C" {
@@ -224,6 +249,15 @@ int syn_dev_select_tokens(const syn_seq *seqs_dev, int batch, const int64_t *pos
                     pm) == cudaSuccess
              ? 0
              : 2;
+}
+
+// one read-only pass over bytes (a multiple of 16, 16-byte aligned) of device memory; ctas = the
+// grid (a multiple of the SM count); sink: one device word, XOR of everything read
+int syn_dev_read_stream(const void *p, int64_t bytes, unsigned *sink, int ctas,
+                        cudaStream_t stream) {
+  if (!p || !sink || bytes % 16 || ((uintptr_t)p & 15) || ctas < 1) return 1;
+  read_stream_kernel<<<ctas, 256, 0, stream>>>((const uint4 *)p, bytes / 16, sink);
+  return cudaGetLastError() == cudaSuccess ? 0 : 2;
 }
 
 }  // extern "C"
