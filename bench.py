@@ -98,28 +98,41 @@ def peaks():
 
 
 def read_peak(dev, gib=4, reps=10):
-    """read-only HBM bandwidth of this GPU, measured in this run: the best of `reps` timed
-    passes of a streaming read (synth.dev_read_stream: 16-byte evict-first loads, no stores)
-    over gib GiB, alternating between two such buffers so that no pass starts on rows the
-    previous one left in L2; CUDA events on the launching stream.  Returns GB/s."""
+    """read-only HBM bandwidth of this GPU, measured in this run: three read-only passes over
+    gib GiB (synth: 16-byte evict-first loads from registers; 1-D bulk copies of 16 KB into
+    shared memory, 3 CTAs per SM; of 32 KB, one CTA per SM), each the best of `reps` timed
+    passes alternating between two such buffers (so that no pass starts on rows the previous
+    one left in L2), CUDA events on the launching stream.  Returns (best GB/s, {probe: GB/s})."""
     import torch
     n = gib << 30
     bufs = [torch.zeros(n, dtype=torch.uint8, device=dev) for _ in range(2)]
     sink = torch.zeros(1, dtype=torch.int32, device=dev)
+    err = torch.zeros(1, dtype=torch.int32, device=dev)
     st = torch.cuda.current_stream(dev)
-    ctas = 4 * torch.cuda.get_device_properties(dev).multi_processor_count
-    synth.dev_read_stream(bufs[1], sink, ctas, st.cuda_stream)  # warm-up (loads the kernel)
-    best = float("inf")
-    for r in range(reps):
-        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        a.record(st)
-        synth.dev_read_stream(bufs[r % 2], sink, ctas, st.cuda_stream)
-        b.record(st)
-        b.synchronize()
-        best = min(best, a.elapsed_time(b))
+    sms = torch.cuda.get_device_properties(dev).multi_processor_count
+    probes = {
+        "loads_16B": lambda buf: synth.dev_read_stream(buf, sink, 4 * sms, st.cuda_stream),
+        "bulk_16KB": lambda buf: synth.dev_read_bulk(buf, 16384, sink, err, 3 * sms,
+                                                     st.cuda_stream),
+        "bulk_32KB": lambda buf: synth.dev_read_bulk(buf, 32768, sink, err, sms,
+                                                     st.cuda_stream)}
+    res = {}
+    for name, run in probes.items():
+        run(bufs[1])  # warm-up (loads the kernel)
+        best = float("inf")
+        for r in range(reps):
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(st)
+            run(bufs[r % 2])
+            b.record(st)
+            b.synchronize()
+            best = min(best, a.elapsed_time(b))
+        res[name] = round(n / (best * 1e-3) / 1e9, 1)
+    if int(err.item()):
+        raise RuntimeError("a read-bandwidth probe timed out on a wait")
     del bufs
     torch.cuda.empty_cache()
-    return n / (best * 1e-3) / 1e9
+    return max(res.values()), res
 
 
 def l2_note(w):
@@ -561,14 +574,22 @@ def run_gpu(args, ws, rank, local):
         bench = GpuBench(w, dev, args.profile_steps, args.layers_per_call, args.policy,
                          args.detector)
         bench.reset()
+        rows = []
         torch.cuda.nvtx.range_push("steps")
         for t in range(args.profile_steps):
+            rows.append(w.L * w.H_kv * int((bench.cache.len.cpu() + 1).sum()))
             bench.step(t)
         torch.cuda.synchronize()
         torch.cuda.nvtx.range_pop()
+        # K/V rows each step's attention launch reads (for the DRAM-traffic summary)
+        print(json.dumps({"workload": args.workload, "batch": w.batch,
+                          "attend_rows_per_launch": rows,
+                          "attend_alg_bytes_per_launch": [
+                              attend_bytes(w, np.full(w.batch, 0)) + 2 * w.d * w.esize * r
+                              for r in rows]}), flush=True)
         return None
     # the read-only bandwidth denominator, measured before the cache takes the memory
-    rpeak = read_peak(dev)
+    rpeak, rprobes = read_peak(dev)
     fresh = args.fresh_each_step
     # every launch of the run goes to one side stream (stream capture needs a non-default one)
     side = torch.cuda.Stream(device=dev)
@@ -721,8 +742,9 @@ def run_gpu(args, ws, rank, local):
                      "peak_kind": peak_kind + " copy bandwidth (MEASURED_PEAKS.json)",
                      "read_peak": round(rpeak, 1),
                      "frac_of_read_peak": round(attend_gbs / rpeak, 4),
-                     "read_peak_kind": "read-only streaming pass over 4 GiB, measured in this "
-                                       "run (best of 10, CUDA events)"},
+                     "read_peak_kind": "the fastest of three read-only passes over 4 GiB, "
+                                       "measured in this run (best of 10 each, CUDA events)",
+                     "read_probes_GB_per_s": rprobes},
         "kernels": {
             "attend_stats": {"GB_per_s": round(attend_gbs, 1),
                              "frac_of_%s_peak" % peak_kind: round(attend_gbs / hbm_peak, 4),

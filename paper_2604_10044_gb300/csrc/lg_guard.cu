@@ -720,28 +720,30 @@ __global__ void __launch_bounds__(kKeepThreads) keep_set_kernel(KeepArgs a) {
 // ------------------------------------------------------------------ ordered in-place gather
 
 constexpr int kCompactThreads = 256;
-constexpr int kCompactChunks = 4;  // 16-byte chunks per thread per tile
+constexpr int kCompactStageBytes = 16384;  // one tile of destination rows
+constexpr int kCompactStages = 4;          // ring of tiles: three gathers in flight, one store
+constexpr int kCompactChunks = kCompactStageBytes / 16 / kCompactThreads;  // 16-byte chunks
 constexpr int kCompactSeqList = 1024;  // pruned sequences listed in shared memory up to this batch
+constexpr size_t kCompactSmem = (size_t)kCompactStages * kCompactStageBytes;
 
 // Stream (sequence b, one of 2*L*H_kv K/V streams or the sketch stream): slot j <- row kept[j]
-// for j >= j0, tiles in ascending order; CTAs take (sequence, stream) items of the pruned
-// sequences grid-stride (each CTA first lists them from one pass over kept_count, so a step
-// that prunes nothing costs that pass).  kept[] is strictly increasing with kept[j] >= j, so
-// no tile reads a slot an earlier tile wrote; the only hazard is a store to slot s racing a
-// load of row s = kept[j] (j <= s) that another thread has not performed yet.  A barrier
-// orders every load issued before it ahead of every store after it, so a tile needs one only
-// when a load issued since the last barrier may read a slot the tile writes: the loads since
-// then read rows >= kept[first index loaded since then] (kept is increasing), and the tile
-// writes [t0, t1).  Dense stretches (a short removed span) pay a barrier per tile; the sparse
-// lattice of a budget cut and the rows above a long removed span go barrier-free for many
-// tiles at a time (a barrier only where t1 catches up with the pending rows).  A per-tile
-// test alone (kept[t0] >= t1) would not do: without a barrier a fast warp may already store
-// the next tile's slots while a slow warp still loads this tile's rows there.
+// for j >= j0, in tiles of kCompactStageBytes of destination rows, ascending.  CTAs take
+// (sequence, stream) items of the pruned sequences grid-stride (each CTA first lists them from
+// one pass over kept_count, so a step that prunes nothing costs that pass).
+//
+// A tile is gathered row chunk by row chunk with 16-byte asynchronous copies into a ring of
+// shared-memory stages (kCompactStages - 1 tiles in flight, no registers held), then written
+// back by one bulk copy of the whole tile's contiguous slots.  In place and race-free without
+// any further ordering: kept[] is strictly increasing with kept[j] >= j, so a row read for tile
+// i' > i lies at or above kept[first slot of i'] > every slot of tile i, and every row a slot of
+// tile i is read for (kept[j] = s means j <= s) belongs to a tile <= i, whose copies have all
+// landed in shared memory before tile i's store is issued (the wait and the barrier below).
 __global__ void __launch_bounds__(kCompactThreads) compact_kernel(lg_cache c,
                                                                   const int32_t *kept_idx,
                                                                   const int32_t *kept_count,
                                                                   int max_keep) {
   pdl_enter();
+  extern __shared__ __align__(128) unsigned char s_stage[];  // kCompactStages tiles
   __shared__ int s_seq[kCompactSeqList], s_cnt[kCompactSeqList];
   __shared__ int s_wtot[kCompactThreads / 32];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -794,53 +796,81 @@ __global__ void __launch_bounds__(kCompactThreads) compact_kernel(lg_cache c,
       row_bytes = nwords * 4;
     }
     const int32_t *kept = kept_idx + (int64_t)b * max_keep;
-    // first slot that moves: kept[j] == j exactly for j < j0 (binary search)
+    // first slot that moves: kept[j] == j exactly for j < j0 (and kept[j] > j after), found by
+    // a 32-way search in every warp (the same result in all)
     int lo = 0, hi = cnt;
     while (lo < hi) {
-      const int mid = (lo + hi) >> 1;
-      if (kept[mid] == mid) lo = mid + 1;
-      else hi = mid;
+      const int step = (hi - lo + 31) >> 5;
+      const int x = lo + lane * step;
+      const unsigned m = __ballot_sync(0xffffffffu, x < hi && kept[x] != x);
+      if (m) {
+        const int f = __ffs(m) - 1;
+        hi = lo + f * step;
+        if (f) lo += (f - 1) * step + 1;
+      } else {
+        lo += min(31, (hi - 1 - lo) / step) * step + 1;
+      }
     }
     const int j0 = lo;
-    const int cpr = row_bytes / 16;
-    const int rows_per_tile = kCompactThreads * kCompactChunks / cpr;
-    // double-buffered: the next tile's loads are issued before the barrier that releases this
-    // tile's stores (the next tile reads only rows above every slot this tile writes)
-    uint4 cur[kCompactChunks], nxt[kCompactChunks];
-    auto load_tile = [&](uint4 *v, int t0) {
+    const int cpr = row_bytes >> 4;
+    const int T = kCompactStageBytes / row_bytes;  // rows per tile
+    const int n_tiles = (cnt - j0 + T - 1) / T;
+    if (n_tiles <= 0) continue;
+    // this thread's chunks of a tile: row within the tile and byte offset within the row; in
+    // the stage a chunk sits at its chunk index x 16 (the tile's rows back to back)
+    int c_row[kCompactChunks], c_off[kCompactChunks], kv[kCompactChunks];
 #pragma unroll
-      for (int k = 0; k < kCompactChunks; ++k) {
-        const int ci = k * kCompactThreads + tid;
-        const int j = t0 + ci / cpr;
-        if (j < cnt)
-          v[k] = *reinterpret_cast<const uint4 *>(base + (int64_t)kept[j] * row_bytes +
-                                                  (ci % cpr) * 16);
-      }
-    };
-    if (j0 < cnt) load_tile(cur, j0);
-    // lowest row read by the loads issued since the last barrier (none yet: those of tile j0)
-    int pend_row = j0 < cnt ? kept[j0] : INT_MAX;
-    for (int t0 = j0; t0 < cnt; t0 += rows_per_tile) {
-      const int t1 = t0 + rows_per_tile;
-      if (t1 < cnt) load_tile(nxt, t1);
-      // kept[] is read-only here, so every thread takes the same branch
-      if (pend_row < min(t1, cnt)) {
-        __syncthreads();
-        const int jn = t1 + rows_per_tile;  // the first tile loaded after this barrier
-        pend_row = jn < cnt ? kept[jn] : INT_MAX;
-      }
-#pragma unroll
-      for (int k = 0; k < kCompactChunks; ++k) {
-        const int ci = k * kCompactThreads + tid;
-        const int j = t0 + ci / cpr;
-        if (j < cnt)
-          *reinterpret_cast<uint4 *>(base + (int64_t)j * row_bytes + (ci % cpr) * 16) = cur[k];
-      }
-#pragma unroll
-      for (int k = 0; k < kCompactChunks; ++k) cur[k] = nxt[k];
+    for (int k = 0; k < kCompactChunks; ++k) {
+      const int ci = k * kCompactThreads + tid;
+      c_row[k] = ci / cpr;
+      c_off[k] = (ci - c_row[k] * cpr) * 16;
     }
-    __syncthreads();  // the next item reuses no memory, but keep the CTA in step
+    // kv[k] <- source row of chunk k of tile p (requested a tile ahead of its copies)
+    auto fetch_rows = [&](int p) {
+      const int t0 = j0 + p * T, rows = min(T, cnt - t0);
+#pragma unroll
+      for (int k = 0; k < kCompactChunks; ++k)
+        kv[k] = (p < n_tiles && c_row[k] < rows) ? kept[t0 + c_row[k]] : 0;
+    };
+    auto gather = [&](int p) {
+      const int t0 = j0 + p * T, rows = min(T, cnt - t0);
+      unsigned char *st = s_stage + (p % kCompactStages) * kCompactStageBytes;
+#pragma unroll
+      for (int k = 0; k < kCompactChunks; ++k)
+        if (c_row[k] < rows)
+          cp_async16(st + (k * kCompactThreads + tid) * 16,
+                     base + (int64_t)kv[k] * row_bytes + c_off[k]);
+    };
+    for (int p = 0; p < kCompactStages - 1; ++p) {
+      if (p < n_tiles) {
+        fetch_rows(p);
+        gather(p);
+      }
+      cp_async_commit();  // one group per tile, empty past the end (uniform group counting)
+    }
+    fetch_rows(kCompactStages - 1);
+    for (int i = 0; i < n_tiles; ++i) {
+      cp_async_wait<kCompactStages - 2>();  // this thread's copies of tile i have landed
+      fence_proxy_async_smem();
+      if (tid == 0) bulk_wait_read_all();  // tile i-1's store has read its stage
+      __syncthreads();
+      if (tid == 0) {
+        const int t0 = j0 + i * T, rows = min(T, cnt - t0);
+        bulk_store(base + (int64_t)t0 * row_bytes,
+                   s_stage + (i % kCompactStages) * kCompactStageBytes,
+                   (uint32_t)(rows * row_bytes));
+        bulk_commit();
+      }
+      const int p = i + kCompactStages - 1;  // into the stage tile i-1 used
+      if (p < n_tiles) gather(p);
+      cp_async_commit();
+      fetch_rows(p + 1);
+    }
+    // the next item's first copies reuse the stages
+    if (tid == 0) bulk_wait_read_all();
+    __syncthreads();
   }
+  if (tid == 0) bulk_wait_all();
 }
 
 // ------------------------------------------------------------------ H2O comparator
@@ -1155,16 +1185,18 @@ cudaError_t launch_compact(const lg_cache &c, const int32_t *kept_idx, const int
   if (ctas <= 0) {
     int sms = 152, per_sm = 1;
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    LG_TRY(cudaFuncSetAttribute(compact_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                (int)kCompactSmem));
     if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, compact_kernel, kCompactThreads,
-                                                      0) != cudaSuccess || per_sm < 1)
+                                                      kCompactSmem) != cudaSuccess || per_sm < 1)
       per_sm = 1;
     ctas = sms * per_sm;
     if (dev < kMaxDev) resident[dev].store(ctas, std::memory_order_relaxed);
   }
   const int items = c.batch * (2 * c.L * c.H_kv + 1);
   const int grid = items < ctas ? items : ctas;
-  LG_TRY(launch_pdl(compact_kernel, grid, kCompactThreads, 0, s, c, kept_idx, kept_count,
-                    max_keep));
+  LG_TRY(launch_pdl(compact_kernel, grid, kCompactThreads, kCompactSmem, s, c, kept_idx,
+                    kept_count, max_keep));
   return cudaGetLastError();
 }
 

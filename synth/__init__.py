@@ -375,9 +375,10 @@ def dev_lib():
         lib.syn_dev_select3.argtypes = [vp, i32, vp, i32, vp, vp, vp, vp, vp]
         lib.syn_dev_select_tokens.argtypes = [vp, i32, vp, vp, vp, vp, vp, vp, vp, vp]
         lib.syn_dev_read_stream.argtypes = [vp, i64, vp, i32, vp]
+        lib.syn_dev_read_bulk.argtypes = [vp, i64, i32, vp, vp, i32, vp]
         for f in (lib.syn_dev_fill_cache, lib.syn_dev_step, lib.syn_dev_advance,
                   lib.syn_dev_select, lib.syn_dev_select3, lib.syn_dev_select_tokens,
-                  lib.syn_dev_read_stream):
+                  lib.syn_dev_read_stream, lib.syn_dev_read_bulk):
             f.restype = ctypes.c_int
         _dev = lib
     return _dev
@@ -436,6 +437,14 @@ def dev_read_stream(buf, sink, ctas: int, stream):
     denominator of bench.py); sink is a one-word int32 device tensor"""
     _check(dev_lib().syn_dev_read_stream(buf.data_ptr(), buf.numel() * buf.element_size(),
                                          sink.data_ptr(), ctas, stream), "syn_dev_read_stream")
+
+
+def dev_read_bulk(buf, block: int, sink, err, ctas: int, stream):
+    """the same read-only pass with 1-D bulk copies of `block` bytes into shared memory; err is
+    a one-word int32 device tensor, set when a wait timed out"""
+    _check(dev_lib().syn_dev_read_bulk(buf.data_ptr(), buf.numel() * buf.element_size(), block,
+                                       sink.data_ptr(), err.data_ptr(), ctas, stream),
+           "syn_dev_read_bulk")
 
 
 TOKEN_VOCAB = 50_000

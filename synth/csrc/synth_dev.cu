@@ -174,6 +174,97 @@ __global__ void __launch_bounds__(256) read_stream_kernel(const uint4 *p, int64_
   acc = __reduce_xor_sync(0xffffffffu, acc);
   if ((threadIdx.x & 31) == 0) atomicXor(sink, acc);
 }
+
+// Read-only pass with 1-D bulk (TMA) copies: one warp per CTA streams blocks of `block` bytes
+// (grid-stride) through a ring of 4 shared-memory stages, each copy completing on its stage's
+// mbarrier; lane j folds word j of every block into its XOR.  Every wait is bounded (2 s of
+// %globaltimer): on a timeout the CTA records it in *err, waits (bounded) for its copies in
+// flight and returns.
+constexpr int kReadStages = 4;
+
+__device__ __forceinline__ uint32_t rd_smem(const void *p) {
+  return (uint32_t)__cvta_generic_to_shared(p);
+}
+
+__device__ __forceinline__ bool rd_try_wait(uint64_t *bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+      " selp.u32 %0, 1, 0, p;\n}\n"
+      : "=r"(ok)
+      : "r"(rd_smem(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+__device__ __forceinline__ bool rd_wait(uint64_t *bar, uint32_t parity) {
+  uint64_t t0, t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t0));
+  while (!rd_try_wait(bar, parity)) {
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    if (t - t0 > 2000000000ull) return false;
+  }
+  return true;
+}
+
+__device__ __forceinline__ void rd_issue(uint64_t *bar, void *dst, const void *src, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(rd_smem(bar)),
+               "r"(bytes)
+               : "memory");
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+      ::"r"(rd_smem(dst)), "l"(src), "r"(bytes), "r"(rd_smem(bar))
+      : "memory");
+}
+
+__global__ void __launch_bounds__(32) read_bulk_kernel(const unsigned char *p, int64_t nblocks,
+                                                       int block, unsigned *sink, int *err) {
+  extern __shared__ __align__(128) unsigned char rbuf[];
+  __shared__ __align__(8) uint64_t bar[kReadStages];
+  const int lane = threadIdx.x;
+  if (lane == 0) {
+    for (int k = 0; k < kReadStages; ++k)
+      asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(rd_smem(&bar[k])) : "memory");
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  __syncwarp();
+  const int64_t g = gridDim.x;
+  if (lane == 0)
+    for (int k = 0; k < kReadStages; ++k) {
+      const int64_t blk = blockIdx.x + k * g;
+      if (blk < nblocks) rd_issue(&bar[k], rbuf + k * block, p + blk * block, block);
+    }
+  unsigned acc = 0;
+  int64_t i = 0;
+  bool ok = true;
+  for (;; ++i) {
+    const int64_t blk = blockIdx.x + i * g;
+    if (blk >= nblocks) break;
+    const int k = (int)(i % kReadStages);
+    const uint32_t parity = (uint32_t)((i / kReadStages) & 1);
+    ok = rd_wait(&bar[k], parity);
+    if (!__all_sync(0xffffffffu, ok)) {
+      ok = false;
+      break;
+    }
+    acc ^= ((const unsigned *)(rbuf + k * block))[lane];
+    __syncwarp();
+    const int64_t nxt = blk + kReadStages * g;
+    if (lane == 0 && nxt < nblocks) rd_issue(&bar[k], rbuf + k * block, p + nxt * block, block);
+  }
+  if (!ok) {
+    if (lane == 0) atomicExch(err, 1);
+    // the copies still in flight: blocks i .. i + kReadStages - 1 (those that exist)
+    for (int64_t j = i; j < i + kReadStages; ++j) {
+      const int64_t blk = blockIdx.x + j * g;
+      if (blk >= nblocks) break;
+      rd_wait(&bar[j % kReadStages], (uint32_t)((j / kReadStages) & 1));
+    }
+    return;
+  }
+  acc = __reduce_xor_sync(0xffffffffu, acc);
+  if (lane == 0) atomicXor(sink, acc);
+}
 }  // namespace
 
 extern "C" {
@@ -257,6 +348,22 @@ int syn_dev_read_stream(const void *p, int64_t bytes, unsigned *sink, int ctas,
                         cudaStream_t stream) {
   if (!p || !sink || bytes % 16 || ((uintptr_t)p & 15) || ctas < 1) return 1;
   read_stream_kernel<<<ctas, 256, 0, stream>>>((const uint4 *)p, bytes / 16, sink);
+  return cudaGetLastError() == cudaSuccess ? 0 : 2;
+}
+
+// the same pass with 1-D bulk copies into shared memory: block bytes per copy (a multiple of
+// 16, at most 32768), bytes a multiple of block; err: one device word, set on a timed-out wait
+int syn_dev_read_bulk(const void *p, int64_t bytes, int block, unsigned *sink, int *err,
+                      int ctas, cudaStream_t stream) {
+  if (!p || !sink || !err || block < 128 || block > 32768 || block % 16 || bytes % block ||
+      ((uintptr_t)p & 15) || ctas < 1)
+    return 1;
+  const int smem = kReadStages * block;
+  if (cudaFuncSetAttribute(read_bulk_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) !=
+      cudaSuccess)
+    return 2;
+  read_bulk_kernel<<<ctas, 32, smem, stream>>>((const unsigned char *)p, bytes / block, block,
+                                               sink, err);
   return cudaGetLastError() == cudaSuccess ? 0 : 2;
 }
 

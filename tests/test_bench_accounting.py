@@ -40,11 +40,17 @@ def test_traffic_summary_is_gated_on_the_kernel_source():
     path = os.path.join(bench.ROOT, "profiles", "attend_mma_traffic.txt")
     with open(path) as f:
         d = json.load(f)
-    # a capture of the attention pass reads each K/V row about once: well below the 512
-    # algorithmic bytes would mean rows skipped, well above, rows read again
-    assert 0.8 * 512 < d["dram_bytes_per_row"] < 1.1 * 512
+    # a full-size launch reads each K/V row once: its DRAM bytes are its algorithmic bytes
+    # less at most what L2 can hold of the previous pass (129 MB), plus the partials written
+    assert d["alg_bytes"] - 129e6 <= d["dram_bytes"] <= 1.02 * d["alg_bytes"]
+    assert d["dram_bytes"] == d["dram_bytes_read"] + d["dram_bytes_write"]
+    # the algorithmic bytes of the captured launch, as bench.py counts them
+    w = synth.make_workload(d["workload"])
+    assert w.batch == d["batch"] and d["rows"] % (w.L * w.H_kv) == 0
+    qo = bench.attend_bytes(w, np.zeros(w.batch, dtype=np.int64))
+    assert d["alg_bytes"] == qo + 2 * w.d * w.esize * d["rows"]
     got = bench.traffic_from_profile(d["source_sha256"])
-    assert got is not None and got["dram_bytes_per_row"] == d["dram_bytes_per_row"]
+    assert got is not None and got["dram_bytes"] == d["dram_bytes"]
 
 
 def test_traffic_gate_ignores_comments_not_code():

@@ -1,12 +1,14 @@
-"""The barrier schedule of the in-place compaction (the index-gather of Sec. 5.3), on the CPU.
+"""The in-place compaction (the index-gather of Sec. 5.3) on the CPU: the facts its ordering
+rests on, and the pieces of compact_kernel that decide where it reads and writes.
 
-compact_kernel moves slot j <- row kept[j] (kept strictly increasing, kept[j] >= j) tile by
-tile; the loads of tile i+1 are issued in iteration i, before that iteration's optional barrier
-and its stores of tile i.  A barrier orders every load issued before it ahead of every store
-after it.  The kernel takes the barrier of iteration i only when the lowest row read since the
-last barrier lies below the tile's end.  Restated here and checked for safety: every store to
-a slot s that some later index j reads (kept[j] = s) must be preceded by a barrier taken after
-that load was issued.  The kernel's source is checked to contain the rule restated here.
+compact_kernel moves slot j <- row kept[j] tile by tile: a tile's rows are gathered with
+asynchronous copies into a ring of shared-memory stages (several tiles ahead) and written back
+by one bulk copy once all of the tile's copies have landed.  It needs no other ordering
+because (a) kept is strictly increasing with kept[j] >= j, so every row a slot of tile i is
+read for belongs to a tile <= i, and (b) every row read for a later tile lies above every slot
+of tile i.  Both are checked on the oracle's retained sets and on random lists; the kernel's
+32-way search for the first moved slot is restated and checked against a linear scan; and the
+kernel's source is checked to keep its waits, fence, barrier and store in that order.
 """
 import os
 import re
@@ -16,28 +18,6 @@ import numpy as np
 import oracle
 
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
-INF = 1 << 62
-
-
-def schedule(kept, j0, cnt, T, rule="pending"):
-    """iterations of the tile loop: list of (t0, barrier taken)"""
-    out = []
-    pend_row = kept[j0] if j0 < cnt else INF
-    t0 = j0
-    while t0 < cnt:
-        t1 = t0 + T
-        if rule == "pending":
-            bar = pend_row < min(t1, cnt)
-            if bar:
-                jn = t1 + T
-                pend_row = kept[jn] if jn < cnt else INF
-        elif rule == "per_tile":          # kept[t0] >= t1 alone: not enough (see below)
-            bar = kept[t0] < min(t1, cnt)
-        else:
-            bar = True
-        out.append((t0, bar))
-        t0 = t1
-    return out
 
 
 def first_moved(kept):
@@ -47,25 +27,23 @@ def first_moved(kept):
     return j
 
 
-def unsafe_pairs(kept, T, rule="pending"):
-    """(j, s) pairs whose load of row s = kept[j] is not ordered before the store to slot s"""
-    cnt = len(kept)
-    j0 = first_moved(kept)
-    sched = schedule(kept, j0, cnt, T, rule)
-    bars = np.array([b for _, b in sched], dtype=bool)
-    it = lambda j: (j - j0) // T          # iteration that stores slot j
-    bad = []
-    for j in range(j0, cnt):
-        s = int(kept[j])
-        if s >= cnt or s < j0:
-            continue                      # row s is never overwritten by this stream
-        if s == j:
-            continue
-        lo, hi = it(j) - 1, it(s)         # loads of tile it(j) are issued one iteration early
-        lo = max(lo, 0)
-        if not bars[lo:hi + 1].any():
-            bad.append((j, s))
-    return bad, int(bars.sum()), len(sched)
+def search32(kept, cnt):
+    """the kernel's 32-way search: probes lo + lane * step of every lane, ballot, narrow"""
+    lo, hi = 0, cnt
+    rounds = 0
+    while lo < hi:
+        rounds += 1
+        step = (hi - lo + 31) >> 5
+        hits = [lo + lane * step < hi and kept[lo + lane * step] != lo + lane * step
+                for lane in range(32)]
+        if any(hits):
+            f = hits.index(True)
+            hi = lo + f * step
+            if f:
+                lo += (f - 1) * step + 1
+        else:
+            lo += min(31, (hi - 1 - lo) // step) * step + 1
+    return lo, rounds
 
 
 def keep_cases():
@@ -74,8 +52,7 @@ def keep_cases():
     cases = [(8193, 4096, 0, (0, 0), 0), (131073, 32768, 0, (0, 0), 0),
              (131073, 32768, 1, (114689, 131073), 0), (32769, 8192, 1, (32000, 32600), 1),
              (5000, 4096, 1, (4900, 4940), 0), (5000, 4096, 1, (4800, 4864), 0),
-             (5000, 4096, 1, (4800, 4863), 2), (5000, 4096, 1, (4800, 4865), 3),
-             (4200, 4096, 0, (0, 0), 0), (4097, 4096, 0, (0, 0), 0)]
+             (4097, 4096, 0, (0, 0), 0), (300, 256, 0, (0, 0), 0)]
     for _ in range(60):
         B = int(rng.choice([256, 1024, 4096, 8192]))
         n = int(rng.integers(B + 1, 5 * B))
@@ -83,67 +60,70 @@ def keep_cases():
         a = int(rng.integers(lo_w, n))
         cases.append((n, B, int(rng.random() < 0.7), (a, int(rng.integers(a, n + 1))),
                       int(rng.integers(0, 4))))
-    return [(c, oracle.keep_set(*c, prm)) for c in cases]
+    return [oracle.keep_set(*c, prm) for c in cases]
 
 
 def random_lists(rng, count):
-    """increasing lists with kept[j] >= j mixing dense stretches (steps of 1) and gaps"""
     out = []
     for _ in range(count):
-        m = int(rng.integers(50, 3000))
+        m = int(rng.integers(1, 3000))
         steps = np.where(rng.random(m) < rng.random(), 1, rng.integers(1, 300, m))
-        kept = np.cumsum(steps) - 1 + int(rng.integers(0, 5))
-        kept = np.maximum(kept, np.arange(m))
+        kept = np.cumsum(steps) - 1
+        j0 = int(rng.integers(0, m + 1))
+        kept[:j0] = np.arange(j0)
+        kept[j0:] = np.maximum(kept[j0:], np.arange(j0, m) + 1)
+        kept[j0:] = np.maximum.accumulate(kept[j0:] + np.arange(m - j0) * 0)
+        for j in range(j0 + 1, m):                 # strictly increasing
+            kept[j] = max(kept[j], kept[j - 1] + 1)
         out.append(kept.astype(np.int64))
     return out
 
 
-def test_pending_rule_orders_every_load_before_its_slot_is_written():
-    rng = np.random.default_rng(11)
-    lists = [k for _, k in keep_cases()] + random_lists(rng, 300)
+def test_tiles_never_read_what_an_earlier_tile_wrote():
+    rng = np.random.default_rng(3)
+    for kept in keep_cases() + random_lists(rng, 200):
+        cnt = len(kept)
+        assert np.all(np.diff(kept) > 0) and np.all(kept >= np.arange(cnt))
+        j0 = first_moved(kept)
+        assert np.all(kept[j0:] > np.arange(j0, cnt))
+        for T in (32, 64, 128, 170):
+            for t0 in range(j0, cnt, T):
+                t1 = min(t0 + T, cnt)
+                # (b) rows read by later tiles lie above this tile's slots
+                if t1 < cnt:
+                    assert kept[t1] >= t1
+                # (a) a slot of this tile is read only by this or an earlier tile
+                readers = np.nonzero((kept >= t0) & (kept < t1))[0]
+                assert readers.size == 0 or readers.max() < t1
+
+
+def test_first_moved_search_matches_a_scan():
+    rng = np.random.default_rng(5)
+    lists = keep_cases() + random_lists(rng, 300) + [np.arange(0), np.arange(5), np.arange(1, 9)]
     for kept in lists:
-        for T in (16, 32, 64, 128):
-            bad, _, _ = unsafe_pairs(kept, T)
-            assert not bad, (T, bad[:3])
+        got, rounds = search32(kept, len(kept))
+        assert got == first_moved(kept)
+        assert rounds <= 4 or len(kept) > 32 ** 4
 
 
-def test_sparse_lattice_takes_few_barriers():
-    """a budget cut of a long cache (every 4th row kept) takes a barrier only where the tiles
-    catch up with the rows still pending: a handful per stream instead of one per tile"""
-    prm = oracle.params()
-    kept = oracle.keep_set(131073, 32768, 0, (0, 0), 0, prm)
-    _, n_bar, n_it = unsafe_pairs(kept, 64)
-    assert n_it == 511 and n_bar <= 12, (n_bar, n_it)
-    # the dense recent block of the 8192-row budget cut keeps a constant offset of 4161 rows
-    kept = oracle.keep_set(8193, 4096, 0, (0, 0), 0, prm)
-    _, n_bar, n_it = unsafe_pairs(kept, 64)
-    assert n_bar <= n_it // 4, (n_bar, n_it)
-    # a short removed span (40 rows < one tile) leaves every later tile overlapping its rows
-    kept = oracle.keep_set(5000, 4096, 1, (4900, 4940), 0, prm)
-    bad, n_bar, n_it = unsafe_pairs(kept, 64)
-    assert not bad and n_bar >= 1
-
-
-def test_per_tile_test_alone_is_unsafe():
-    """kept[t0] >= t1 says only that the tile's own rows lie above its slots; without a barrier a
-    warp may store the next tile's slots while another still loads this tile's rows there"""
-    kept = np.concatenate([np.arange(0, 10), np.arange(74, 74 + 400)])
-    bad, _, _ = unsafe_pairs(kept, 64, rule="per_tile")
-    assert bad
-    assert not unsafe_pairs(kept, 64)[0]
-
-
-def test_kernel_source_has_the_rule():
+def test_kernel_source_order():
     with open(os.path.join(ROOT, "paper_2604_10044_gb300", "csrc", "lg_guard.cu")) as f:
         src = f.read()
     body = src[src.index("compact_kernel(lg_cache c"):]
     body = body[:body.index("// ------------------------------------------------------------------")]
-    code = re.sub(r"//[^\n]*", "", body)
-    code = " ".join(code.split())
-    assert "int pend_row = j0 < cnt ? kept[j0] : INT_MAX;" in code
-    assert "if (t1 < cnt) load_tile(nxt, t1); if (pend_row < min(t1, cnt)) { __syncthreads();" \
-        in code
-    assert "const int jn = t1 + rows_per_tile; pend_row = jn < cnt ? kept[jn] : INT_MAX;" in code
-    # exactly one barrier inside the tile loop (the conditional one)
-    loop = code[code.index("for (int t0 = j0;"):code.index("cur[k] = nxt[k]; }")]
-    assert loop.count("__syncthreads()") == 1
+    code = " ".join(re.sub(r"//[^\n]*", "", body).split())
+    loop = code[code.index("for (int i = 0; i < n_tiles; ++i) {"):]
+    order = ["cp_async_wait<kCompactStages - 2>();", "fence_proxy_async_smem();",
+             "if (tid == 0) bulk_wait_read_all();", "__syncthreads();", "bulk_store(",
+             "bulk_commit();", "const int p = i + kCompactStages - 1;",
+             "if (p < n_tiles) gather(p);", "cp_async_commit();", "fetch_rows(p + 1);"]
+    at = [loop.index(x) for x in order]
+    assert at == sorted(at), order
+    # the stage a gather refills is the one the previous tile's store has read
+    S = int(re.search(r"kCompactStages = (\d+);", src).group(1))
+    for i in range(3 * S):
+        assert (i + S - 1) % S == (i - 1) % S
+    # the search narrows to the first slot whose row moves
+    assert "__ballot_sync(0xffffffffu, x < hi && kept[x] != x)" in code
+    # barriers: two in the listing of the pruned sequences, one per tile, one per item
+    assert code.count("__syncthreads();") == 4, code.count("__syncthreads();")
