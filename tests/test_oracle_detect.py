@@ -328,3 +328,22 @@ def test_tail_repetition_at_the_shortest_cache_that_can_show_it():
     _, _, diag = oracle.detect(_stats_for(0.9, 1.0, 1, 2, 16, 16), sk, 4096, prm,
                                oracle.new_state())
     assert int(diag["P"]) == 4
+
+
+@pytest.mark.parametrize("theta_nov", [0.02, 0.1, 0.25, 0.2501, 0.3])
+def test_stall_gate_takes_the_novel_fraction_of_the_last_rows(theta_nov):
+    """Stall: the novel fraction of the last stall_len = 4 rows is below theta_nov.  The
+    fraction takes only the values k/4, so every theta_nov in (0, 1/4] gives the same gate
+    (none of the last 4 rows novel) and the paper's 0.02 acts as any of them; above 1/4 one
+    novel row of four no longer blocks it"""
+    rng = np.random.default_rng(17)
+    n = 60
+    prm = oracle.params(theta_nov=theta_nov, t_min=0)
+    stats = _stats_for(0.4, 3.0, 1, 2, n, 64)
+    for k_novel in (0, 1, 2):
+        sk = _sketches(rng, n, 8)                  # random rows: every row novel
+        for j, i in enumerate(range(n - 4, n)):
+            if j >= k_novel:
+                sk[i] = sk[10 + j]                 # a copy of an earlier window row
+        _, _, diag = oracle.detect(stats, sk, 1024, prm, oracle.new_state())
+        assert bool(diag["stall"]) == (k_novel / 4 < theta_nov), (k_novel, theta_nov)
