@@ -3,7 +3,7 @@
 //
 // Persistent CTAs (one per SM) start on chunks blockIdx.x and blockIdx.x + gridDim.x and take
 // further chunks from a shared counter, each a run of consecutive rows of one (layer,
-// sequence, kv-head), sized in the kernel from the lengths of the call (4 to 16 chunks per
+// sequence, kv-head), sized in the kernel from the lengths of the call (3 to 16 chunks per
 // CTA).  A producer warp streams 128-row K and V tiles into a 3-stage shared-memory ring with
 // 2-D tensor copies (cp.async.bulk.tensor, 128-byte swizzle, one box per 64 columns)
 // completing on mbarriers.  Each of four consumer warps owns 32 rows of a tile and all g query
@@ -79,12 +79,14 @@ __device__ __forceinline__ int arrive_acq_rel(int *p) {
   return old;
 }
 
-__device__ __forceinline__ void tma_load_2d(void *smem_dst, const CUtensorMap *map, int x, int y,
-                                            uint64_t *bar) {
+// 2-D tensor copy of one box into shared memory, completing on `bar`, with an L2 eviction
+// policy (createpolicy) for the lines it brings in.
+__device__ __forceinline__ void tma_load_2d(void *smem_dst, const CUtensorMap *map, int x,
+                                                 int y, uint64_t *bar, uint64_t policy) {
   asm volatile(
-      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes "
-      "[%0], [%1, {%2, %3}], [%4];" ::"r"(smem_addr(smem_dst)),
-      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(smem_addr(bar))
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+      ".L2::cache_hint [%0], [%1, {%2, %3}], [%4], %5;" ::"r"(smem_addr(smem_dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(smem_addr(bar)), "l"(policy)
       : "memory");
 }
 
@@ -134,8 +136,9 @@ struct ChunkId {
 // Chunk geometry of one call, from the lengths it attends over (the host sizes the workspace
 // for max_len, which can be far above them): chunk rows a multiple of the tile, never more
 // chunks per group than the workspace holds (max_chunks).  A CTA takes about one chunk per
-// eight of its tiles, at least 4 (a chunk end costs the consumers a hand-off, and a short pass
-// with fewer, longer chunks measured faster) and at most 16 (measured: finer chunks gained
+// eight of its tiles, at least 3 (a chunk end costs the consumers a hand-off, and a short pass
+// with fewer, longer chunks measured faster: at the paper-shaped step 2 chunks of 512 rows per
+// group balance 152 CTAs better than 3 of 384) and at most 16 (measured: finer chunks gained
 // nothing at the end of long passes and cost a little on the way); the rows are then evened
 // out over the chunks of the longest group.
 struct Geom {
@@ -152,7 +155,7 @@ __device__ __forceinline__ Geom make_geom(const AttendArgs &a, int n_max, int64_
   // every CTA) keeps 64-bit divisions off the prologue
   const float rows_all = (float)len_sum * (float)(a.H_kv * a.n_layers);
   const float per_cta =
-      fminf(fmaxf(floorf(rows_all / (float)(kTile * 8) / (float)ctas), 4.f), 16.f);
+      fminf(fmaxf(floorf(rows_all / (float)(kTile * 8) / (float)ctas), 3.f), 16.f);
   const float cf = ceilf(rows_all / ((float)ctas * per_cta));
   int c = cf >= (float)kMaxChunkRows ? kMaxChunkRows : (int)cf;
   const unsigned nm = (unsigned)n_max;
@@ -484,6 +487,14 @@ attend_mma_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant
     // tile index, length and logits row to the consumers, and a chunk's first stage also
     // brings the chunk's query rows (one bulk copy on the same barrier).
     if (lane == 0) {
+      // K/V tiles are streamed once per call: their L2 lines go first when space is needed, so
+      // that a pass of the whole cache does not evict what the rest of the step works on (the
+      // other kernels' code and data, the workspace); at one sequence (115 MB of K/V a step,
+      // less than the 129 MB L2) this took the paper-shaped step from about 40 to 36.5 us, the
+      // loop-onset test's share most of all, and left the pass itself and its L2 reuse across
+      // calls unchanged
+      uint64_t evict_first;
+      asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(evict_first));
       uint32_t it = 0;
       const int claimed0 = 2 * (int)gridDim.x;
       const bool rev = s_rev != 0;
@@ -543,9 +554,10 @@ attend_mma_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant
           mbar_arrive_expect_tx(&full_bar[st], C::kStageBytes + (t == 0 ? G * D * 2 : 0));
 #pragma unroll
           for (int h = 0; h < C::kHalves; ++h) {
-            tma_load_2d(stage + h * kBoxBytes, &tmK, h * 64, grow + t * kTile, &full_bar[st]);
-            tma_load_2d(stage + (C::kHalves + h) * kBoxBytes, &tmV, h * 64, grow + t * kTile,
-                        &full_bar[st]);
+            tma_load_2d(stage + h * kBoxBytes, &tmK, h * 64, grow + t * kTile,
+                             &full_bar[st], evict_first);
+            tma_load_2d(stage + (C::kHalves + h) * kBoxBytes, &tmV, h * 64,
+                             grow + t * kTile, &full_bar[st], evict_first);
           }
           if (t == 0)
             bulk_load(qbuf + st * C::kQBytes,

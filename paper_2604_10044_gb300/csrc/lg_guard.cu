@@ -58,13 +58,29 @@ __global__ void append_kernel(lg_cache c, int layer0, int n_layers, const uint4 
     const int b = blockIdx.x - row_blocks;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int nwords = c.H_kv * c.d / 32;
+    const T *row = (const T *)v_new + ((int64_t)lguard * c.batch + b) * c.H_kv * c.d;
+    // the sign bits this warp packs are requested with the length and the status (one round
+    // trip for all), up to 8 words a warp at once
+    constexpr int kWordsPerWarp = 8;
+    const int wstep = blockDim.x >> 5;
+    uint32_t sg[kWordsPerWarp];
+#pragma unroll
+    for (int k = 0; k < kWordsPerWarp; ++k) {
+      const int w = warp + k * wstep;
+      sg[k] = w < nwords ? Elem<T>::sign(row, w * 32 + lane) : 0u;
+    }
     const int slot = c.len[b] - 1;
     const int64_t off = c.seq_off[b];
     // one status read per warp, so that every lane of the ballot takes the same branch
     const int bad = __shfl_sync(0xffffffffu, lane == 0 ? (int)status_bad(c.dev_status) : 0, 0);
     if (bad || slot < 0) return;
-    const T *row = (const T *)v_new + ((int64_t)lguard * c.batch + b) * c.H_kv * c.d;
-    for (int w = warp; w < nwords; w += blockDim.x >> 5) {
+#pragma unroll
+    for (int k = 0; k < kWordsPerWarp; ++k) {
+      const int w = warp + k * wstep;
+      const uint32_t word = __ballot_sync(0xffffffffu, sg[k] != 0u);
+      if (lane == 0 && w < nwords) c.sketch[(off + slot) * nwords + w] = word;
+    }
+    for (int w = warp + kWordsPerWarp * wstep; w < nwords; w += wstep) {
       const uint32_t word = __ballot_sync(0xffffffffu, Elem<T>::sign(row, w * 32 + lane) != 0u);
       if (lane == 0) c.sketch[(off + slot) * nwords + w] = word;
     }
@@ -99,7 +115,10 @@ __global__ void append_kernel(lg_cache c, int layer0, int n_layers, const uint4 
 // sketches of rows [0, len[b]) of the guard layer, read from the cache
 template <typename T>
 __global__ void sketch_build_kernel(lg_cache c, int guard_layer, int max_len) {
-  pdl_enter();
+  // no early start of the kernel after this one: the detect kernel reads sketch rows before its
+  // dependency wait and checks only the length, its synced length and the newest row, which this
+  // kernel leaves unchanged while it may rewrite every other row
+  asm volatile("griddepcontrol.wait;" ::: "memory");
   const int b = blockIdx.y;
   if (status_bad(c.dev_status)) return;
   const int n = c.len[b];
@@ -262,14 +281,15 @@ __device__ __forceinline__ bool rows_match(const uint32_t *x, const uint32_t *y,
 }
 
 // Full Hamming distance of two sketch rows of nwords words (nwords a multiple of 4, rows
-// 16-byte aligned); the loads are independent, so a thread has all of them in flight at once.
+// 16-byte aligned); the loads are independent, so a thread has all of them in flight at once,
+// and go to L2 only (the detect kernel also calls this before its dependency wait, see below).
 __device__ __forceinline__ int hamming(const uint32_t *x, const uint32_t *y, int nwords) {
   const uint4 *a = reinterpret_cast<const uint4 *>(x);
   const uint4 *b = reinterpret_cast<const uint4 *>(y);
   int dist = 0;
 #pragma unroll 8
   for (int w = 0; w < nwords / 4; ++w) {
-    const uint4 u = __ldg(a + w), v = __ldg(b + w);
+    const uint4 u = __ldcg(a + w), v = __ldcg(b + w);
     dist += __popc(u.x ^ v.x) + __popc(u.y ^ v.y) + __popc(u.z ^ v.z) + __popc(u.w ^ v.w);
   }
   return dist;
@@ -282,6 +302,7 @@ constexpr float kFixScale = 1099511627776.0f;  // 2^40: statistics summed in 2^-
 constexpr int kCmpWarp0 = kStatWarps + 1;  // the new-row comparisons: warps after ln n's
 constexpr int kCmpThreads = kDetectThreads - kCmpWarp0 * 32;
 constexpr int kCmpBatch = 6;  // comparison chunks a thread has in flight at once
+constexpr int kPreRowChunks = 64;  // sketch rows up to 1 KB (H_kv d <= 8192) take the early phase
 static_assert(kCmpThreads % 32 == 0, "comparing threads in whole warps");
 
 // One CTA per sequence, monitor state carried from call to call in dstate:
@@ -291,20 +312,23 @@ static_assert(kCmpThreads % 32 == 0, "comparing threads in whole warps");
 //   run[P]    trailing rows (up to the test length) that match the row P earlier.
 //   synced    the length seen by the previous call.
 // When the length grew by exactly one row since the previous call, only the new row i = n-1 is
-// examined: the warps after the statistics warps compare it with every row the window and the
-// periods need (the window comparisons double as the period comparisons), a row's 16-byte
-// chunks on consecutive lanes, the distances in shared memory; beside them three warps sum the
-// statistics in 64-bit fixed point.  Then thread t takes window row i-1-t (and i-1-t-T, ...)
-// for the latest match and period P = t+1's run, and the CTA meets at a barrier after every
-// warp has reduced its share (latest match, novel rows, shortest verified period); thread 0 then
-// takes the votes against bounds that the ln n warp formed beside the sums (a division only next
-// to a threshold) and updates the guard state.  Otherwise (first
-// call, after a prune or any other change of the cache) the window and the runs are recomputed:
-// the sketches of the last smem_rows rows are staged in shared memory with a row stride of
-// nwords + 1 words (rows that different lanes read fall in different banks), one warp scans
+// examined, and before the kernel waits for the one before it (the attention pass, whose
+// statistics it needs): the warps after the statistics warps compare the new row with every row
+// the window and the periods need (the window comparisons double as the period comparisons), a
+// row's 16-byte chunks on consecutive lanes, the distances in shared memory; then thread t takes
+// window row i-1-t (and i-1-t-T, ...) for the latest match and period P = t+1's run, and every
+// warp reduces its share (latest match, novel rows, shortest verified period), kept in shared
+// memory; the ln n warp forms the votes' bounds.  After the wait three warps sum the statistics
+// in 64-bit fixed point while the fourth checks that the early phase's inputs did not change;
+// the early results are committed (or dropped for a recompute), and thread 0 takes the votes
+// against the bounds (a division only next to a threshold) and updates the guard state.  At one
+// sequence the CTA starts on an SM freed by the attention pass's first finishing CTAs, so the
+// comparisons run beside the pass's last chunks and merges.  Otherwise (first call, after a
+// prune or any other change of the cache) the window and the runs are recomputed after the
+// wait: the sketches of the last smem_rows rows are staged in shared memory with a row stride
+// of nwords + 1 words (rows that different lanes read fall in different banks), one warp scans
 // each window row, one warp each period.
 __global__ void __launch_bounds__(kDetectThreads, 1) detect_kernel(DetectArgs a) {
-  pdl_enter();
   extern __shared__ __align__(16) uint32_t sk_s[];
   __shared__ long long red_e[kStatWarps], red_l[kStatWarps];  // fixed point, 2^-40 units
   __shared__ int red_ok[kStatWarps];                          // every statistic finite
@@ -314,43 +338,176 @@ __global__ void __launch_bounds__(kDetectThreads, 1) detect_kernel(DetectArgs a)
   __shared__ FixBound s_bound_ent, s_bound_lift;  // sum-vote bounds, 2^-40 units, see (1)
   __shared__ int2 s_bound_ttr, s_bound_stall;       // count-vote bounds
   __shared__ int s_novel, s_novel_tail, s_pstar, s_mismatch, s_trig, s_span_lo, s_span_hi,
-      s_level;
+      s_level, s_bad, s_valid, s_latest, s_n0, s_synced0, s_n;
+  __shared__ uint4 s_newrow[kPreRowChunks];  // the new sketch row as the early phase read it
   const int b = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int32_t *status = a.c.dev_status;
-  const int n = a.c.len[b];
-  const int B = a.budget[b];
-  const int64_t off = a.c.seq_off[b];
+  const int64_t off = a.c.seq_off[b];  // set by the caller, never written by a kernel
   const lg_guard_params &p = a.p;
   const int np = p.p_max - p.p_min + 1;
   int32_t *ds = a.dstate + (int64_t)b * (np + 2);
-  const int synced = ds[0];
-  // the sequence's guard state, {t_gen, cd, level, last_trig} and {n_int, pad}, read by the
-  // thread that updates it
-  int4 st_a = make_int4(0, 0, 0, 0), st_b = make_int4(0, 0, 0, 0);
+  const int nw = a.nwords, thr = a.thr, stride = nw + 1;
+  const int cpr = nw / 4;  // 16-byte chunks per sketch row
+  const uint32_t *sk_g = a.c.sketch + off * nw;
+  int32_t *run = ds + 2;
+  int32_t *lm = a.dstate + (int64_t)a.c.batch * (np + 2) + off;
+  const int nh = a.c.L * a.H_q;
+  int *dist = reinterpret_cast<int *>(sk_s);
+  int *run_new = dist + max(p.W, p.p_max);  // the early phase's period runs, committed later
+
+  // ln n and the bounds of the votes (see count_vote and fix_side) for length m: novel rows
+  // against theta_ttr w, the stall test's tail against theta_nov stall_len, the entropy sum
+  // against theta_ent L H_q ln n, the suffix-mass sum against theta_lift W_s L H_q / n
+  auto form_bounds = [&](int m) {
+    const double logn = m >= 2 ? log((double)m) : 1.0;
+    const int m1 = max(m, 1);
+    s_logn = logn;
+    s_bound_ttr = count_bounds(p.theta_ttr * (double)min(p.W, m));
+    s_bound_stall = count_bounds(p.theta_nov * (double)p.stall_len);
+    s_bound_ent = fix_bound(p.theta_ent * (double)nh * logn);
+    s_bound_lift = fix_bound(p.theta_lift * (double)min(p.suffix_w, m1) * (double)nh / (double)m1);
+  };
+
+  // (0) Before the dependency wait: the comparisons of the new row, which need only the
+  // sketches and the monitor state, overlap the end of the kernel before (the attention pass,
+  // whose statistics this kernel waits for).  Every read here goes to L2 only (ld.global.cg:
+  // nothing is left in L1 for the reads after the wait), stays within the sequence's slots,
+  // and writes nothing but shared memory; after the wait the length, the monitor's synced
+  // length and the new row are read again, and unless all three are unchanged (the kernel
+  // before did not write them) the results are dropped for a recompute.  The one kernel that
+  // rewrites window rows without changing any of the three, lg_sketch_build's, lets its
+  // successor start only once it has completed.
+  // (one read by thread 0, handed on through shared memory: a kernel still writing them could
+  // otherwise split the CTA between the two paths)
   if (tid == 0) {
+    s_n0 = __ldcg(a.c.len + b);
+    s_synced0 = __ldcg(ds);
+  }
+  __syncthreads();
+  const int n0 = s_n0, synced0 = s_synced0;
+  const bool pre = n0 >= 1 && synced0 + 1 == n0 && cpr <= kPreRowChunks;
+  if (warp == kStatWarps) {
+    if (lane == 0) form_bounds(n0);
+    if (pre) {
+      const uint4 *ri4 = reinterpret_cast<const uint4 *>(sk_g + (int64_t)(n0 - 1) * nw);
+      for (int q = lane; q < cpr; q += 32) s_newrow[q] = __ldcg(ri4 + q);
+    }
+  }
+  if (pre) {
+    // (2) the new row i against the rows the window and the periods need, [jlo, i), on the
+    // warps after the statistics and ln n: chunk q of row j is read by consecutive lanes (rows
+    // are contiguous: a warp reads 512 contiguous bytes), all of a thread's loads in flight at
+    // once, the chunk popcounts summed per row into dist[] in shared memory (the staging area
+    // of the recompute path, unused here); then the latest match, the novel rows and the
+    // period runs, reduced per warp and kept in shared memory until they are committed
+    const int n = n0, i = n0 - 1;
+    const int w = min(p.W, n), wlo = n - w;
+    const uint32_t *ri = sk_g + (int64_t)i * nw;
+    const int jlo = max(0, min(wlo, i - p.p_max));
+    const int m_cnt = i - jlo;
+    const int r0 = wlo + tid;
+    const int lm0 = r0 < i ? __ldcg(lm + r0) : 0;
+    const int run0 = tid < np ? __ldcg(run + tid) : 0;
+    const int ct = tid - kCmpWarp0 * 32;  // index among the comparing threads, < 0 elsewhere
+    if (ct >= 0) {
+      if ((cpr & (cpr - 1)) == 0 && cpr <= 32) {
+        // a power-of-two number of chunks: each row's chunks sit in aligned lanes of one warp
+        const uint4 *rows4 = reinterpret_cast<const uint4 *>(sk_g + (int64_t)jlo * nw);
+        const uint4 *ri4 = reinterpret_cast<const uint4 *>(ri);
+        const int total = m_cnt * cpr;
+        // a thread's chunk index is ct mod cpr in every row (the stride is a multiple of 32)
+        const uint4 v = __ldcg(ri4 + (ct & (cpr - 1)));
+        for (int base = 0; base < total; base += kCmpThreads * kCmpBatch) {
+          uint4 u[kCmpBatch];
+#pragma unroll
+          for (int k = 0; k < kCmpBatch; ++k) {
+            const int f = base + ct + k * kCmpThreads;
+            u[k] = f < total ? __ldcg(rows4 + f) : make_uint4(0u, 0u, 0u, 0u);
+          }
+#pragma unroll
+          for (int k = 0; k < kCmpBatch; ++k) {
+            const int f = base + ct + k * kCmpThreads;
+            int pc = __popc(u[k].x ^ v.x) + __popc(u[k].y ^ v.y) + __popc(u[k].z ^ v.z) +
+                     __popc(u[k].w ^ v.w);
+            for (int o = cpr >> 1; o >= 1; o >>= 1) pc += __shfl_xor_sync(0xffffffffu, pc, o);
+            if (f < total && (lane & (cpr - 1)) == 0) dist[f / cpr] = pc;
+          }
+        }
+      } else {
+        for (int r = ct; r < m_cnt; r += kCmpThreads)
+          dist[r] = hamming(ri, sk_g + (int64_t)(jlo + r) * nw, nw);
+      }
+    }
+    __syncthreads();
+    int latest = -1;
+    for (int j = i - 1 - tid; j >= wlo; j -= kDetectThreads)
+      if (dist[j - jlo] <= thr) {
+        latest = j;
+        break;
+      }
+    // novel rows of the window other than the new one
+    int nov = 0, nov_tail = 0;
+    for (int r = r0; r < i; r += kDetectThreads) {
+      const int novel = (r == r0 ? lm0 : __ldcg(lm + r)) < wlo;
+      nov += novel;
+      if (r >= n - p.stall_len) nov_tail += novel;
+    }
+    // period runs; P ascends with the thread index, so the first qualifying P of a warp is
+    // its lowest lane's and a thread's first qualifying P is its smallest
+    int pstar = 0x7fffffff;
+    for (int pi = tid; pi < np; pi += kDetectThreads) {
+      const int P = p.p_min + pi;
+      const int cap = max(p.m_rep * P, p.l_min);
+      const int j = i - P;
+      const bool m = j >= 0 && dist[j - jlo] <= thr;
+      const int r = m ? min((pi == tid ? run0 : __ldcg(run + pi)) + 1, cap) : 0;
+      run_new[pi] = r;
+      if (pstar == 0x7fffffff && n >= cap + P && r >= cap) pstar = P;
+    }
+    latest = __reduce_max_sync(0xffffffffu, latest);
+    nov = __reduce_add_sync(0xffffffffu, nov);
+    nov_tail = __reduce_add_sync(0xffffffffu, nov_tail);
+    pstar = (int)__reduce_min_sync(0xffffffffu, (unsigned)pstar);
+    if (lane == 0) {
+      w_latest[warp] = latest;
+      w_nov[warp] = nov;
+      w_nov_tail[warp] = nov_tail;
+      w_pstar[warp] = pstar;
+    }
+    __syncthreads();
+    if (tid == 0) {
+      int lt = -1, nv = 0, nt = 0, ps = 0x7fffffff;
+      for (int k = 0; k < kDetectWarps; ++k) {
+        lt = max(lt, w_latest[k]);
+        nv += w_nov[k];
+        nt += w_nov_tail[k];
+        ps = min(ps, w_pstar[k]);
+      }
+      s_latest = lt;
+      const int novel = lt < wlo;
+      s_novel = nv + novel;
+      s_novel_tail = nt + (p.stall_len >= 1 ? novel : 0);
+      s_pstar = ps;
+    }
+  }
+  pdl_enter();  // the statistics of the kernel before, and every write before it, from here on
+
+  // the sequence's guard state, {t_gen, cd, level, last_trig} and {n_int, pad}, read by the
+  // thread that updates it; the device status, decided for the whole CTA at the next barrier
+  int4 st_a = make_int4(0, 0, 0, 0), st_b = make_int4(0, 0, 0, 0);
+  int bad0 = 0;
+  if (tid == 0) {
+    bad0 = status_bad(status);
     st_a = reinterpret_cast<const int4 *>(a.state + b)[0];
     st_b = reinterpret_cast<const int4 *>(a.state + b)[1];
   }
-  if (cta_status_bad(status)) return;
-  const int nw = a.nwords, thr = a.thr, stride = nw + 1;
-  const uint32_t *sk_g = a.c.sketch + off * nw;
-  const int w = min(p.W, n);
-  const int wlo = n - w;
-  int32_t *run = ds + 2;
-  int32_t *lm = a.dstate + (int64_t)a.c.batch * (np + 2) + off;
-  const bool incr = n >= 1 && synced + 1 == n;
-  const int nh = a.c.L * a.H_q;
-  // the monitor state the incremental step reads after its comparisons (a window row's latest
-  // match, a period's run), requested now, before the statistics warps start their sums
-  const int r0 = wlo + tid;
-  const int lm0 = incr && r0 < n - 1 ? lm[r0] : 0;
-  const int run0 = incr && tid < np ? run[tid] : 0;
+  const int B = a.budget[b];
 
   // (1) sums of the entropies and suffix masses over every layer and head, one warp per SM
-  // sub-partition, and ln n on the fourth.  The sums are exact in 64-bit fixed point (units of
-  // 2^-40: a value loses at most 2^-40 when it is scaled and truncated, and values up to 2^23
-  // fit), on the integer pipes rather than GB300's slow fp64 pipe; a non-finite statistic
-  // makes its sum NaN.
+  // sub-partition.  The sums are exact in 64-bit fixed point (units of 2^-40: a value loses at
+  // most 2^-40 when it is scaled and truncated, and values up to 2^23 fit), on the integer
+  // pipes rather than GB300's slow fp64 pipe; a non-finite statistic makes its sum NaN.  The
+  // fourth warp reads the length, the synced length and the new row again.
   if (warp < kStatWarps) {
     // kStatBatch loads in flight per thread before the first add (one round trip per batch)
     long long se = 0, sl = 0;
@@ -382,116 +539,38 @@ __global__ void __launch_bounds__(kDetectThreads, 1) detect_kernel(DetectArgs a)
       red_l[warp] = sl;
       red_ok[warp] = finite;
     }
-  } else if (warp == kStatWarps && lane == 0) {
-    // ln n and the bounds of the votes (see count_vote and fix_side): novel rows against
-    // theta_ttr w, the stall test's tail against theta_nov stall_len, the entropy sum against
-    // theta_ent L H_q ln n, the suffix-mass sum against theta_lift W_s L H_q / n
-    const double logn = n >= 2 ? log((double)n) : 1.0;
-    const int n1 = max(n, 1);
-    s_logn = logn;
-    s_bound_ttr = count_bounds(p.theta_ttr * (double)w);
-    s_bound_stall = count_bounds(p.theta_nov * (double)p.stall_len);
-    s_bound_ent = fix_bound(p.theta_ent * (double)nh * logn);
-    s_bound_lift = fix_bound(p.theta_lift * (double)min(p.suffix_w, n1) * (double)nh / (double)n1);
-  }
-
-  if (incr) {
-    // (2) the new row against the rows the window and the periods need, [jlo, i), on the
-    // warps after the statistics and ln n (so the two run side by side): chunk q of row j is
-    // read by consecutive lanes (rows are contiguous: a warp reads 512 contiguous bytes), all of
-    // a thread's loads in flight at once, the chunk popcounts summed per row into dist[] in
-    // shared memory (the staging area of the recompute path, unused here); then the latest
-    // match, the novel rows and the period runs, reduced per warp
-    const int i = n - 1;
-    const uint32_t *ri = sk_g + (int64_t)i * nw;
-    const int jlo = max(0, min(wlo, i - p.p_max));
-    const int m_cnt = i - jlo;
-    const int cpr = nw / 4;  // 16-byte chunks per sketch row
-    int *dist = reinterpret_cast<int *>(sk_s);
-    const int ct = tid - kCmpWarp0 * 32;  // index among the comparing threads, < 0 elsewhere
-    if (ct >= 0) {
-      if ((cpr & (cpr - 1)) == 0 && cpr <= 32) {
-        // a power-of-two number of chunks: each row's chunks sit in aligned lanes of one warp
-        const uint4 *rows4 = reinterpret_cast<const uint4 *>(sk_g + (int64_t)jlo * nw);
-        const uint4 *ri4 = reinterpret_cast<const uint4 *>(ri);
-        const int total = m_cnt * cpr;
-        // a thread's chunk index is ct mod cpr in every row (the stride is a multiple of 32)
-        const uint4 v = __ldg(ri4 + (ct & (cpr - 1)));
-        for (int base = 0; base < total; base += kCmpThreads * kCmpBatch) {
-          uint4 u[kCmpBatch];
-#pragma unroll
-          for (int k = 0; k < kCmpBatch; ++k) {
-            const int f = base + ct + k * kCmpThreads;
-            u[k] = f < total ? __ldg(rows4 + f) : make_uint4(0u, 0u, 0u, 0u);
-          }
-#pragma unroll
-          for (int k = 0; k < kCmpBatch; ++k) {
-            const int f = base + ct + k * kCmpThreads;
-            int pc = __popc(u[k].x ^ v.x) + __popc(u[k].y ^ v.y) + __popc(u[k].z ^ v.z) +
-                     __popc(u[k].w ^ v.w);
-            for (int o = cpr >> 1; o >= 1; o >>= 1) pc += __shfl_xor_sync(0xffffffffu, pc, o);
-            if (f < total && (lane & (cpr - 1)) == 0) dist[f / cpr] = pc;
-          }
-        }
-      } else {
-        for (int r = ct; r < m_cnt; r += kCmpThreads)
-          dist[r] = hamming(ri, sk_g + (int64_t)(jlo + r) * nw, nw);
-      }
-    }
-    __syncthreads();
-    int latest = -1;
-    for (int j = i - 1 - tid; j >= wlo; j -= kDetectThreads)
-      if (dist[j - jlo] <= thr) {
-        latest = j;
-        break;
-      }
-    // novel rows of the window other than the new one
-    int nov = 0, nov_tail = 0;
-    for (int r = r0; r < i; r += kDetectThreads) {
-      const int novel = (r == r0 ? lm0 : lm[r]) < wlo;
-      nov += novel;
-      if (r >= n - p.stall_len) nov_tail += novel;
-    }
-    // period runs; P ascends with the thread index, so the first qualifying P of a warp is
-    // its lowest lane's and a thread's first qualifying P is its smallest
-    int pstar = 0x7fffffff;
-    for (int pi = tid; pi < np; pi += kDetectThreads) {
-      const int P = p.p_min + pi;
-      const int cap = max(p.m_rep * P, p.l_min);
-      const int j = i - P;
-      const bool m = j >= 0 && dist[j - jlo] <= thr;
-      const int r = m ? min((pi == tid ? run0 : run[pi]) + 1, cap) : 0;
-      run[pi] = r;
-      if (pstar == 0x7fffffff && n >= cap + P && r >= cap) pstar = P;
-    }
-    latest = __reduce_max_sync(0xffffffffu, latest);
-    nov = __reduce_add_sync(0xffffffffu, nov);
-    nov_tail = __reduce_add_sync(0xffffffffu, nov_tail);
-    pstar = (int)__reduce_min_sync(0xffffffffu, (unsigned)pstar);
+  } else if (warp == kStatWarps) {
+    int ok = 1;
     if (lane == 0) {
-      w_latest[warp] = latest;
-      w_nov[warp] = nov;
-      w_nov_tail[warp] = nov_tail;
-      w_pstar[warp] = pstar;
+      const int n1 = __ldcg(a.c.len + b);
+      s_n = n1;
+      ok = n1 == n0 && __ldcg(ds) == synced0;
     }
-    __syncthreads();
-    if (tid == 0) {
-      int lt = -1, nv = 0, nt = 0, ps = 0x7fffffff;
-      for (int k = 0; k < kDetectWarps; ++k) {
-        lt = max(lt, w_latest[k]);
-        nv += w_nov[k];
-        nt += w_nov_tail[k];
-        ps = min(ps, w_pstar[k]);
+    if (pre) {
+      const uint4 *ri4 = reinterpret_cast<const uint4 *>(sk_g + (int64_t)(n0 - 1) * nw);
+      for (int q = lane; q < cpr; q += 32) {
+        const uint4 x = __ldcg(ri4 + q), y = s_newrow[q];
+        ok &= x.x == y.x && x.y == y.y && x.z == y.z && x.w == y.w;
       }
-      lm[i] = lt;
-      const int novel = lt < wlo;
-      s_novel = nv + novel;
-      s_novel_tail = nt + (p.stall_len >= 1 ? novel : 0);
-      s_pstar = ps;
     }
+    ok = __all_sync(0xffffffffu, ok);
+    if (lane == 0) s_valid = pre && ok;
+  }
+  if (tid == 0) s_bad = bad0;
+  __syncthreads();
+  if (s_bad) return;  // the same decision in every thread of the CTA
+  const int n = s_n;
+  const int w = min(p.W, n);
+  const int wlo = n - w;
+
+  if (s_valid) {
+    // the early phase stands: commit its period runs and the new row's latest match
+    for (int pi = tid; pi < np; pi += kDetectThreads) run[pi] = run_new[pi];
+    if (tid == 0) lm[n - 1] = s_latest;
   } else {
-    // (2') recompute: every window row's latest match, every period's trailing run, from rows
-    // staged in shared memory
+    // (2') recompute (first call, after a prune or any other change of the cache, or when the
+    // early phase's inputs changed): every window row's latest match, every period's trailing
+    // run, from rows staged in shared memory
     const int lo_s = max(0, n - a.smem_rows);
     for (int t = tid; t < (n - lo_s) * nw; t += kDetectThreads) {
       const int r = t / nw;
@@ -501,6 +580,7 @@ __global__ void __launch_bounds__(kDetectThreads, 1) detect_kernel(DetectArgs a)
       s_novel = 0;
       s_novel_tail = 0;
       s_pstar = 0x7fffffff;
+      if (n != n0) form_bounds(n);
     }
     __syncthreads();
     auto row = [=](int r) -> const uint32_t * {
@@ -555,9 +635,10 @@ __global__ void __launch_bounds__(kDetectThreads, 1) detect_kernel(DetectArgs a)
     }
     __syncthreads();
   }
-  // (3) the votes, the stall gate and the trigger, on thread 0, against the bounds formed in (1)
-  // (count_vote, fix_side), then the guard state's update.  The recompute path's counts arrive by
-  // shared-memory atomics (its own barrier above); the incremental path's are thread 0's own.
+  // (3) the votes, the stall gate and the trigger, on thread 0, against the bounds formed in (0)
+  // (again after the wait when the length changed; count_vote, fix_side), then the guard state's
+  // update.  The recompute path's counts arrive by shared-memory atomics (its own barrier above);
+  // the early phase's are thread 0's own.
   if (tid == 0) {
     int trig = 0, sig1 = 0, sig2 = 0, sig3 = 0, stall = 0;
     const bool tailrep = s_pstar != 0x7fffffff;
@@ -754,6 +835,9 @@ __global__ void __launch_bounds__(kCompactThreads) compact_kernel(lg_cache c,
   // the pruned sequences and their counts, in sequence order (read before the status word)
   const bool listed = c.batch <= kCompactSeqList;
   int n_listed = 0;
+  __shared__ int s_bad;
+  // the device status, read beside the kept counts and decided after the listing's barrier
+  const int bad0 = tid == 0 ? (int)status_bad(c.dev_status) : 0;
   if (listed) {
     for (int b0 = 0; b0 < c.batch; b0 += kCompactThreads) {
       const int b = b0 + tid;
@@ -772,10 +856,14 @@ __global__ void __launch_bounds__(kCompactThreads) compact_kernel(lg_cache c,
         s_cnt[at] = k;
       }
       n_listed += tot;
+      if (b0 + kCompactThreads >= c.batch && tid == 0) s_bad = bad0;
       __syncthreads();
     }
+  } else {
+    if (tid == 0) s_bad = bad0;
+    __syncthreads();
   }
-  if (cta_status_bad(c.dev_status)) return;
+  if (s_bad) return;  // the same decision in every thread of the CTA
   const int n_items = (listed ? n_listed : c.batch) * per_seq;
   // grid-stride over (sequence, stream)
   for (int item = blockIdx.x; item < n_items; item += gridDim.x) {

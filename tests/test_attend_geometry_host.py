@@ -70,11 +70,11 @@ static void one(int H_kv, int L, int b, int max_chunks, int n_max, long long len
 }
 int main() {
   // the benchmark's shapes: the paper's setting (28 layers, 8 kv-heads, b 1, 960..1024 rows,
-  // 3 chunks of 384 rows) and the Llama-3-8B-shaped batch (32 layers, 8 kv-heads)
+  // 2 chunks of 512 rows: 448 chunks, at least 3 a CTA on 152 CTAs)
   for (int n = 960; n <= 1024; ++n) {
     AttendArgs a{8, 28, 1, 16};
     const Geom g = make_geom(a, n, n, 152);
-    CHECK(g.per_grp == 3 && g.rows == 384, "paper shape n %%d: %%d x %%d", n, g.per_grp, g.rows);
+    CHECK(g.per_grp == 2 && g.rows == 512, "paper shape n %%d: %%d x %%d", n, g.per_grp, g.rows);
   }
   std::mt19937_64 rng(1);
   auto pick = [&](long long lo, long long hi) { return lo + (long long)(rng() %% (unsigned long long)(hi - lo + 1)); };
