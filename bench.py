@@ -40,7 +40,8 @@ import synth  # noqa: E402
 METRIC = "guarded decode steps/s (attend+stats, detect, prune/compact) and achieved HBM GB/s"
 UNIT = "steps/s"
 L2_BYTES = 129e6
-EV_EVERY = 8  # timing events on every 8th timed step
+EV_EVERY = 8  # timing events on every 8th timed step,
+EV_SAMPLES = 40  # or on about 40 steps of a longer run (each sampled step loses its overlap)
 DEFAULT_STEPS = 400
 DEFAULT_STEPS_W5 = 20   # about 0.25 s of GPU time from the fresh 275 GB cache
 ORACLE_TARGET_S = 20.0  # CPU seconds of the oracle's timed sample (both oracle figures)
@@ -284,7 +285,6 @@ class GpuBench:
         self.n0_d = torch.as_tensor(w.n0, device=dev)
         self.budget_d = torch.as_tensor(w.budget.astype(np.int32), device=dev)
         self.seqs_d = synth.seqs_tensor(w.seqs, dev)
-        self.pos_d = torch.as_tensor(w.n0.astype(np.int64), device=dev)
         bf = torch.bfloat16 if w.dtype == "bf16" else torch.float32
         S, L, b = total_steps, w.L, w.batch
         # both input variants of every step (A = loop continues, B = loop-free), packed per
@@ -305,7 +305,11 @@ class GpuBench:
         self.vn = torch.empty_like(self.kn)
         self.esz = 2 if w.dtype == "bf16" else 4
         e = self.esz
-        self.sel = synth.Select3(w, self.seqs_d, self.pos_d, (self.q, self.kn, self.vn),
+        # each sequence's inputs turn loop-free once the guard has intervened on it (its
+        # state's intervention count); under the comparator policies loops persist
+        self.gstate = self.guard.state if policy == "loopguard" else None
+        self.sel = synth.Select3(w, self.gstate, lg.STATE_BYTES // 4, lg.STATE_WORD_N_INT,
+                                 (self.q, self.kn, self.vn),
                                  (w.H_q * w.d * e, w.H_kv * w.d * e, w.H_kv * w.d * e))
         if detector == "token":
             # generated token ids and top-1 probabilities of every step, both variants
@@ -335,7 +339,6 @@ class GpuBench:
         self.guard.dstate.zero_()
         if self.detector == "token":
             self.tstate.zero_()
-        self.pos_d.copy_(self.n0_d.to(torch.int64))
         self.cache.status.zero_()
         torch.cuda.synchronize()
 
@@ -405,8 +408,9 @@ class GpuBench:
                 tl, tf, pl, pf = self.st_tok
             else:
                 tl, tf, pl, pf = self.tokA[t], self.tokB[t], self.pmA[t], self.pmB[t]
-            synth.dev_select_tokens(w, self.seqs_d, self.pos_d, tl, tf, pl, pf, self.tok,
-                                    self.pm, self.s)
+            synth.dev_select_tokens(w, self.gstate, self.lg.STATE_BYTES // 4,
+                                    self.lg.STATE_WORD_N_INT, tl, tf, pl, pf, self.tok, self.pm,
+                                    self.s)
             lg.lg_token_detect(c, self.tok, self.pm, g.state, p, self.tp, g.flags, g.spans,
                                None, self.tstate, g.kept_idx, g.kept_count, self.s)
         elif guard_path and not split:
@@ -428,7 +432,6 @@ class GpuBench:
             lg.lg_streaming_evict(c, self.budget_d, pos_t, lg.N_SINK, g.max_len, self.s)
         if ev:
             ev[3].record(self.stream)
-        synth.dev_advance(w, self.seqs_d, g.flags if guard_path else None, self.pos_d, self.s)
 
     # launches of this repository's kernels per step (harness + path)
     def launches_per_step(self):
@@ -437,7 +440,7 @@ class GpuBench:
         # partials); a partial pass and a merge on the fp32 path; H2O adds the score update
         attend = 2 + (1 if self.policy == "h2o" else 0)
         path = 1 + 1 + attend * calls               # begin, append (+sketch), attend
-        harness = 1 + 1                             # select, advance
+        harness = 1                                 # the step's inputs
         if self.policy in ("h2o", "streaming"):     # evict, lengths
             path += 2
         elif self.policy == "loopguard" and self.detector == "token":
@@ -612,7 +615,7 @@ def run_gpu(args, ws, rank, local):
     # launch overlap, so events on every step would slow the steps they time)
     # (starting at step every/2, so that the first step's one-off budget cut of every sequence,
     # one step in K of the timed region, does not weigh as one in K/every of the sample)
-    every = 1 if fresh else min(EV_EVERY, max(1, K // 4))
+    every = 1 if fresh else max(min(EV_EVERY, max(1, K // 4)), K // EV_SAMPLES)
     sampled = set(range(every // 2, K, every))
     ev_note = ("every step" if every == 1 else
                "every %dth step of the timed region from step %d (%d of %d), events around the "

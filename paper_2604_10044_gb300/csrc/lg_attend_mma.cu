@@ -45,6 +45,7 @@ constexpr int kTickets = 2 * kMergers;  // finished chunks queued from the consu
                                         // (ticket k in slot k % kTickets, owned by merger k % 4)
 constexpr int kMaxChunkRows = 4096;  // chunk rows at most (the tail of a call is about one chunk)
 constexpr int kStagedSeqs = 256;     // lengths and offsets kept in shared memory up to this batch
+constexpr int kL2KeepBytes = 32 << 20;  // K/V a short pass leaves in L2 at normal priority
 
 template <int D>
 struct MmaCfg {
@@ -489,12 +490,18 @@ attend_mma_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant
     if (lane == 0) {
       // K/V tiles are streamed once per call: their L2 lines go first when space is needed, so
       // that a pass of the whole cache does not evict what the rest of the step works on (the
-      // other kernels' code and data, the workspace); at one sequence (115 MB of K/V a step,
-      // less than the 129 MB L2) this took the paper-shaped step from about 40 to 36.5 us, the
-      // loop-onset test's share most of all, and left the pass itself and its L2 reuse across
-      // calls unchanged
-      uint64_t evict_first;
+      // other kernels' code and data, the workspace).  Same-box A/B at one sequence (115 MB of
+      // K/V a step, less than the 129 MB L2; bench.py --workload 6): 41.7 -> 39.4 us per step,
+      // the loop-onset test's share most of all.
+      uint64_t evict_first, evict_normal;
       asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(evict_first));
+      asm volatile("createpolicy.fractional.L2::evict_normal.b64 %0, 1.0;" : "=l"(evict_normal));
+      // Except the chunks a short pass claims last, about kL2KeepBytes of them: the next call
+      // walks the chunks the other way and starts on these, so they keep normal priority (its
+      // first tiles came from DRAM otherwise: same-box A/B 35.4 -> 34.2 us per step).
+      const int chunk_bytes = gm.rows * 4 * D;  // K and V rows of a full chunk
+      const int keep_from =
+          gm.long_pass ? gm.total : gm.total - max(1, (int)(kL2KeepBytes / chunk_bytes));
       uint32_t it = 0;
       const int claimed0 = 2 * (int)gridDim.x;
       const bool rev = s_rev != 0;
@@ -508,10 +515,12 @@ attend_mma_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant
         const int cm = rev && !gm.long_pass ? gm.total - 1 - c : c;
         int ntiles = 0, grow = 0, n = 0, c_next = 0;
         int64_t lrow0 = 0, head0 = 0;
+        uint64_t policy = evict_first;
         if (alive) {
           c_next = first ? (int)(blockIdx.x + gridDim.x) : claimed0 + atomicAdd(next_chunk, 1);
           first = false;
           const ChunkId id = decode_chunk(a, cm, gm);
+          policy = c >= keep_from ? evict_normal : evict_first;
           n = staged ? s_len[id.b] : a.len[id.b];
           const int64_t off = staged ? s_off[id.b] : a.seq_off[id.b];
           const int row0 = id.ch * gm.rows;
@@ -555,9 +564,9 @@ attend_mma_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant
 #pragma unroll
           for (int h = 0; h < C::kHalves; ++h) {
             tma_load_2d(stage + h * kBoxBytes, &tmK, h * 64, grow + t * kTile,
-                             &full_bar[st], evict_first);
+                             &full_bar[st], policy);
             tma_load_2d(stage + (C::kHalves + h) * kBoxBytes, &tmV, h * 64,
-                             grow + t * kTile, &full_bar[st], evict_first);
+                             grow + t * kTile, &full_bar[st], policy);
           }
           if (t == 0)
             bulk_load(qbuf + st * C::kQBytes,

@@ -52,6 +52,7 @@ class LgTokenParams(ctypes.Structure):
 
 
 STATE_BYTES = 32  # lg_guard_state: 8 x int32
+STATE_WORD_N_INT = 4  # lg_guard_state.n_int: interventions so far
 
 _lib = None
 

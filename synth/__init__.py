@@ -370,14 +370,12 @@ def dev_lib():
                                            vp, vp, vp]
         lib.syn_dev_step.argtypes = [ctypes.POINTER(SynWorkload), vp, i32, vp, i32, vp, vp, vp,
                                      vp]
-        lib.syn_dev_advance.argtypes = [vp, i32, vp, vp, vp]
-        lib.syn_dev_select.argtypes = [vp, i32, vp, i32, i64, vp, vp, vp, vp]
-        lib.syn_dev_select3.argtypes = [vp, i32, vp, i32, vp, vp, vp, vp, vp]
-        lib.syn_dev_select_tokens.argtypes = [vp, i32, vp, vp, vp, vp, vp, vp, vp, vp]
+        lib.syn_dev_select3.argtypes = [vp, i32, i32, i32, i32, vp, vp, vp, vp, vp]
+        lib.syn_dev_select_tokens.argtypes = [vp, i32, i32, i32, vp, vp, vp, vp, vp, vp, vp]
         lib.syn_dev_read_stream.argtypes = [vp, i64, vp, i32, vp]
         lib.syn_dev_read_bulk.argtypes = [vp, i64, i32, vp, vp, i32, vp]
-        for f in (lib.syn_dev_fill_cache, lib.syn_dev_step, lib.syn_dev_advance,
-                  lib.syn_dev_select, lib.syn_dev_select3, lib.syn_dev_select_tokens,
+        for f in (lib.syn_dev_fill_cache, lib.syn_dev_step, lib.syn_dev_select3,
+                  lib.syn_dev_select_tokens,
                   lib.syn_dev_read_stream, lib.syn_dev_read_bulk):
             f.restype = ctypes.c_int
         _dev = lib
@@ -410,22 +408,13 @@ def dev_step(w: Workload, seqs_dev, pos_dev, q, kn, vn, stream, mode: int = 0):
                                   vn.data_ptr(), stream), "syn_dev_step")
 
 
-def dev_advance(w: Workload, seqs_dev, flags_dev, pos_dev, stream):
-    _check(dev_lib().syn_dev_advance(seqs_dev.data_ptr(), w.batch,
-                                     None if flags_dev is None else flags_dev.data_ptr(),
-                                     pos_dev.data_ptr(), stream), "syn_dev_advance")
-
-
-def dev_select(w: Workload, seqs_dev, pos_dev, rowlen_bytes: int, loop_buf, fresh_buf, out,
-               stream):
-    _check(dev_lib().syn_dev_select(seqs_dev.data_ptr(), w.batch, pos_dev.data_ptr(), w.L,
-                                    rowlen_bytes, loop_buf.data_ptr(), fresh_buf.data_ptr(),
-                                    out.data_ptr(), stream), "syn_dev_select")
-
-
-def dev_select_tokens(w: Workload, seqs_dev, pos_dev, tok_loop, tok_fresh, pm_loop, pm_fresh,
-                      tok, pm, stream):
-    _check(dev_lib().syn_dev_select_tokens(seqs_dev.data_ptr(), w.batch, pos_dev.data_ptr(),
+def dev_select_tokens(w: Workload, state, state_words: int, n_int_word: int, tok_loop, tok_fresh,
+                      pm_loop, pm_fresh, tok, pm, stream):
+    """each sequence's token id and top-1 probability of the step: the loop-free variant once the
+    guard state's intervention count (word n_int_word of each state_words-word record) is
+    positive, else the loop-continuing one"""
+    _check(dev_lib().syn_dev_select_tokens(None if state is None else state.data_ptr(),
+                                           state_words, n_int_word, w.batch,
                                            tok_loop.data_ptr(), tok_fresh.data_ptr(),
                                            pm_loop.data_ptr(), pm_fresh.data_ptr(),
                                            tok.data_ptr(), pm.data_ptr(), stream),
@@ -488,10 +477,15 @@ def token_streams(w: Workload, steps: int):
 
 class Select3:
     """one launch that picks each sequence's inputs of a step (q, k_new, v_new) from the
-    loop-continuing or the loop-free variant; argument arrays marshalled once"""
+    loop-continuing or the loop-free variant: the loop-free one once the guard has intervened on
+    the sequence (its state's intervention count, word n_int_word of each state_words-word
+    record, is positive; the paper reports diversity restored after pruning, Sec. 6.2); with no
+    state (the comparator policies) loops persist.  Argument arrays marshalled once."""
 
-    def __init__(self, w, seqs_dev, pos_dev, outs, rowlens):
-        self.w, self.seqs, self.pos = w, seqs_dev, pos_dev
+    def __init__(self, w, state, state_words, n_int_word, outs, rowlens):
+        self.w = w
+        self.state = None if state is None else state.data_ptr()
+        self.state_words, self.n_int_word = state_words, n_int_word
         self.rowlens = (ctypes.c_int64 * 3)(*rowlens)
         self.outs = (ctypes.c_void_p * 3)(*[o.data_ptr() for o in outs])
         self.loop = (ctypes.c_void_p * 3)()
@@ -501,9 +495,9 @@ class Select3:
         for k in range(3):
             self.loop[k] = loop_bufs[k].data_ptr()
             self.fresh[k] = fresh_bufs[k].data_ptr()
-        _check(dev_lib().syn_dev_select3(self.seqs.data_ptr(), self.w.batch, self.pos.data_ptr(),
-                                         self.w.L, self.rowlens, self.loop, self.fresh,
-                                         self.outs, stream), "syn_dev_select3")
+        _check(dev_lib().syn_dev_select3(self.state, self.state_words, self.n_int_word,
+                                         self.w.batch, self.w.L, self.rowlens, self.loop,
+                                         self.fresh, self.outs, stream), "syn_dev_select3")
 
 
 def build(out_dir: str = _HERE, jobs=None):

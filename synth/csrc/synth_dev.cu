@@ -87,31 +87,6 @@ __global__ void step_kv_kernel(syn_workload w, const syn_seq *seqs, int batch,
   store(w, v_new, t, syn_row_value(&w, &s, 1, layer, kvh, b, pos[b], e));
 }
 
-// After a step: a sequence whose guard intervened turns loop-free from the next token on, and
-// every sequence moves to its next position.
-__global__ void advance_kernel(syn_seq *seqs, int batch, const int32_t *flags, int64_t *pos) {
-  pdl_enter();
-  int b = blockIdx.x * blockDim.x + threadIdx.x;
-  if (b >= batch) return;
-  if (flags && flags[b] && seqs[b].fresh_from == SYN_NEVER) seqs[b].fresh_from = (int)pos[b] + 1;
-  pos[b] += 1;
-}
-
-// out = fresh rows for sequences already past fresh_from, else the loop-continuing rows.
-// Buffers are [L][batch][rowlen] elements of esz bytes.
-__global__ void select_kernel(const syn_seq *seqs, int batch, const int64_t *pos, int L,
-                              int64_t rowlen_bytes, const char *loop_buf, const char *fresh_buf,
-                              char *out) {
-  pdl_enter();
-  int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;  // 16-byte chunk index
-  int64_t chunks = rowlen_bytes / 16;
-  int64_t total = (int64_t)L * batch * chunks;
-  if (t >= total) return;
-  int b = (t / chunks) % batch;
-  const char *src = pos[b] >= seqs[b].fresh_from ? fresh_buf : loop_buf;
-  ((uint4 *)out)[t] = ((const uint4 *)src)[t];
-}
-
 // the three selections of one step (q, k_new, v_new) in one launch
 struct Sel3 {
   const char *loop[3];
@@ -120,14 +95,24 @@ struct Sel3 {
   int64_t chunks[3];  // 16-byte chunks per (layer, sequence) row of each tensor
 };
 
-__global__ void select3_kernel(const syn_seq *seqs, int batch, const int64_t *pos, int L, Sel3 s) {
+// Whether sequence b takes the loop-free variant this step: once the guard has intervened on
+// it (the guard state's intervention count, word n_int_word of its state_words-word record, is
+// positive), its next tokens are loop-free; without a guard state (the comparator policies)
+// loops persist.
+__device__ __forceinline__ bool fresh_variant(const int32_t *state, int state_words, int n_int_word,
+                                              int b) {
+  return state && state[(int64_t)b * state_words + n_int_word] > 0;
+}
+
+__global__ void select3_kernel(const int32_t *state, int state_words, int n_int_word, int batch,
+                               int L, Sel3 s) {
   pdl_enter();
   int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   for (int k = 0; k < 3; ++k) {
     const int64_t total = (int64_t)L * batch * s.chunks[k];
     if (t < total) {
       const int b = (int)((t / s.chunks[k]) % batch);
-      const char *src = pos[b] >= seqs[b].fresh_from ? s.fresh[k] : s.loop[k];
+      const char *src = fresh_variant(state, state_words, n_int_word, b) ? s.fresh[k] : s.loop[k];
       ((uint4 *)s.out[k])[t] = ((const uint4 *)src)[t];
       return;
     }
@@ -136,19 +121,18 @@ __global__ void select3_kernel(const syn_seq *seqs, int batch, const int64_t *po
 }
 
 // each sequence's token id and top-1 probability of the step: the loop-continuing variant
-// until the guard has intervened (pos >= fresh_from), the loop-free one after
-__global__ void select_tokens_kernel(const syn_seq *seqs, int batch, const int64_t *pos,
-                                     const int32_t *tok_loop, const int32_t *tok_fresh,
+// until the guard has intervened, the loop-free one after
+__global__ void select_tokens_kernel(const int32_t *state, int state_words, int n_int_word,
+                                     int batch, const int32_t *tok_loop, const int32_t *tok_fresh,
                                      const float *pm_loop, const float *pm_fresh, int32_t *tok,
                                      float *pm) {
   pdl_enter();
   const int b = blockIdx.x * blockDim.x + threadIdx.x;
   if (b >= batch) return;
-  const bool fresh = pos[b] >= seqs[b].fresh_from;
+  const bool fresh = fresh_variant(state, state_words, n_int_word, b);
   tok[b] = fresh ? tok_fresh[b] : tok_loop[b];
   pm[b] = fresh ? pm_fresh[b] : pm_loop[b];
 }
-
 
 // Read-only streaming pass (harness, not part of the generator's recipe): every 16-byte word of
 // the buffer is loaded once with an evict-first hint and folded by XOR into one word per warp,
@@ -269,7 +253,7 @@ __global__ void __launch_bounds__(32) read_bulk_kernel(const unsigned char *p, i
 
 extern "C" {
 
-int syn_dev_select3(const syn_seq *seqs_dev, int batch, const int64_t *pos_dev, int L,
+int syn_dev_select3(const int32_t *state, int state_words, int n_int_word, int batch, int L,
                     const int64_t *rowlen_bytes, const void *const *loop_bufs,
                     const void *const *fresh_bufs, void *const *outs, cudaStream_t stream) {
   Sel3 s;
@@ -283,7 +267,7 @@ int syn_dev_select3(const syn_seq *seqs_dev, int batch, const int64_t *pos_dev, 
     total += (int64_t)L * batch * s.chunks[k];
   }
   return launch_pdl(select3_kernel, dim3((unsigned)((total + 255) / 256)), dim3(256), stream,
-                    seqs_dev, batch, pos_dev, L, s) == cudaSuccess
+                    state, state_words, n_int_word, batch, L, s) == cudaSuccess
              ? 0
              : 2;
 }
@@ -312,31 +296,11 @@ int syn_dev_step(const syn_workload *w, const syn_seq *seqs_dev, int batch, cons
   return cudaGetLastError() == cudaSuccess ? 0 : 2;
 }
 
-int syn_dev_advance(syn_seq *seqs_dev, int batch, const int32_t *flags_dev, int64_t *pos_dev,
-                    cudaStream_t stream) {
-  return launch_pdl(advance_kernel, dim3((batch + 127) / 128), dim3(128), stream, seqs_dev,
-                    batch, flags_dev, pos_dev) == cudaSuccess
-             ? 0
-             : 2;
-}
-
-int syn_dev_select(const syn_seq *seqs_dev, int batch, const int64_t *pos_dev, int L,
-                   int64_t rowlen_bytes, const void *loop_buf, const void *fresh_buf, void *out,
-                   cudaStream_t stream) {
-  if (rowlen_bytes % 16) return 1;
-  int64_t total = (int64_t)L * batch * (rowlen_bytes / 16);
-  return launch_pdl(select_kernel, dim3((unsigned)((total + 255) / 256)), dim3(256), stream,
-                    seqs_dev, batch, pos_dev, L, rowlen_bytes, (const char *)loop_buf,
-                    (const char *)fresh_buf, (char *)out) == cudaSuccess
-             ? 0
-             : 2;
-}
-
-int syn_dev_select_tokens(const syn_seq *seqs_dev, int batch, const int64_t *pos_dev,
+int syn_dev_select_tokens(const int32_t *state, int state_words, int n_int_word, int batch,
                           const int32_t *tok_loop, const int32_t *tok_fresh, const float *pm_loop,
                           const float *pm_fresh, int32_t *tok, float *pm, cudaStream_t stream) {
-  return launch_pdl(select_tokens_kernel, dim3((batch + 127) / 128), dim3(128), stream,
-                    seqs_dev, batch, pos_dev, tok_loop, tok_fresh, pm_loop, pm_fresh, tok,
+  return launch_pdl(select_tokens_kernel, dim3((batch + 127) / 128), dim3(128), stream, state,
+                    state_words, n_int_word, batch, tok_loop, tok_fresh, pm_loop, pm_fresh, tok,
                     pm) == cudaSuccess
              ? 0
              : 2;
