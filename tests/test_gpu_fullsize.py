@@ -8,6 +8,8 @@ The device cache comes from the device generator, the oracle's rows from the hos
              full-size attention) and each side's own sketches of the guard layer;
   prune:     every sequence's kept list, the compacted bytes of sampled streams, and the
              moved sketches of one pruned sequence.
+The Llama-3-8B-shaped workload also runs four whole steps at full size, the attention's own
+statistics driving the loop-onset test, every output and the whole cache compared each step.
 """
 import math
 
@@ -18,7 +20,7 @@ import torch
 import oracle
 import synth
 from paper_2604_10044_gb300 import lg
-from parity_util import OUT_TOL, STAT_TOL, assert_close
+from parity_util import OUT_TOL, STAT_TOL, assert_close, run_loopguard
 
 pytestmark = pytest.mark.gpu
 
@@ -199,3 +201,17 @@ def test_paper_shaped_full_size(cuda):
     B=1024): the first step's attention, detection on seeded statistics and the budget cut"""
     w = synth.make_workload(6)
     assert run_full_size(w, cuda, n_groups=4, n_streams=3) == w.batch
+
+
+def test_llama8b_full_size_four_steps(cuda):
+    """workload 2 at full size (32 layers, 32/8 heads, 8 sequences of 8192 rows, B = 4096) for
+    four guarded steps through the whole path and the oracle side by side: outputs and
+    statistics of every head within tolerance, the votes taken on the attention's own
+    statistics, flags, spans, kept lists, guard state and every cached byte bit for bit (the
+    first step triggers on the looping sequences and cuts every sequence to the budget)"""
+    w = synth.make_workload(2, steps=4)
+    free, _ = torch.cuda.mem_get_info(cuda)
+    if free < w.kv_bytes() + (4 << 30):
+        pytest.skip("needs %.1f GB of free device memory" % ((w.kv_bytes() + (4 << 30)) / 1e9))
+    c = run_loopguard(w, cuda, steps=4)
+    assert c["steps"] == 4 and c["triggers"] >= 1 and c["prunes"] >= w.batch, c

@@ -1,8 +1,8 @@
 """The GPU parity runs compare the guard's decisions bit for bit, float votes included: that is
 sound only if no step's mean entropy or suffix lift lands next to its threshold, where fp32
 statistics on the GPU and fp64 ones in the oracle could take different sides.  This runs the
-oracle alone over the loop-guard workloads of tests/test_gpu_parity.py (the same seeds, shapes
-and step counts) and checks that every step keeps both means at least 1 % from theta_ent and
+oracle alone over the loop-guard workloads of tests/test_gpu_parity.py and the full-size
+multi-step one of tests/test_gpu_fullsize.py (the same seeds, shapes and step counts) and checks that every step keeps both means at least 1 % from theta_ent and
 theta_lift (the tie band of the statistics' tolerance is 1e-4)."""
 import numpy as np
 import pytest
@@ -46,6 +46,8 @@ CASES = [
     ("six-kv-heads", lambda: synth.make_workload(2, L=2, batch=4, n=1200, budget=768, steps=40,
                                                  tail=(300, 500), periods=(8, 40), H_q=12,
                                                  H_kv=6), {}),
+    # test_gpu_fullsize.py::test_llama8b_full_size_four_steps (about 25 s here)
+    ("llama-full-size", lambda: synth.make_workload(2, steps=4), {}),
 ] + [("%s-d%d" % (dt, d), (lambda dt=dt, d=d: _dtype_case(dt, d)), {})
      for dt, d in (("f32", 128), ("bf16", 64), ("f32", 64))]
 
