@@ -338,10 +338,13 @@ __global__ void attend_combine_kernel(AttendArgs a, void *out, float *stats, flo
   }
 }
 
+constexpr int kH2ORows = 4;  // rows of the score update a thread has in flight
+
 // H2O score: h2o[layer][kvh][slot] += sum over the heads of the group of a_i, from the logits
 // kept by the partial pass and the merged (M, l) of every head.
 template <int G>
-__global__ void h2o_accumulate_kernel(AttendArgs a, float *h2o, const float *final_ml) {
+__global__ void __launch_bounds__(256) h2o_accumulate_kernel(AttendArgs a, float *h2o,
+                                                              const float *final_ml) {
   pdl_enter();
   const int kvh = blockIdx.y, b = blockIdx.z % a.batch, lloc = blockIdx.z / a.batch;
   const int layer = a.layer0 + lloc;
@@ -357,12 +360,45 @@ __global__ void h2o_accumulate_kernel(AttendArgs a, float *h2o, const float *fin
   }
   const int64_t lrow0 = ((int64_t)lloc * a.H_kv + kvh) * a.S_total + a.seq_off[b];
   float *sc = h2o + ((int64_t)layer * a.H_kv + kvh) * a.S_total + a.seq_off[b];
-  for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < n; i += gridDim.x * blockDim.x) {
-    const float *lg = a.logits + (lrow0 + i) * G;
-    float acc = 0.f;
+  // kH2ORows rows per thread with all their loads in flight; a row's G logits in 16- or 8-byte
+  // loads where G allows (the logits start 256-byte aligned, a row at a multiple of 4 G bytes)
+  const int stride = gridDim.x * blockDim.x;
+  for (int i0 = blockIdx.x * blockDim.x + threadIdx.x; i0 < n; i0 += kH2ORows * stride) {
+    float lg[kH2ORows][G], old[kH2ORows];
 #pragma unroll
-    for (int g = 0; g < G; ++g) acc += exp2f(lg[g] - M[g]) * inv_l[g];
-    sc[i] += acc;
+    for (int k = 0; k < kH2ORows; ++k) {
+      const int i = i0 + k * stride;
+      if (i < n) {
+        const float *src = a.logits + (lrow0 + i) * G;
+        if (G % 4 == 0) {
+#pragma unroll
+          for (int g = 0; g < G; g += 4) {
+            const float4 v = *reinterpret_cast<const float4 *>(src + g);
+            lg[k][g] = v.x, lg[k][g + 1] = v.y, lg[k][g + 2] = v.z, lg[k][g + 3] = v.w;
+          }
+        } else if (G % 2 == 0) {
+#pragma unroll
+          for (int g = 0; g < G; g += 2) {
+            const float2 v = *reinterpret_cast<const float2 *>(src + g);
+            lg[k][g] = v.x, lg[k][g + 1] = v.y;
+          }
+        } else {
+#pragma unroll
+          for (int g = 0; g < G; ++g) lg[k][g] = src[g];
+        }
+        old[k] = sc[i];
+      }
+    }
+#pragma unroll
+    for (int k = 0; k < kH2ORows; ++k) {
+      const int i = i0 + k * stride;
+      if (i < n) {
+        float acc = 0.f;
+#pragma unroll
+        for (int g = 0; g < G; ++g) acc += exp2f(lg[k][g] - M[g]) * inv_l[g];
+        sc[i] = old[k] + acc;
+      }
+    }
   }
 }
 
@@ -393,8 +429,11 @@ static cudaError_t launch_typed(const AttendArgs &a, int64_t rows_total, void *o
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
   }
   if (h2o) {
-    int gx = (a.max_len + 255) / 256;
-    if (gx > 64) gx = 64;
+    // at most 16 CTAs a (layer, sequence, kv-head) stream: up to 16 K rows a stream leave each
+    // thread its kH2ORows rows in flight (a grid sized for one row a thread ran with half the
+    // warps resident and most of its CTAs idle on short sequences)
+    int gx = (a.max_len + 256 * kH2ORows - 1) / (256 * kH2ORows);
+    if (gx > 16) gx = 16;
     LG_TRY(launch_pdl(h2o_accumulate_kernel<G>, dim3(gx, a.H_kv, a.n_layers * a.batch), 256, 0, s,
                       a, h2o, final_ml));
     e = cudaGetLastError();

@@ -717,8 +717,16 @@ attend_mma_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant
           const int rl = r_w + mb * 16 + g + half * 8;
           if (rl < tile_rows) {
             float *dst = logits + (lrow0 + t * kTile + rl) * G;
-            if (2 * t4 < G) dst[2 * t4] = s[mb][half * 2];
-            if (2 * t4 + 1 < G) dst[2 * t4 + 1] = s[mb][half * 2 + 1];
+            if (G % 2 == 0) {
+              // heads 2 t4 and 2 t4 + 1 side by side: one 8-byte store (rows of an even G
+              // start 8-byte aligned)
+              if (2 * t4 < G)
+                *reinterpret_cast<float2 *>(dst + 2 * t4) =
+                    make_float2(s[mb][half * 2], s[mb][half * 2 + 1]);
+            } else {
+              if (2 * t4 < G) dst[2 * t4] = s[mb][half * 2];
+              if (2 * t4 + 1 < G) dst[2 * t4 + 1] = s[mb][half * 2 + 1];
+            }
           }
         }
       }
