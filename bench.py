@@ -81,6 +81,7 @@ def parse():
                          "print its measures instead of the step benchmark")
     ap.add_argument("--eager", action="store_true",
                     help="time the steps as eager launches instead of one CUDA graph replay")
+    ap.add_argument("--oracle-one-thread", action="store_true", help=argparse.SUPPRESS)
     ap.add_argument("--profile-steps", type=int, default=0,
                     help="run this many steps untimed and exit (for ncu launch lists)")
     args = ap.parse_args()
@@ -911,7 +912,7 @@ def time_oracle(w, n_seq, n_layers, steps, warm=0, policy="loopguard"):
     return run(steps)
 
 
-def oracle_sample(w, K, W, policy="loopguard", target_s=ORACLE_TARGET_S):
+def oracle_sample(w, K, W, policy="loopguard", target_s=ORACLE_TARGET_S, max_layers=None):
     """The oracle on a bounded sample of the GPU arm's timed run: sequence 0 of the batch and its
     first n_layers layers, W warm-up steps, then the same K consecutive guarded decode steps from
     a fresh cache (the first carries the budget cut, as on the GPU).  n_layers is sized from a
@@ -919,28 +920,45 @@ def oracle_sample(w, K, W, policy="loopguard", target_s=ORACLE_TARGET_S):
     of bench.py (the GPU line's cpu_baseline and the --impl reference line) are this sample.
     Returns a dict: value (batch steps/s, the sample scaled by sequences and layers), the
     measured seconds, the scale and a description."""
-    cal = min(K, 3)
-    t_cal, _ = time_oracle(w, 1, 1, cal, policy=policy)
-    per_layer = t_cal[0] + (K - 1) * (float(np.mean(t_cal[1:])) if cal > 1 else t_cal[0])
-    n_layers = int(max(1, min(w.L, target_s // max(per_layer, 1e-6))))
+    if max_layers == 1:
+        n_layers = 1
+    else:
+        cal = min(K, 3)
+        t_cal, _ = time_oracle(w, 1, 1, cal, policy=policy)
+        per_layer = t_cal[0] + (K - 1) * (float(np.mean(t_cal[1:])) if cal > 1 else t_cal[0])
+        n_layers = int(max(1, min(max_layers or w.L, target_s // max(per_layer, 1e-6))))
     times, threads = time_oracle(w, 1, n_layers, K, warm=W, policy=policy)
     sec = sum(times)
     scale = (1.0 / w.batch) * (n_layers / w.L)   # batch steps per sampled step
     return {"value": K * scale / sec, "sec": sec, "steps": K, "scale": scale,
             "threads": threads, "n_layers": n_layers,
-            "sample": "%d guarded decode steps from a fresh cache (after %d warm-up step(s)), the "
-                      "same trajectory as the GPU arm's timed steps, of sequence 0 of %d and its "
+            "sample": "the first %d guarded decode steps of the GPU arm's timed trajectory, from "
+                      "its fresh cache (after %d warm-up step(s)), of sequence 0 of %d and its "
                       "layers 0..%d of %d; value = steps x %.6f batch steps per sampled step / "
                       "%.2f s" % (K, W, w.batch, n_layers - 1, w.L, scale, sec)}
 
 
 def cpu_baseline(w, args):
-    """the oracle on the host cores: the bounded sample of oracle_sample, as batch steps/s"""
+    """the oracle on the host cores: the bounded sample of oracle_sample, as batch steps/s; and
+    beside it the same trajectory's first steps on one thread (one layer, at most 2 steps, in a
+    fresh interpreter: the oracle takes its thread count when it loads)"""
     o = oracle_sample(w, args.steps, args.warmup, args.policy)
-    return {"value": round(o["value"], 6), "unit": UNIT, "cores": o["threads"],
+    line = {"value": round(o["value"], 6), "unit": UNIT, "cores": o["threads"],
             "kind": "oracle", "affinity_cores": len(os.sched_getaffinity(0)),
             "sample": o["sample"], "sample_scale": o["scale"],
             "ms_per_sample_step": round(o["sec"] / o["steps"] * 1e3, 3)}
+    try:
+        env = dict(os.environ, OMP_NUM_THREADS="1")
+        r = subprocess.run([sys.executable, os.path.abspath(__file__), "--oracle-one-thread",
+                            "--workload", str(args.workload), "--steps", str(min(args.steps, 2)),
+                            "--policy", args.policy], env=env, capture_output=True, text=True,
+                           timeout=600)
+        one = json.loads(r.stdout.strip().splitlines()[-1])
+        line["single_thread"] = {"value": round(one["value"], 6), "unit": UNIT,
+                                 "cores": one["threads"], "sample": one["sample"]}
+    except Exception as e:  # a reported extra: its failure leaves the main figure
+        line["single_thread"] = {"value": None, "error": str(e)[:200]}
+    return line
 
 
 def run_reference(args, ws, rank):
@@ -994,6 +1012,13 @@ def run_ablation(args, local):
 
 def main():
     args = parse()
+    if args.oracle_one_thread:
+        # internal: the oracle's sample on this process's threads (one, from the environment)
+        w = synth.make_workload(args.workload, steps=max(args.steps, 1))
+        o = oracle_sample(w, args.steps, 0, args.policy, target_s=0.0, max_layers=1)
+        print(json.dumps({"value": o["value"], "threads": o["threads"], "sample": o["sample"]}),
+              flush=True)
+        return
     ws, rank, local = dist_setup()
     if args.ablation:
         if rank == 0:
