@@ -74,7 +74,7 @@ def parse():
     ap.add_argument("--detector", default="kv", choices=["kv", "token"],
                     help="loop-onset test of the LoopGuard policy: over attention statistics and "
                          "V-row sketches (lg_detect_prune), or over the generated token ids and "
-                         "top-1 probabilities (lg_token_detect + lg_prune_compact)")
+                         "top-1 probabilities (lg_token_detect_prune)")
     ap.add_argument("--ablation", action="store_true",
                     help="run the synthetic analog of the paper's ablation (no guard, always-on "
                          "pruning, the confidence streak alone, the full guard) on the GPU path and "
@@ -161,7 +161,7 @@ def run_config(w, args, ws):
     return dict(w.describe(), decode_steps=args.steps, l2=l2_note(w), policy=args.policy,
                 timed_steps="each from a fresh cache" if args.fresh_each_step
                 else "consecutive decode steps from a fresh cache",
-                detector="token ids and p_max (lg_token_detect)"
+                detector="token ids and p_max (lg_token_detect_prune)"
                 if args.detector == "token" else "attention statistics and V-row sketches",
                 parallelism="dp%d (independent batches, no collective)" % ws,
                 tokens_per_step=w.batch * ws)
@@ -377,16 +377,25 @@ class GpuBench:
         return torch.cat(rows, 1).contiguous().pin_memory()
 
     def select_inputs(self, t):
-        if getattr(self, "stage", None) is not None:
-            self.sel(self.st_A, self.st_B, self.s)
+        """the step's q, k_new, v_new (and, for the token-level monitor, its token id and top-1
+        probability) in one launch, each sequence's variant chosen by its guard state"""
+        staged = getattr(self, "stage", None) is not None
+        tokens = None
+        if self.detector == "token" and self.policy == "loopguard":
+            tl, tf, pl, pf = (self.st_tok if staged else
+                              (self.tokA[t], self.tokB[t], self.pmA[t], self.pmB[t]))
+            tokens = (tl, tf, pl, pf, self.tok, self.pm)
+        if staged:
+            self.sel(self.st_A, self.st_B, self.s, tokens)
             return
         self.sel((self.qA[t], self.kA[t], self.vA[t]), (self.qB[t], self.kB[t], self.vB[t]),
-                 self.s)
+                 self.s, tokens)
 
     def step(self, t, ev=None, split=False):
         """one guarded decode step; ev = (a0, a1, p0, p1) events around attend and the guard
         (a1 -> p1); split: the loop-onset test and the compaction as separate calls
-        (lg_detect, lg_prune_compact: the same results) with p0 between them"""
+        (lg_detect or lg_token_detect, then lg_prune_compact: the same results) with p0 between
+        them"""
         lg, c, g, p, w = self.lg, self.cache, self.guard, self.p, self.w
         h2o = self.policy == "h2o"
         guard_path = self.policy == "loopguard"
@@ -403,15 +412,13 @@ class GpuBench:
         if ev:
             ev[1].record(self.stream)
         token = guard_path and self.detector == "token"
-        if token:
-            # the caller's generated token and top-1 probability, then the token-level monitor
-            if getattr(self, "stage", None) is not None:
-                tl, tf, pl, pf = self.st_tok
-            else:
-                tl, tf, pl, pf = self.tokA[t], self.tokB[t], self.pmA[t], self.pmB[t]
-            synth.dev_select_tokens(w, self.gstate, self.lg.STATE_BYTES // 4,
-                                    self.lg.STATE_WORD_N_INT, tl, tf, pl, pf, self.tok, self.pm,
-                                    self.s)
+        if token and not split:
+            # the token-level monitor on the step's token and top-1 probability (picked with the
+            # step's inputs), its retained set, then the compaction
+            lg.lg_token_detect_prune(c, self.tok, self.pm, g.state, self.budget_d, p, self.tp,
+                                     g.flags, g.spans, None, self.tstate, g.kept_idx,
+                                     g.kept_count, g.max_keep, g.max_len, self.s)
+        elif token:
             lg.lg_token_detect(c, self.tok, self.pm, g.state, p, self.tp, g.flags, g.spans,
                                None, self.tstate, g.kept_idx, g.kept_count, self.s)
         elif guard_path and not split:
@@ -424,7 +431,7 @@ class GpuBench:
                          g.dstate, self.s)
         if ev:
             ev[2].record(self.stream)
-        if guard_path and (split or token):
+        if guard_path and split:
             lg.lg_prune_compact(c, g.flags, g.spans, g.state, self.budget_d, p, g.kept_idx,
                                 g.kept_count, g.max_keep, g.max_len, self.s)
         elif h2o:
@@ -445,8 +452,7 @@ class GpuBench:
         if self.policy in ("h2o", "streaming"):     # evict, lengths
             path += 2
         elif self.policy == "loopguard" and self.detector == "token":
-            path += 3                               # token monitor, keep set, compact
-            harness += 1                            # the step's token and p_max
+            path += 2                               # token monitor + keep, compact
         elif self.policy == "loopguard":
             path += 2                               # detect + keep, compact
         return path, harness
@@ -1006,7 +1012,7 @@ def run_ablation(args, local):
         "variants": res, "data": "synthetic",
         "config": {"sequences": streams.batch, "prompt": 3853, "budget": 1024,
                    "steps": streams.steps, "onset": "U{800..1300}", "period": "U{16..64}",
-                   "detector": "token-level monitor (lg_token_detect) + lg_prune_compact"}}),
+                   "detector": "token-level monitor and retained set (lg_token_detect_prune)"}}),
         flush=True)
 
 

@@ -10,7 +10,9 @@
  *
  * A decode step on this ABI:
  *   lg_begin_step -> lg_append -> lg_decode_attend -> lg_detect -> lg_prune_compact
- *   (lg_detect_prune fuses the last two)
+ *   (lg_detect_prune fuses the last two), or with the token-level monitor:
+ *   lg_begin_step -> lg_append -> lg_decode_attend -> lg_token_detect -> lg_prune_compact
+ *   (lg_token_detect_prune fuses the last two)
  * or, on the comparator path:
  *   lg_begin_step -> lg_append -> lg_decode_attend(accumulate_h2o=1) -> lg_h2o_evict
  *
@@ -23,9 +25,14 @@
  *  - Kernels are launched with programmatic stream serialization (programmatic dependent
  *    launch): each may be scheduled while the kernel before it in the stream is still running,
  *    and waits (griddepcontrol.wait) for that kernel to complete before it touches memory, so
- *    stream order holds as usual.  A kernel of the caller's that follows one of the library's
- *    on the same stream keeps full stream order unless the caller launches it with the same
- *    attribute, in which case it must wait the same way.
+ *    stream order holds as usual.  One exception, invisible to the caller: lg_detect's kernel
+ *    reads the lengths, the monitor state and the sketches before its wait, then reads the
+ *    length, the synced length and the new row again after it and drops everything read early
+ *    unless all three are unchanged.  Only a library kernel can be running at that point: a
+ *    kernel of the caller's (launched without the attribute) completes before the next
+ *    kernel starts.  A kernel of the caller's that follows one of the library's on the same
+ *    stream keeps full stream order unless the caller launches it with the same attribute, in
+ *    which case it must wait the same way.
  *  - Arguments are validated on the host before any launch (null or misaligned pointers,
  *    unsupported shapes, short workspaces): the call returns an error and launches nothing.
  *  - Errors only visible on the device (a length above its capacity or above the call's
@@ -265,6 +272,20 @@ LG_API lg_status lg_token_detect(const lg_cache *c, const int32_t *tokens, const
                                  int max_keep, lg_guard_state *state, const lg_guard_params *p,
                                  const lg_token_params *tp, int32_t *flags, int32_t *spans,
                                  double *diag, void *tstate, cudaStream_t s);
+
+/* lg_token_detect (passed the kept lists) followed by lg_prune_compact (same results, same
+   device state), with the retained set formed by the token-level monitor's own kernel: two
+   kernel launches instead of three.  kept_idx and kept_count are required: the kernel reads
+   the previous prune's lists from them (as lg_token_detect does) and then writes this step's
+   over them (as lg_prune_compact does).  budget, max_keep and max_len as for lg_prune_compact;
+   validation is the union of both calls'. */
+LG_API lg_status lg_token_detect_prune(const lg_cache *c, const int32_t *tokens,
+                                       const float *pmax, lg_guard_state *state,
+                                       const int32_t *budget, const lg_guard_params *p,
+                                       const lg_token_params *tp, int32_t *flags, int32_t *spans,
+                                       double *diag, void *tstate, int32_t *kept_idx,
+                                       int32_t *kept_count, int max_keep, int max_len,
+                                       cudaStream_t s);
 
 /* Bytes of lg_detect's dstate: (batch * (p_max - p_min + 3) + S_total) 32-bit words. */
 LG_API size_t lg_detect_state_size(const lg_cache *c, const lg_guard_params *p);

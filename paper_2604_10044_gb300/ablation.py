@@ -42,12 +42,12 @@ def run_variant(streams, over, device, budget=1024, stream=None):
         pm_d.copy_(torch.from_numpy(pm))
         lg.lg_begin_step(cache, stream)
         if over is not None:
-            lg.lg_token_detect(cache, tok_d, pm_d, state, prm, tp, flags, spans, None, tstate,
-                               kept_idx, kept_count, stream)
-        lg.lg_prune_compact(cache, flags if over is not None else None,
-                            spans if over is not None else None,
-                            state if over is not None else None, budget_d, prm, kept_idx,
-                            kept_count, max_keep, int(cap.max()), stream)
+            lg.lg_token_detect_prune(cache, tok_d, pm_d, state, budget_d, prm, tp, flags, spans,
+                                     None, tstate, kept_idx, kept_count, max_keep, int(cap.max()),
+                                     stream)
+        else:
+            lg.lg_prune_compact(cache, None, None, None, budget_d, prm, kept_idx, kept_count,
+                                max_keep, int(cap.max()), stream)
         f = flags.cpu().numpy() if over is not None else np.zeros(b, dtype=np.int32)
         kc = kept_count.cpu().numpy()
         kept = [None] * b

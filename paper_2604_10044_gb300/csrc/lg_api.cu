@@ -289,8 +289,30 @@ lg_status lg_token_detect(const lg_cache *c, const int32_t *tokens, const float 
   if (((uintptr_t)state & 15u) || ((uintptr_t)tstate & 7u)) return LG_ERR_INVALID_ARG;
   if ((kept_idx == nullptr) != (kept_count == nullptr) || (kept_idx && max_keep < 1))
     return LG_ERR_INVALID_ARG;
-  return cuda_status(lg::launch_token_detect(*c, tokens, pmax, kept_idx, kept_count, max_keep,
-                                             state, *p, *tp, flags, spans, diag, tstate, s));
+  return cuda_status(lg::launch_token_detect(*c, tokens, pmax, const_cast<int32_t *>(kept_idx),
+                                             const_cast<int32_t *>(kept_count), max_keep, state,
+                                             *p, *tp, flags, spans, diag, tstate, nullptr, 0, s));
+}
+
+lg_status lg_token_detect_prune(const lg_cache *c, const int32_t *tokens, const float *pmax,
+                                lg_guard_state *state, const int32_t *budget,
+                                const lg_guard_params *p, const lg_token_params *tp,
+                                int32_t *flags, int32_t *spans, double *diag, void *tstate,
+                                int32_t *kept_idx, int32_t *kept_count, int max_keep,
+                                int max_len, cudaStream_t s) {
+  lg_status st = check_cache(c);
+  if (st != LG_OK) return st;
+  if ((st = check_params(p)) != LG_OK) return st;
+  if ((st = check_token_params(p, tp)) != LG_OK) return st;
+  if (!tokens || !pmax || !state || !budget || !flags || !spans || !tstate)
+    return LG_ERR_INVALID_ARG;
+  if (((uintptr_t)state & 15u) || ((uintptr_t)tstate & 7u)) return LG_ERR_INVALID_ARG;
+  if (!kept_idx || !kept_count || max_keep < 1 || max_len < 0) return LG_ERR_INVALID_ARG;
+  st = cuda_status(lg::launch_token_detect(*c, tokens, pmax, kept_idx, kept_count, max_keep,
+                                           state, *p, *tp, flags, spans, diag, tstate, budget,
+                                           max_len, s));
+  if (st != LG_OK) return st;
+  return cuda_status(lg::launch_compact(*c, kept_idx, kept_count, max_keep, s));
 }
 
 size_t lg_detect_state_size(const lg_cache *c, const lg_guard_params *p) {

@@ -62,11 +62,13 @@ cudaError_t launch_compact(const lg_cache &c, const int32_t *kept_idx, const int
 // token-level monitor (lg_token.cu)
 size_t token_state_words(const lg_guard_params &p, const lg_token_params &tp);
 size_t token_smem_bytes(const lg_guard_params &p, const lg_token_params &tp);
+// budget non-null: the kernel also writes this step's kept lists over kept_idx/kept_count
 cudaError_t launch_token_detect(const lg_cache &c, const int32_t *tokens, const float *pmax,
-                                const int32_t *kept_idx, const int32_t *kept_count, int max_keep,
+                                int32_t *kept_idx, int32_t *kept_count, int max_keep,
                                 lg_guard_state *state, const lg_guard_params &p,
                                 const lg_token_params &tp, int32_t *flags, int32_t *spans,
-                                double *diag, void *tstate, cudaStream_t s);
+                                double *diag, void *tstate, const int32_t *budget, int max_len,
+                                cudaStream_t s);
 cudaError_t launch_h2o_reset(const lg_cache &c, int max_len, cudaStream_t s);
 cudaError_t launch_h2o_evict(const lg_cache &c, const int32_t *budget, const int32_t *pos_now,
                              int max_len, cudaStream_t s);

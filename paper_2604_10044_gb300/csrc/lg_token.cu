@@ -25,6 +25,7 @@
 
 #include "lg_common.cuh"
 #include "lg_internal.h"
+#include "lg_keep.cuh"
 
 namespace lg {
 
@@ -38,9 +39,14 @@ struct TokenArgs {
   lg_cache c;
   const int32_t *tokens;  // [batch] this step's token of each sequence
   const float *pmax;      // [batch] this step's top-1 probability
-  const int32_t *kept_idx;    // nullable [batch][max_keep]: the prune after the previous step
-  const int32_t *kept_count;  // nullable [batch], -1 = that sequence was not pruned
+  int32_t *kept_idx;    // nullable [batch][max_keep]: the prune after the previous step
+  int32_t *kept_count;  // nullable [batch], -1 = that sequence was not pruned
   int max_keep;
+  // set: the same CTA goes on to this step's retained set (as lg_prune_compact's kernel forms
+  // it), written over the previous kept lists once they have been read
+  const int32_t *budget;
+  int max_len;
+  int prune;
   lg_guard_state *state;
   lg_guard_params p;
   lg_token_params tp;
@@ -71,7 +77,8 @@ __global__ void __launch_bounds__(kTokThreads, 1) token_detect_kernel(TokenArgs 
   __shared__ int red[kTokWarps];
   __shared__ int w_latest[kTokWarps], w_nov[kTokWarps], w_tail[kTokWarps], w_pstar[kTokWarps],
       w_run[kTokWarps];
-  __shared__ int s_mismatch, s_trig, s_P, s_n_tok, s_appended;
+  __shared__ int s_mismatch, s_trig, s_P, s_n_tok, s_appended, s_flag, s_level, s_span_lo,
+      s_span_hi;
   const int b = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const lg_guard_params &p = a.p;
   const lg_token_params &tp = a.tp;
@@ -91,6 +98,7 @@ __global__ void __launch_bounds__(kTokThreads, 1) token_detect_kernel(TokenArgs 
   const int t = ts[0];  // tokens before this one: this token is position t
   const int synced = ts[2] - 1, app_old = ts[3];
   const int kc = a.kept_count ? a.kept_count[b] : -1;
+  const int B = a.prune ? a.budget[b] : 0;
   int4 st_a = make_int4(0, 0, 0, 0), st_b = make_int4(0, 0, 0, 0);
   if (tid == 0) {
     st_a = reinterpret_cast<const int4 *>(a.state + b)[0];
@@ -270,6 +278,9 @@ __global__ void __launch_bounds__(kTokThreads, 1) token_detect_kernel(TokenArgs 
     s_n_tok = Tn;
     s_appended = appended;
     s_mismatch = -1;
+    s_flag = trig;
+    s_level = st_a.z;
+    s_span_lo = s_span_hi = 0;
     a.flags[b] = trig;
     a.spans[2 * b] = 0;
     a.spans[2 * b + 1] = 0;
@@ -297,7 +308,20 @@ __global__ void __launch_bounds__(kTokThreads, 1) token_detect_kernel(TokenArgs 
       const int bad = min(s_n_tok - (s - P), s_appended);
       a.spans[2 * b] = n - bad;
       a.spans[2 * b + 1] = n;
+      s_span_lo = n - bad;
+      s_span_hi = n;
     }
+  }
+
+  // (5) fused prune: the retained set of this sequence from the decision just taken, the span
+  // clipped to W^recent by keep_plan as in lg_prune_compact.  Every read of the previous kept
+  // lists (1) lies before the barrier of (3), so they may be overwritten now.
+  if (a.prune) {
+    __syncthreads();  // thread 0's span
+    const int code = write_keep(a.c, b, n, B, s_flag, s_span_lo, s_span_hi, s_level, p,
+                                a.kept_idx, a.kept_count, a.max_keep, a.max_len, tid,
+                                kTokThreads);
+    if (code && tid == 0) set_status(a.c.dev_status, code);
   }
 }
 
@@ -312,10 +336,11 @@ size_t token_smem_bytes(const lg_guard_params &p, const lg_token_params &tp) {
 }
 
 cudaError_t launch_token_detect(const lg_cache &c, const int32_t *tokens, const float *pmax,
-                                const int32_t *kept_idx, const int32_t *kept_count, int max_keep,
+                                int32_t *kept_idx, int32_t *kept_count, int max_keep,
                                 lg_guard_state *state, const lg_guard_params &p,
                                 const lg_token_params &tp, int32_t *flags, int32_t *spans,
-                                double *diag, void *tstate, cudaStream_t s) {
+                                double *diag, void *tstate, const int32_t *budget, int max_len,
+                                cudaStream_t s) {
   TokenArgs a;
   a.c = c;
   a.tokens = tokens;
@@ -323,6 +348,9 @@ cudaError_t launch_token_detect(const lg_cache &c, const int32_t *tokens, const 
   a.kept_idx = kept_idx;
   a.kept_count = kept_count;
   a.max_keep = max_keep;
+  a.budget = budget;
+  a.max_len = max_len;
+  a.prune = budget != nullptr;
   a.state = state;
   a.p = p;
   a.tp = tp;

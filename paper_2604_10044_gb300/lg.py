@@ -82,6 +82,8 @@ def lib():
             "lg_token_state_size": [P(LgCache), P(LgGuardParams), P(LgTokenParams)],
             "lg_token_detect": [P(LgCache), vp, vp, vp, vp, i32, vp, P(LgGuardParams),
                                 P(LgTokenParams), vp, vp, vp, vp, vp],
+            "lg_token_detect_prune": [P(LgCache), vp, vp, vp, vp, P(LgGuardParams),
+                                      P(LgTokenParams), vp, vp, vp, vp, vp, vp, i32, i32, vp],
             "lg_prune_compact": [P(LgCache), vp, vp, vp, vp, P(LgGuardParams), vp, vp, i32, i32,
                                  vp],
             "lg_h2o_reset": [P(LgCache), i32, vp],
@@ -111,7 +113,7 @@ def exported_symbols():
             "lg_prune_compact", "lg_h2o_reset", "lg_h2o_evict", "lg_read_device_status",
             "lg_decode_attend_noalloc", "lg_detect_state_size", "lg_streaming_evict",
             "lg_detect_prune", "lg_default_token_params", "lg_token_state_size",
-            "lg_token_detect"]
+            "lg_token_detect", "lg_token_detect_prune"]
 
 NOALLOC_SCRATCH_BYTES = 32 << 20  # LG_NOALLOC_SCRATCH_BYTES in include/lg.h
 
@@ -215,6 +217,16 @@ def lg_token_detect(cache, tokens, pmax, state, params, tparams, flags, spans, d
     _call("lg_token_detect", ctypes.byref(cache.c), _ptr(tokens), _ptr(pmax), _ptr(kept_idx),
           _ptr(kept_count), max_keep, _ptr(state), ctypes.byref(params), ctypes.byref(tparams),
           _ptr(flags), _ptr(spans), _ptr(diag), _ptr(tstate), _stream(stream))
+
+
+def lg_token_detect_prune(cache, tokens, pmax, state, budget, params, tparams, flags, spans,
+                          diag, tstate, kept_idx, kept_count, max_keep, max_len, stream=None):
+    """lg_token_detect then lg_prune_compact in two launches; kept_idx / kept_count carry the
+    previous prune's lists in and this step's out"""
+    _call("lg_token_detect_prune", ctypes.byref(cache.c), _ptr(tokens), _ptr(pmax), _ptr(state),
+          _ptr(budget), ctypes.byref(params), ctypes.byref(tparams), _ptr(flags), _ptr(spans),
+          _ptr(diag), _ptr(tstate), _ptr(kept_idx), _ptr(kept_count), max_keep, max_len,
+          _stream(stream))
 
 
 def lg_detect(cache, stats, H_q, state, budget, params, flags, spans, diag, dstate, stream=None):

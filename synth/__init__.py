@@ -370,12 +370,11 @@ def dev_lib():
                                            vp, vp, vp]
         lib.syn_dev_step.argtypes = [ctypes.POINTER(SynWorkload), vp, i32, vp, i32, vp, vp, vp,
                                      vp]
-        lib.syn_dev_select3.argtypes = [vp, i32, i32, i32, i32, vp, vp, vp, vp, vp]
-        lib.syn_dev_select_tokens.argtypes = [vp, i32, i32, i32, vp, vp, vp, vp, vp, vp, vp]
+        lib.syn_dev_select3.argtypes = [vp, i32, i32, i32, i32, vp, vp, vp, vp, vp, vp, vp, vp,
+                                        vp, vp, vp]
         lib.syn_dev_read_stream.argtypes = [vp, i64, vp, i32, vp]
         lib.syn_dev_read_bulk.argtypes = [vp, i64, i32, vp, vp, i32, vp]
         for f in (lib.syn_dev_fill_cache, lib.syn_dev_step, lib.syn_dev_select3,
-                  lib.syn_dev_select_tokens,
                   lib.syn_dev_read_stream, lib.syn_dev_read_bulk):
             f.restype = ctypes.c_int
         _dev = lib
@@ -406,19 +405,6 @@ def dev_step(w: Workload, seqs_dev, pos_dev, q, kn, vn, stream, mode: int = 0):
     _check(dev_lib().syn_dev_step(ctypes.byref(cw), seqs_dev.data_ptr(), w.batch,
                                   pos_dev.data_ptr(), mode, q.data_ptr(), kn.data_ptr(),
                                   vn.data_ptr(), stream), "syn_dev_step")
-
-
-def dev_select_tokens(w: Workload, state, state_words: int, n_int_word: int, tok_loop, tok_fresh,
-                      pm_loop, pm_fresh, tok, pm, stream):
-    """each sequence's token id and top-1 probability of the step: the loop-free variant once the
-    guard state's intervention count (word n_int_word of each state_words-word record) is
-    positive, else the loop-continuing one"""
-    _check(dev_lib().syn_dev_select_tokens(None if state is None else state.data_ptr(),
-                                           state_words, n_int_word, w.batch,
-                                           tok_loop.data_ptr(), tok_fresh.data_ptr(),
-                                           pm_loop.data_ptr(), pm_fresh.data_ptr(),
-                                           tok.data_ptr(), pm.data_ptr(), stream),
-           "syn_dev_select_tokens")
 
 
 def dev_read_stream(buf, sink, ctas: int, stream):
@@ -491,13 +477,16 @@ class Select3:
         self.loop = (ctypes.c_void_p * 3)()
         self.fresh = (ctypes.c_void_p * 3)()
 
-    def __call__(self, loop_bufs, fresh_bufs, stream):
+    def __call__(self, loop_bufs, fresh_bufs, stream, tokens=None):
+        """tokens: None, or (tok_loop, tok_fresh, pm_loop, pm_fresh, tok, pm), [batch] each:
+        the same launch also picks each sequence's token id and top-1 probability"""
         for k in range(3):
             self.loop[k] = loop_bufs[k].data_ptr()
             self.fresh[k] = fresh_bufs[k].data_ptr()
+        tk = [None] * 6 if tokens is None else [x.data_ptr() for x in tokens]
         _check(dev_lib().syn_dev_select3(self.state, self.state_words, self.n_int_word,
                                          self.w.batch, self.w.L, self.rowlens, self.loop,
-                                         self.fresh, self.outs, stream), "syn_dev_select3")
+                                         self.fresh, self.outs, *tk, stream), "syn_dev_select3")
 
 
 def build(out_dir: str = _HERE, jobs=None):

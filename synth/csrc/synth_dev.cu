@@ -93,6 +93,11 @@ struct Sel3 {
   const char *fresh[3];
   char *out[3];
   int64_t chunks[3];  // 16-byte chunks per (layer, sequence) row of each tensor
+  // nullable: each sequence's token id and top-1 probability of the step, both variants
+  const int32_t *tok_loop, *tok_fresh;
+  const float *pm_loop, *pm_fresh;
+  int32_t *tok;
+  float *pm;
 };
 
 // Whether sequence b takes the loop-free variant this step: once the guard has intervened on
@@ -108,6 +113,12 @@ __global__ void select3_kernel(const int32_t *state, int state_words, int n_int_
                                int L, Sel3 s) {
   pdl_enter();
   int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (s.tok && t < batch) {
+    const int b = (int)t;
+    const bool fresh = fresh_variant(state, state_words, n_int_word, b);
+    s.tok[b] = fresh ? s.tok_fresh[b] : s.tok_loop[b];
+    s.pm[b] = fresh ? s.pm_fresh[b] : s.pm_loop[b];
+  }
   for (int k = 0; k < 3; ++k) {
     const int64_t total = (int64_t)L * batch * s.chunks[k];
     if (t < total) {
@@ -118,20 +129,6 @@ __global__ void select3_kernel(const int32_t *state, int state_words, int n_int_
     }
     t -= total;
   }
-}
-
-// each sequence's token id and top-1 probability of the step: the loop-continuing variant
-// until the guard has intervened, the loop-free one after
-__global__ void select_tokens_kernel(const int32_t *state, int state_words, int n_int_word,
-                                     int batch, const int32_t *tok_loop, const int32_t *tok_fresh,
-                                     const float *pm_loop, const float *pm_fresh, int32_t *tok,
-                                     float *pm) {
-  pdl_enter();
-  const int b = blockIdx.x * blockDim.x + threadIdx.x;
-  if (b >= batch) return;
-  const bool fresh = fresh_variant(state, state_words, n_int_word, b);
-  tok[b] = fresh ? tok_fresh[b] : tok_loop[b];
-  pm[b] = fresh ? pm_fresh[b] : pm_loop[b];
 }
 
 // Read-only streaming pass (harness, not part of the generator's recipe): every 16-byte word of
@@ -255,8 +252,17 @@ extern "C" {
 
 int syn_dev_select3(const int32_t *state, int state_words, int n_int_word, int batch, int L,
                     const int64_t *rowlen_bytes, const void *const *loop_bufs,
-                    const void *const *fresh_bufs, void *const *outs, cudaStream_t stream) {
+                    const void *const *fresh_bufs, void *const *outs, const int32_t *tok_loop,
+                    const int32_t *tok_fresh, const float *pm_loop, const float *pm_fresh,
+                    int32_t *tok, float *pm, cudaStream_t stream) {
   Sel3 s;
+  if (tok && (!tok_loop || !tok_fresh || !pm_loop || !pm_fresh || !pm)) return 1;
+  s.tok_loop = tok_loop;
+  s.tok_fresh = tok_fresh;
+  s.pm_loop = pm_loop;
+  s.pm_fresh = pm_fresh;
+  s.tok = tok;
+  s.pm = pm;
   int64_t total = 0;
   for (int k = 0; k < 3; ++k) {
     if (rowlen_bytes[k] % 16) return 1;
@@ -294,16 +300,6 @@ int syn_dev_step(const syn_workload *w, const syn_seq *seqs_dev, int batch, cons
   step_kv_kernel<<<(unsigned)((nkv + 255) / 256), 256, 0, stream>>>(*w, seqs_dev, batch, pos_dev,
                                                                     mode, k_new, v_new);
   return cudaGetLastError() == cudaSuccess ? 0 : 2;
-}
-
-int syn_dev_select_tokens(const int32_t *state, int state_words, int n_int_word, int batch,
-                          const int32_t *tok_loop, const int32_t *tok_fresh, const float *pm_loop,
-                          const float *pm_fresh, int32_t *tok, float *pm, cudaStream_t stream) {
-  return launch_pdl(select_tokens_kernel, dim3((batch + 127) / 128), dim3(128), stream, state,
-                    state_words, n_int_word, batch, tok_loop, tok_fresh, pm_loop, pm_fresh, tok,
-                    pm) == cudaSuccess
-             ? 0
-             : 2;
 }
 
 // one read-only pass over bytes (a multiple of 16, 16-byte aligned) of device memory; ctas = the

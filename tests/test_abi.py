@@ -19,7 +19,7 @@ def declared():
 
 def test_every_declared_symbol_is_exported():
     names = declared()
-    assert len(names) == 20
+    assert len(names) == 21
     assert sorted(lg.exported_symbols()) == names
     L = lg.lib()
     for n in names:
@@ -147,6 +147,15 @@ def test_each_call_validates_its_arguments_on_the_host():
          1),
         ("token kept lists paired", lambda: L.lg_token_detect(by(c), F, F, F, None, 4, F, by(p),
                                                               by(tp), F, F, None, F, None), 1),
+        ("token_prune kept lists", lambda: L.lg_token_detect_prune(by(c), F, F, F, F, by(p),
+                                                                   by(tp), F, F, None, F, None,
+                                                                   F, 10, 10, None), 1),
+        ("token_prune budget", lambda: L.lg_token_detect_prune(by(c), F, F, F, None, by(p),
+                                                               by(tp), F, F, None, F, F, F, 10,
+                                                               10, None), 1),
+        ("token_prune max_keep", lambda: L.lg_token_detect_prune(by(c), F, F, F, F, by(p), by(tp),
+                                                                 F, F, None, F, F, F, 0, 10,
+                                                                 None), 1),
         ("h2o evict without scores", lambda: L.lg_h2o_evict(by(c), F, F, 10, None), 1),
         ("streaming sinks", lambda: L.lg_streaming_evict(by(_fake_cache(h2o=F, pos=F)), F, F, -1,
                                                          10, None), 1),

@@ -24,7 +24,7 @@ def declarations():
 
 def test_every_declaration_has_a_wrapper():
     decl = declarations()
-    assert len(decl) == 20
+    assert len(decl) == 21
     for name in decl:
         assert callable(getattr(lg, name, None)), name
 

@@ -47,11 +47,15 @@ OTHER = (dict(W=300, p_min=2, p_max=50, m_rep=2, l_min=24, stall_len=6, cooldown
          dict(hist=320, cr_every=5, theta_streak=4))
 
 
-@pytest.mark.parametrize("pass_kept,params", [(True, None), (False, None), (True, OTHER)])
-def test_token_monitor_and_prune_match_oracle(cuda, pass_kept, params):
+@pytest.mark.parametrize("pass_kept,params,fused", [(True, None, False), (False, None, False),
+                                                    (True, OTHER, False), (True, None, True),
+                                                    (True, OTHER, True)])
+def test_token_monitor_and_prune_match_oracle(cuda, pass_kept, params, fused):
     """pass_kept: the monitor gets the previous prune's retained lists (rows kept in order at
     the tail stay mapped to their tokens), or not (only rows appended since a prune are);
-    params: (guard, token) parameter overrides, the same on both sides"""
+    params: (guard, token) parameter overrides, the same on both sides; fused: one
+    lg_token_detect_prune call (the monitor's kernel forms the retained set over the previous
+    lists it has just read) in place of lg_token_detect + lg_prune_compact"""
     rng = np.random.default_rng(7)
     toks, pmax = _streams(rng)
     b = toks.shape[0]
@@ -86,11 +90,16 @@ def test_token_monitor_and_prune_match_oracle(cuda, pass_kept, params):
     keys = ("ttr", "cr", "streak", "sig1", "sig2", "sig3", "stall", "P")
     for t in range(STEPS):
         lg.lg_begin_step(cache)
-        lg.lg_token_detect(cache, toks_d[t], pmax_d[t], state, prm_g, tp_g, flags, spans, diag,
-                           tstate, kept_idx if pass_kept else None,
-                           kept_count if pass_kept else None)
-        lg.lg_prune_compact(cache, flags, spans, state, budget, prm_g, kept_idx, kept_count,
-                            max_keep, int(cap.max()))
+        if fused:
+            lg.lg_token_detect_prune(cache, toks_d[t], pmax_d[t], state, budget, prm_g, tp_g,
+                                     flags, spans, diag, tstate, kept_idx, kept_count, max_keep,
+                                     int(cap.max()))
+        else:
+            lg.lg_token_detect(cache, toks_d[t], pmax_d[t], state, prm_g, tp_g, flags, spans,
+                               diag, tstate, kept_idx if pass_kept else None,
+                               kept_count if pass_kept else None)
+            lg.lg_prune_compact(cache, flags, spans, state, budget, prm_g, kept_idx, kept_count,
+                                max_keep, int(cap.max()))
         torch.cuda.synchronize()
         assert lg.lg_read_device_status(cache) == 0, t
         f_g, sp_g, dg_g = flags.cpu().numpy(), spans.cpu().numpy(), diag.cpu().numpy()

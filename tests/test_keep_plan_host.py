@@ -1,4 +1,4 @@
-"""The retained set the detect kernel writes (keep_plan and keep_row in csrc/lg_guard.cu, slot j
+"""The retained set the guard kernels write (keep_plan and keep_row in csrc/lg_keep.cuh, slot j
 of I_keep as a function of j, Sec. 5.3, Eq. 10, Eq. 11), compiled for the host from the kernel's
 own source text, against the oracle's I_keep (anchors, the sparse lattice, the tail-cleaned
 recent rows, marked and collected) on a few thousand random prune events: triggered or over
@@ -15,7 +15,7 @@ import pytest
 import oracle
 
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
-SRC = os.path.join(ROOT, "paper_2604_10044_gb300", "csrc", "lg_guard.cu")
+SRC = os.path.join(ROOT, "paper_2604_10044_gb300", "csrc", "lg_keep.cuh")
 CUDA_INC = "/usr/local/cuda/include"
 
 
