@@ -78,6 +78,27 @@ def test_other_dtypes_and_head_dims(cuda, dtype, d):
     run_loopguard(w, cuda)
 
 
+@pytest.mark.parametrize("H_q,H_kv,d", [(8, 8, 128), (6, 2, 128), (10, 2, 128), (7, 1, 128),
+                                        (20, 4, 64)])
+def test_every_gqa_group(cuda, H_q, H_kv, d):
+    """the tensor-core pass at the GQA groups the benchmark shapes do not reach (g = 1, 3, 5,
+    7; odd groups store their logits one by one and pad the MMA columns differently) on the
+    guarded path, budget cuts and loops included"""
+    w = synth.make_workload(2, L=2, batch=3, n=600, budget=384, steps=4, tail=(150, 250),
+                            periods=(5, 16), H_q=H_q, H_kv=H_kv)
+    w.d = d
+    w.__post_init__()
+    run_loopguard(w, cuda)
+
+
+@pytest.mark.parametrize("H_q,H_kv", [(2, 2), (4, 2), (6, 2), (16, 2)])
+def test_h2o_every_load_width(cuda, H_q, H_kv):
+    """the H2O score update at g = 1, 2, 3, 8: logits read one, two, one and four at a time"""
+    w = synth.make_workload(2, L=2, batch=3, n=400, budget=256, steps=4, H_q=H_q, H_kv=H_kv,
+                            tail=(100, 150), periods=(6, 20))
+    assert run_h2o(w, cuda) >= 3 * 4
+
+
 def test_h2o_comparator(cuda):
     """H2O path: first cut from n > B + 1 to B (radix select + ordered gather), then one
     swap-remove per step"""
