@@ -60,21 +60,9 @@ __host__ __device__ __forceinline__ int64_t state_stride(int hist, int np) {
   return ((int64_t)kHdrWords + 2 * (int64_t)hist + np + 3) / 4 * 4;
 }
 
-__device__ __forceinline__ int block_max(int v, int *red, int lane, int warp) {
-  v = __reduce_max_sync(0xffffffffu, v);
-  if (lane == 0) red[warp] = v;
-  __syncthreads();
-  int r = red[0];
-#pragma unroll
-  for (int k = 1; k < kTokWarps; ++k) r = max(r, red[k]);
-  __syncthreads();
-  return r;
-}
-
 __global__ void __launch_bounds__(kTokThreads, 1) token_detect_kernel(TokenArgs a) {
   pdl_enter();
   extern __shared__ __align__(16) int32_t sm[];
-  __shared__ int red[kTokWarps];
   __shared__ int w_latest[kTokWarps], w_nov[kTokWarps], w_tail[kTokWarps], w_pstar[kTokWarps],
       w_run[kTokWarps];
   __shared__ int s_mismatch, s_trig, s_P, s_n_tok, s_appended, s_flag, s_level, s_span_lo,
@@ -86,8 +74,11 @@ __global__ void __launch_bounds__(kTokThreads, 1) token_detect_kernel(TokenArgs 
   const int np = p.p_max - p.p_min + 1;
   int32_t *tok_s = sm;          // [H] token of position q at q % H
   int32_t *lm_s = sm + H;       // [H] latest earlier equal token of the window at arrival
-  int32_t *x_s = sm + 2 * H;    // [W] the window, for the compression ratio
-  unsigned char *has2 = reinterpret_cast<unsigned char *>(x_s + W);  // [W]
+  // the compression ratio's arrays: the window, each position's phrase end (two buffers for
+  // the pointer jumping) and phrase count
+  int32_t *x_s = sm + 2 * H;  // [W]
+  auto nx_s = [&](int buf) { return x_s + (1 + buf) * W; };  // [W] each, buf 0 or 1
+  auto ct_s = [&](int buf) { return x_s + (3 + buf) * W; };  // [W] each
   int32_t *ts = a.tstate + (int64_t)b * state_stride(H, np);
   int32_t *ring_tok = ts + kHdrWords, *ring_lm = ts + kHdrWords + H;
   int32_t *run = ts + kHdrWords + 2 * H;
@@ -176,34 +167,58 @@ __global__ void __launch_bounds__(kTokThreads, 1) token_detect_kernel(TokenArgs 
     w_run[warp] = first_bad;
   }
 
-  // (2) compression ratio of the window, every cr_every tokens
+  // (2) compression ratio of the window, every cr_every tokens.  The greedy parse takes at
+  // position i the longest earlier match (overlap allowed) when it is two tokens or more, else
+  // one literal token.  The longest match at every i comes first, all at once: along each
+  // diagonal d (an earlier start i - d) the run of equal pairs from i to the window's end,
+  // scanned from the end, a lane per diagonal and the warp's maximum at each position; the
+  // parse is then a chain of phrase ends from 0, whose length pointer jumping finds in
+  // ceil(log2 w) rounds.
   const bool eval_cr = t % tp.cr_every == 0;
   int phrases = 0;
   if (eval_cr) {
-    for (int k = tid; k < w; k += kTokThreads) x_s[k] = tok(wlo + k);
-    __syncthreads();
-    // positions whose next two tokens occur earlier: the only ones a reference can start at
-    for (int i = tid; i < w; i += kTokThreads) {
-      unsigned char h = 0;
-      if (i + 1 < w)
-        for (int j = 0; j < i && !h; ++j) h = x_s[j] == x_s[i] && x_s[j + 1] == x_s[i + 1];
-      has2[i] = h;
+    for (int k = tid; k < w; k += kTokThreads) {
+      x_s[k] = tok(wlo + k);
+      nx_s(0)[k] = 0;  // longest earlier match at k, kept only from two tokens on
     }
     __syncthreads();
-    for (int i = 0; i < w;) {
-      ++phrases;
-      if (has2[i]) {
-        int best = 0;
-        for (int j = tid; j < i; j += kTokThreads) {
-          int k = 0;
-          while (i + k < w && x_s[j + k] == x_s[i + k]) ++k;
-          best = max(best, k);
+    for (int d0 = 1 + warp * 32; d0 < w; d0 += kTokThreads) {
+      const int d = d0 + lane;
+      int r = 0;
+      // 32-position blocks [base, top] from the end; the lane of position i keeps the warp's
+      // maximum at i and writes it once per block
+      for (int top = w - 1; top >= d0;) {
+        const int base = max(top & ~31, d0);
+        int acc = 0;
+#pragma unroll 4
+        for (int i = top; i >= base; --i) {
+          r = (i >= d && x_s[i] == x_s[i - d]) ? r + 1 : 0;
+          const int m = (int)__reduce_max_sync(0xffffffffu, (unsigned)r);
+          acc = lane == (i & 31) ? m : acc;
         }
-        i += block_max(best, red, lane, warp);
-      } else {
-        i += 1;
+        const int pos = (top & ~31) + lane;
+        if (pos >= base && pos <= top && acc >= 2) atomicMax(&nx_s(0)[pos], acc);
+        top = base - 1;
       }
     }
+    __syncthreads();
+    for (int k = tid; k < w; k += kTokThreads) {
+      nx_s(0)[k] = k + max(nx_s(0)[k], 1);  // the next phrase's start (w: none)
+      ct_s(0)[k] = 1;
+    }
+    __syncthreads();
+    int cur = 0;
+    for (int span = 1; span < w; span *= 2) {
+      for (int k = tid; k < w; k += kTokThreads) {
+        const int nk = nx_s(cur)[k];
+        const bool in = nk < w;
+        nx_s(cur ^ 1)[k] = in ? nx_s(cur)[nk] : nk;
+        ct_s(cur ^ 1)[k] = ct_s(cur)[k] + (in ? ct_s(cur)[nk] : 0);
+      }
+      __syncthreads();
+      cur ^= 1;
+    }
+    phrases = ct_s(cur)[0];
   }
   __syncthreads();
 
@@ -332,7 +347,7 @@ size_t token_state_words(const lg_guard_params &p, const lg_token_params &tp) {
 }
 
 size_t token_smem_bytes(const lg_guard_params &p, const lg_token_params &tp) {
-  return (size_t)(2 * tp.hist + p.W) * 4 + (size_t)p.W;
+  return (size_t)(2 * tp.hist + 5 * p.W) * 4;
 }
 
 cudaError_t launch_token_detect(const lg_cache &c, const int32_t *tokens, const float *pmax,
