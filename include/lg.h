@@ -19,7 +19,9 @@
  * Conventions
  *  - Every pointer inside lg_cache and every array argument marked "device" is device memory
  *    owned by the caller; the library allocates nothing and keeps no global state, except
- *    the static scratch array that lg_decode_attend_noalloc uses in place of a workspace.
+ *    the static scratch array that lg_decode_attend_noalloc uses in place of a workspace and
+ *    two lookups cached for the process (the driver's tensor-map encoder, and per GPU the
+ *    compaction kernel's resident CTAs), which no result depends on.
  *  - Every call is asynchronous on the caller's stream; nothing synchronises except
  *    lg_read_device_status.
  *  - Kernels are launched with programmatic stream serialization (programmatic dependent
