@@ -1,7 +1,8 @@
 """Device-side error reporting through the sticky status word (no fault, trap or hang):
 a sequence at capacity, a length above the call's max_len, and a budget with no room for the
-retained set each record their code, later kernels skip their work, and the host reads the
-code with lg_read_device_status.  Host-side validation errors return before any launch."""
+retained set (in the retained-set kernel and in the token-level monitor's) each record their
+code, later kernels skip their work, and the host reads the code with lg_read_device_status.
+Host-side validation errors return before any launch."""
 import numpy as np
 import pytest
 import torch
@@ -49,6 +50,29 @@ def test_budget_without_room_sets_status(cuda):
     lg.lg_prune_compact(cache, None, None, None, budget, g.p, g.kept_idx, g.kept_count,
                         g.max_keep, g.max_len)
     assert lg.lg_read_device_status(cache) == 7   # LG_ERR_BUDGET
+
+
+def test_token_prune_budget_without_room_sets_status(cuda):
+    """lg_token_detect_prune: the token-level monitor's kernel records LG_ERR_BUDGET when the
+    budget leaves no room for the retained set, before it writes a kept list or a length, and
+    the compaction after it skips its work"""
+    w, cache = _small(cuda)
+    g = lg.Guard(cache, w.H_q)
+    tp = lg.lg_default_token_params()
+    tstate = torch.zeros(lg.lg_token_state_size(cache, g.p, tp) // 4, dtype=torch.int32,
+                         device=cuda)
+    lg.lg_state_init(cache, g.state, 0)
+    tok = torch.arange(w.batch, dtype=torch.int32, device=cuda)
+    pm = torch.full((w.batch,), 0.5, dtype=torch.float32, device=cuda)
+    budget = torch.full((w.batch,), 60, dtype=torch.int32, device=cuda)   # < anchors + headroom
+    g.kept_count.fill_(-1)
+    before, k0 = cache.lengths().copy(), cache.k.clone()
+    lg.lg_token_detect_prune(cache, tok, pm, g.state, budget, g.p, tp, g.flags, g.spans, None,
+                             tstate, g.kept_idx, g.kept_count, g.max_keep, g.max_len)
+    assert lg.lg_read_device_status(cache) == 7   # LG_ERR_BUDGET
+    assert np.array_equal(cache.lengths(), before)
+    assert (g.kept_count.cpu() == -1).all()
+    assert torch.equal(cache.k, k0)
 
 
 def test_host_validation_launches_nothing(cuda):
