@@ -932,6 +932,30 @@ __global__ void __launch_bounds__(kH2OThreads) evict_kernel(lg_cache c, const in
   auto protected_row = [&](int i) -> bool {
     return ps[i] > thrp || (kMode == kEvictStreaming && ps[i] < n_sink);
   };
+  auto refill = [&](int x) {  // slot x takes the last slot's row, score and position
+    for (int ch = tid; ch < cpr; ch += kH2OThreads) {
+      K4[(int64_t)x * cpr + ch] = K4[(int64_t)(n - 1) * cpr + ch];
+      V4[(int64_t)x * cpr + ch] = V4[(int64_t)(n - 1) * cpr + ch];
+    }
+    if (tid == 0) {
+      sc[x] = sc[n - 1];
+      ps[x] = ps[n - 1];
+    }
+  };
+  if (kMode == kEvictStreaming && n == B + 1 && B > n_sink) {
+    // Sliding window: after the first cut its slots [n_sink, B) hold consecutive positions in
+    // slot order, and each step's row takes the slot of the oldest, so the slots stay a ring in
+    // position order and the row to evict (position thrp) sits at n_sink + (thrp - ps[n_sink])
+    // mod (B - n_sink).  One check of that slot's position replaces the scan below, which
+    // runs whenever the check fails (the same slot in every case the ring holds).
+    const int w = B - n_sink;
+    const int64_t r = ((int64_t)thrp - ps[n_sink]) % w;
+    const int x = n_sink + (int)(r < 0 ? r + w : r);
+    if (ps[x] == thrp) {
+      refill(x);
+      return;
+    }
+  }
   if (n == B + 1) {
     // one row over budget: evict the lowest key outside the protected rows and refill its
     // slot from the last slot
@@ -950,14 +974,7 @@ __global__ void __launch_bounds__(kH2OThreads) evict_kernel(lg_cache c, const in
     __syncthreads();
     const int x = s_slot;
     if (x < 0 || x == n - 1) return;
-    for (int ch = tid; ch < cpr; ch += kH2OThreads) {
-      K4[(int64_t)x * cpr + ch] = K4[(int64_t)(n - 1) * cpr + ch];
-      V4[(int64_t)x * cpr + ch] = V4[(int64_t)(n - 1) * cpr + ch];
-    }
-    if (tid == 0) {
-      sc[x] = sc[n - 1];
-      ps[x] = ps[n - 1];
-    }
+    refill(x);
     return;
   }
   if (kMode == kEvictStreaming) {

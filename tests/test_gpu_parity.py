@@ -147,6 +147,15 @@ def test_streaming_comparator(cuda):
     run_streaming(w, cuda)
 
 
+def test_streaming_window_wraps(cuda):
+    """StreamingLLM over 150 steps with a 64-row budget (4 sinks + a 60-row window): the window's
+    slots are refilled in ring order and wrap twice; every step's rows and positions match the
+    oracle's oldest-row eviction"""
+    w = synth.make_workload(4, L=1, batch=3, len_range=(100, 300), budget_max=64, steps=150,
+                            periods=(4, 8), onset_max=2)
+    run_streaming(w, cuda)
+
+
 def test_paper_shaped_guard(cuda):
     """workload 6 structure (the paper's setting: 16/8 heads, one 3853-token prompt, B=1024):
     the first budget cut from 3854 rows, periodic budget cuts every B - T_keep steps, and a
