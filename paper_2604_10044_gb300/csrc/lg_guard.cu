@@ -901,7 +901,8 @@ __global__ void __launch_bounds__(kH2OThreads) evict_kernel(lg_cache c, const in
                                                             const int32_t *pos_now, int max_len,
                                                             int n_sink) {
   pdl_enter();
-  __shared__ unsigned long long s_min;
+  __shared__ unsigned long long s_wbest[kH2OThreads / 32];
+  __shared__ int s_wslot[kH2OThreads / 32];
   __shared__ int s_slot, s_count, s_out;
   __shared__ unsigned int hist[256];
   __shared__ unsigned long long s_prefix;
@@ -958,19 +959,42 @@ __global__ void __launch_bounds__(kH2OThreads) evict_kernel(lg_cache c, const in
   }
   if (n == B + 1) {
     // one row over budget: evict the lowest key outside the protected rows and refill its
-    // slot from the last slot
+    // slot from the last slot.  Keys are unique (the position is part of the key), so one pass
+    // keeps each thread's lowest key with its slot, and a reduction picks the CTA's.
     unsigned long long best = ~0ull;
+    int slot = -1;
     for (int i = tid; i < n; i += kH2OThreads)
-      if (!protected_row(i)) best = min(best, evict_key(i));
-    if (tid == 0) {
-      s_min = ~0ull;
-      s_slot = -1;
+      if (!protected_row(i)) {
+        const unsigned long long key = evict_key(i);
+        if (key < best) {
+          best = key;
+          slot = i;
+        }
+      }
+#pragma unroll
+    for (int o = 16; o >= 1; o >>= 1) {
+      const unsigned long long ob = __shfl_xor_sync(0xffffffffu, best, o);
+      const int os = __shfl_xor_sync(0xffffffffu, slot, o);
+      if (ob < best) {
+        best = ob;
+        slot = os;
+      }
+    }
+    if ((tid & 31) == 0) {
+      s_wbest[tid >> 5] = best;
+      s_wslot[tid >> 5] = slot;
     }
     __syncthreads();
-    atomicMin(&s_min, best);
-    __syncthreads();
-    for (int i = tid; i < n; i += kH2OThreads)
-      if (!protected_row(i) && evict_key(i) == s_min) s_slot = i;
+    if (tid == 0) {
+      unsigned long long m = ~0ull;
+      int x = -1;
+      for (int w = 0; w < kH2OThreads / 32; ++w)
+        if (s_wbest[w] < m) {
+          m = s_wbest[w];
+          x = s_wslot[w];
+        }
+      s_slot = x;
+    }
     __syncthreads();
     const int x = s_slot;
     if (x < 0 || x == n - 1) return;
