@@ -44,7 +44,11 @@ EV_EVERY = 8  # timing events on every 8th timed step,
 EV_SAMPLES = 40  # or on about 40 steps of a longer run (each sampled step loses its overlap)
 DEFAULT_STEPS = 400
 DEFAULT_STEPS_W5 = 20   # about 0.25 s of GPU time from the fresh 275 GB cache
-ORACLE_TARGET_S = 20.0  # CPU seconds of the oracle's timed sample (both oracle figures)
+ORACLE_TARGET_S = 20.0  # CPU seconds the oracle's timed sample may take, about (a cap)
+# (row, kv-head) reads of the oracle's sample over its K steps: the sampled layer count follows
+# from the workload and K alone, so both oracle figures time the same sample (about 11 s on the
+# 16 Grace cores at the default line: 10 of 32 layers of sequence 0)
+ORACLE_SAMPLE_ROW_HEADS = 6.0e7
 
 
 def parse():
@@ -921,18 +925,26 @@ def time_oracle(w, n_seq, n_layers, steps, warm=0, policy="loopguard"):
 def oracle_sample(w, K, W, policy="loopguard", target_s=ORACLE_TARGET_S, max_layers=None):
     """The oracle on a bounded sample of the GPU arm's timed run: sequence 0 of the batch and its
     first n_layers layers, W warm-up steps, then the same K consecutive guarded decode steps from
-    a fresh cache (the first carries the budget cut, as on the GPU).  n_layers is sized from a
-    one-layer calibration run so that the K timed steps take about target_s.  Both oracle figures
+    a fresh cache (the first carries the budget cut, as on the GPU).  n_layers follows from the
+    sample's work (ORACLE_SAMPLE_ROW_HEADS), capped by a one-layer timing run so that the K timed
+    steps take at most about 2 target_s on a slow host.  Both oracle figures
     of bench.py (the GPU line's cpu_baseline and the --impl reference line) are this sample.
     Returns a dict: value (batch steps/s, the sample scaled by sequences and layers), the
     measured seconds, the scale and a description."""
     if max_layers == 1:
         n_layers = 1
     else:
+        # from the sample's work: sequence 0 reads its n0 + 1 rows on the first step and at most
+        # its budget's on every later one, once per kv-head and layer
+        n0, B = int(w.n0[0]), int(w.budget[0])
+        per_layer = ((n0 + 1) + (K - 1) * min(n0 + 1, B)) * w.H_kv
+        n_layers = int(min(max_layers or w.L, max(1, round(ORACLE_SAMPLE_ROW_HEADS / per_layer))))
+        # a cap from a one-layer timing run, for a host much slower than the one the work figure
+        # was set on (one layer on few cores overstates a layer's share, so this rarely binds)
         cal = min(K, 3)
         t_cal, _ = time_oracle(w, 1, 1, cal, policy=policy)
-        per_layer = t_cal[0] + (K - 1) * (float(np.mean(t_cal[1:])) if cal > 1 else t_cal[0])
-        n_layers = int(max(1, min(max_layers or w.L, target_s // max(per_layer, 1e-6))))
+        t_layer = t_cal[0] + (K - 1) * (float(np.mean(t_cal[1:])) if cal > 1 else t_cal[0])
+        n_layers = int(max(1, min(n_layers, (2 * target_s) // max(t_layer, 1e-6))))
     times, threads = time_oracle(w, 1, n_layers, K, warm=W, policy=policy)
     sec = sum(times)
     scale = (1.0 / w.batch) * (n_layers / w.L)   # batch steps per sampled step
