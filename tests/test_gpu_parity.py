@@ -156,6 +156,19 @@ def test_streaming_window_wraps(cuda):
     run_streaming(w, cuda)
 
 
+@pytest.mark.parametrize("policy", ["h2o", "streaming"])
+def test_comparators_at_the_paper_shape(cuda, policy):
+    """H2O and StreamingLLM at the paper's setting with all 28 layers (16/8 heads, the 3853-row
+    prompt, B = 1024): the first cut to the budget, then 80 steps of one eviction each (H2O's
+    one-pass choice of the lowest score, StreamingLLM's slot of the window's oldest row),
+    every step's outputs, statistics, rows and positions against the oracle"""
+    w = synth.make_workload(6, steps=80)
+    if policy == "h2o":
+        run_h2o(w, cuda)
+    else:
+        run_streaming(w, cuda)
+
+
 def test_paper_shaped_guard(cuda):
     """workload 6 structure (the paper's setting: 16/8 heads, one 3853-token prompt, B=1024):
     the first budget cut from 3854 rows, periodic budget cuts every B - T_keep steps, and a
