@@ -410,9 +410,10 @@ class GpuBench:
         if ev:
             ev[0].record(self.stream)
         for l0 in range(0, w.L, self.nl):
-            lg.lg_decode_attend(c, l0, self.nl, self.q[l0:l0 + self.nl], w.H_q, g.scale,
-                                g.out[l0:l0 + self.nl], g.stats[l0:l0 + self.nl], p.suffix_w,
-                                1 if h2o else 0, g.max_len, g.ws, self.s)
+            nl = min(self.nl, w.L - l0)   # the last call takes what is left
+            lg.lg_decode_attend(c, l0, nl, self.q[l0:l0 + nl], w.H_q, g.scale, g.out[l0:l0 + nl],
+                                g.stats[l0:l0 + nl], p.suffix_w, 1 if h2o else 0, g.max_len,
+                                g.ws, self.s)
         if ev:
             ev[1].record(self.stream)
         token = guard_path and self.detector == "token"

@@ -393,8 +393,8 @@ class Guard:
         c, p = self.cache, self.p
         lg_begin_step(c, stream)
         lg_append(c, 0, c.L, k_new, v_new, pos_new, p, stream)
-        nl = self.n_layers_per_call
-        for l0 in range(0, c.L, nl):
+        for l0 in range(0, c.L, self.n_layers_per_call):
+            nl = min(self.n_layers_per_call, c.L - l0)   # the last call takes what is left
             lg_decode_attend(c, l0, nl, q[l0:l0 + nl], self.H_q, self.scale, self.out[l0:l0 + nl],
                              self.stats[l0:l0 + nl], p.suffix_w, 1 if self.policy == "h2o" else 0,
                              self.max_len, self.ws, stream)

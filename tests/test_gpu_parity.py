@@ -30,11 +30,13 @@ def test_llama_shaped_small_multistep(cuda):
     assert c["triggers"] >= 1 and c["prunes"] >= 4
 
 
-def test_per_layer_calls_match(cuda):
-    """the same workload with one lg_decode_attend call per layer"""
+@pytest.mark.parametrize("per_call", [1, 2])
+def test_per_layer_calls_match(cuda, per_call):
+    """the same workload with lg_decode_attend called per layer, or per two layers (calls of 2
+    and 1 layers on one workspace: a different group count per call)"""
     w = synth.make_workload(2, L=3, batch=2, n=700, budget=512, steps=6, tail=(200, 300),
                             periods=(10, 30))
-    run_loopguard(w, cuda, n_layers_per_call=1)
+    run_loopguard(w, cuda, n_layers_per_call=per_call)
 
 
 def test_separate_detect_and_prune_calls(cuda):
