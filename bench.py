@@ -988,7 +988,7 @@ def run_reference(args, ws, rank):
     if rank != 0:
         return
     K, W = args.steps, args.warmup
-    w = synth.make_workload(args.workload, steps=max(K, W, 1))
+    w = gpu_workload(args, rank)   # rank 0's batch: the GPU arm's, --batch included
     o = oracle_sample(w, K, W, args.policy)
     value = o["value"]
     line = {"impl": "reference", "metric": METRIC, "value": round(value, 6), "unit": UNIT,
