@@ -894,24 +894,53 @@ def oracle_sample_workload(w, n_seq):
     return sub
 
 
-def time_oracle(w, n_seq, n_layers, steps, warm=0, policy="loopguard"):
+def time_oracle(w, n_seq, n_layers, steps, warm=0, policy="loopguard", detector="kv"):
     """the oracle (as it stands) running `steps` guarded decode steps of the first n_seq
     sequences restricted to the first n_layers layers, from a fresh cache (after `warm`
-    warm-up steps, themselves from a fresh cache); returns (seconds per step, threads)"""
+    warm-up steps, themselves from a fresh cache); detector "token": the token-level monitor
+    on the generated-token streams in place of the KV-space test, as on the GPU arm (tokens
+    counted from 0, each sequence's loop-free tokens once the guard has intervened on it).
+    Returns (seconds per step, threads)"""
     import oracle
     sub = oracle_sample_workload(w, n_seq)
     sub.L = n_layers
     K, V = synth.host_cache(sub)
+    token = policy == "loopguard" and detector == "token"
 
     def run(n):
-        g = oracle.OracleGuard(sub, K.copy(), V.copy(), policy=policy)
+        g = oracle.OracleGuard(sub, K.copy(), V.copy(), policy=policy,
+                               t_gen0=0 if token else 64)
         seqs = sub.seqs.copy()
         pos = sub.n0.astype(np.int64)
+        if token:
+            tl, tf, pl, pf = synth.token_streams(sub, n)
+            tp = oracle.token_params()
+            ts = [oracle.new_token_state() for _ in range(sub.batch)]
+            hist = np.zeros((n, sub.batch), dtype=np.int32)
+            prev_kept = [None] * sub.batch
         times = []
         for t in range(n):
             q, kn, vn = synth.host_step(sub, pos, seqs)
             t0 = time.perf_counter()
-            r = g.step(q, kn, vn, pos)
+            if token:
+                g.append(kn, vn)
+                g.attend(q)
+                flags = np.zeros(sub.batch, dtype=np.int32)
+                spans = np.zeros((sub.batch, 2), dtype=np.int32)
+                for b in range(sub.batch):
+                    fresh = g.state[b].n_int > 0
+                    hist[t, b] = tf[t, b] if fresh else tl[t, b]
+                    pm = float(pf[t, b] if fresh else pl[t, b])
+                    flags[b], spans[b], _ = oracle.token_detect(
+                        hist[:t + 1, b], pm, int(g.len[b]), g.prm, tp, g.state[b], ts[b],
+                        kept=prev_kept[b])
+                n_before = g.len.copy()
+                kept = g.prune(flags, spans)
+                prev_kept = [kept[b] if flags[b] or n_before[b] > sub.budget[b] else None
+                             for b in range(sub.batch)]
+                r = {"flags": flags}
+            else:
+                r = g.step(q, kn, vn, pos)
             times.append(time.perf_counter() - t0)
             if policy == "loopguard":
                 synth.note_interventions(seqs, pos, r["flags"])
@@ -923,7 +952,8 @@ def time_oracle(w, n_seq, n_layers, steps, warm=0, policy="loopguard"):
     return run(steps)
 
 
-def oracle_sample(w, K, W, policy="loopguard", target_s=ORACLE_TARGET_S, max_layers=None):
+def oracle_sample(w, K, W, policy="loopguard", target_s=ORACLE_TARGET_S, max_layers=None,
+                  detector="kv"):
     """The oracle on a bounded sample of the GPU arm's timed run: sequence 0 of the batch and its
     first n_layers layers, W warm-up steps, then the same K consecutive guarded decode steps from
     a fresh cache (the first carries the budget cut, as on the GPU).  n_layers follows from the
@@ -943,10 +973,10 @@ def oracle_sample(w, K, W, policy="loopguard", target_s=ORACLE_TARGET_S, max_lay
         # a cap from a one-layer timing run, for a host much slower than the one the work figure
         # was set on (one layer on few cores overstates a layer's share, so this rarely binds)
         cal = min(K, 3)
-        t_cal, _ = time_oracle(w, 1, 1, cal, policy=policy)
+        t_cal, _ = time_oracle(w, 1, 1, cal, policy=policy, detector=detector)
         t_layer = t_cal[0] + (K - 1) * (float(np.mean(t_cal[1:])) if cal > 1 else t_cal[0])
         n_layers = int(max(1, min(n_layers, (2 * target_s) // max(t_layer, 1e-6))))
-    times, threads = time_oracle(w, 1, n_layers, K, warm=W, policy=policy)
+    times, threads = time_oracle(w, 1, n_layers, K, warm=W, policy=policy, detector=detector)
     sec = sum(times)
     scale = (1.0 / w.batch) * (n_layers / w.L)   # batch steps per sampled step
     return {"value": K * scale / sec, "sec": sec, "steps": K, "scale": scale,
@@ -961,17 +991,19 @@ def cpu_baseline(w, args):
     """the oracle on the host cores: the bounded sample of oracle_sample, as batch steps/s; and
     beside it the same trajectory's first steps on one thread (one layer, at most 2 steps, in a
     fresh interpreter: the oracle takes its thread count when it loads)"""
-    o = oracle_sample(w, args.steps, args.warmup, args.policy)
+    o = oracle_sample(w, args.steps, args.warmup, args.policy, detector=args.detector)
     line = {"value": round(o["value"], 6), "unit": UNIT, "cores": o["threads"],
             "kind": "oracle", "affinity_cores": len(os.sched_getaffinity(0)),
             "sample": o["sample"], "sample_scale": o["scale"],
             "ms_per_sample_step": round(o["sec"] / o["steps"] * 1e3, 3)}
     try:
         env = dict(os.environ, OMP_NUM_THREADS="1")
-        r = subprocess.run([sys.executable, os.path.abspath(__file__), "--oracle-one-thread",
-                            "--workload", str(args.workload), "--steps", str(min(args.steps, 2)),
-                            "--policy", args.policy], env=env, capture_output=True, text=True,
-                           timeout=600)
+        cmd = [sys.executable, os.path.abspath(__file__), "--oracle-one-thread",
+               "--workload", str(args.workload), "--steps", str(min(args.steps, 2)),
+               "--policy", args.policy, "--detector", args.detector]
+        if args.batch:
+            cmd += ["--batch", str(args.batch)]
+        r = subprocess.run(cmd, env=env, capture_output=True, text=True, timeout=600)
         one = json.loads(r.stdout.strip().splitlines()[-1])
         line["single_thread"] = {"value": round(one["value"], 6), "unit": UNIT,
                                  "cores": one["threads"], "sample": one["sample"]}
@@ -989,7 +1021,7 @@ def run_reference(args, ws, rank):
         return
     K, W = args.steps, args.warmup
     w = gpu_workload(args, rank)   # rank 0's batch: the GPU arm's, --batch included
-    o = oracle_sample(w, K, W, args.policy)
+    o = oracle_sample(w, K, W, args.policy, detector=args.detector)
     value = o["value"]
     line = {"impl": "reference", "metric": METRIC, "value": round(value, 6), "unit": UNIT,
             "n_gpus": ws, "steps": K, "warmup": W,
@@ -1033,8 +1065,9 @@ def main():
     args = parse()
     if args.oracle_one_thread:
         # internal: the oracle's sample on this process's threads (one, from the environment)
-        w = synth.make_workload(args.workload, steps=max(args.steps, 1))
-        o = oracle_sample(w, args.steps, 0, args.policy, target_s=0.0, max_layers=1)
+        w = gpu_workload(args)
+        o = oracle_sample(w, args.steps, 0, args.policy, target_s=0.0, max_layers=1,
+                          detector=args.detector)
         print(json.dumps({"value": o["value"], "threads": o["threads"], "sample": o["sample"]}),
               flush=True)
         return

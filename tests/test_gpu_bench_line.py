@@ -47,11 +47,15 @@ def test_bench_line_keeps_the_contract():
     assert d["gpu_launches"] == 7 * 6
 
 
-def test_reference_line_is_on_the_same_config():
-    args = ["--workload", "2", "--batch", "2", "--steps", "4", "--warmup", "3"]
+@pytest.mark.parametrize("detector", ["kv", "token"])
+def test_reference_line_is_on_the_same_config(detector):
+    """the reference arm times the GPU arm's batch (--batch) and detector (--detector)"""
+    args = ["--workload", "2", "--batch", "2", "--steps", "4", "--warmup", "3", "--detector",
+            detector]
     d = _line(*args, "--no-cpu-baseline")
     r = _line(*args, "--impl", "reference")
     assert r["impl"] == "reference" and r["metric"] == d["metric"] and r["unit"] == d["unit"]
     assert r["config"] == d["config"] and r["higher_is_better"] is True
     assert r["value"] > 0 and r["cpu_baseline"]["kind"] == "oracle"
     assert r["e2e"]["h2d_bytes_per_step"] == 0 and r["e2e"]["d2h_bytes_per_step"] == 0
+    assert "of 2" in r["cpu_baseline"]["sample"]   # sequence 0 of the GPU arm's 2
