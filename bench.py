@@ -894,12 +894,14 @@ def oracle_sample_workload(w, n_seq):
     return sub
 
 
-def time_oracle(w, n_seq, n_layers, steps, warm=0, policy="loopguard", detector="kv"):
+def time_oracle(w, n_seq, n_layers, steps, warm=0, policy="loopguard", detector="kv",
+                fresh=False):
     """the oracle (as it stands) running `steps` guarded decode steps of the first n_seq
     sequences restricted to the first n_layers layers, from a fresh cache (after `warm`
     warm-up steps, themselves from a fresh cache); detector "token": the token-level monitor
     on the generated-token streams in place of the KV-space test, as on the GPU arm (tokens
-    counted from 0, each sequence's loop-free tokens once the guard has intervened on it).
+    counted from 0, each sequence's loop-free tokens once the guard has intervened on it);
+    fresh: every timed step from a fresh cache (the first step, as --fresh-each-step times it).
     Returns (seconds per step, threads)"""
     import oracle
     sub = oracle_sample_workload(w, n_seq)
@@ -949,11 +951,17 @@ def time_oracle(w, n_seq, n_layers, steps, warm=0, policy="loopguard", detector=
 
     if warm:
         run(warm)          # warm-up steps; the timed steps start again from the fresh cache
+    if fresh:
+        times, threads = [], 1
+        for _ in range(steps):
+            t, threads = run(1)
+            times += t
+        return times, threads
     return run(steps)
 
 
 def oracle_sample(w, K, W, policy="loopguard", target_s=ORACLE_TARGET_S, max_layers=None,
-                  detector="kv"):
+                  detector="kv", fresh=False):
     """The oracle on a bounded sample of the GPU arm's timed run: sequence 0 of the batch and its
     first n_layers layers, W warm-up steps, then the same K consecutive guarded decode steps from
     a fresh cache (the first carries the budget cut, as on the GPU).  n_layers follows from the
@@ -968,30 +976,34 @@ def oracle_sample(w, K, W, policy="loopguard", target_s=ORACLE_TARGET_S, max_lay
         # from the sample's work: sequence 0 reads its n0 + 1 rows on the first step and at most
         # its budget's on every later one, once per kv-head and layer
         n0, B = int(w.n0[0]), int(w.budget[0])
-        per_layer = ((n0 + 1) + (K - 1) * min(n0 + 1, B)) * w.H_kv
+        per_layer = ((n0 + 1) * K if fresh else (n0 + 1) + (K - 1) * min(n0 + 1, B)) * w.H_kv
         n_layers = int(min(max_layers or w.L, max(1, round(ORACLE_SAMPLE_ROW_HEADS / per_layer))))
         # a cap from a one-layer timing run, for a host much slower than the one the work figure
         # was set on (one layer on few cores overstates a layer's share, so this rarely binds)
         cal = min(K, 3)
-        t_cal, _ = time_oracle(w, 1, 1, cal, policy=policy, detector=detector)
+        t_cal, _ = time_oracle(w, 1, 1, cal, policy=policy, detector=detector, fresh=fresh)
         t_layer = t_cal[0] + (K - 1) * (float(np.mean(t_cal[1:])) if cal > 1 else t_cal[0])
         n_layers = int(max(1, min(n_layers, (2 * target_s) // max(t_layer, 1e-6))))
-    times, threads = time_oracle(w, 1, n_layers, K, warm=W, policy=policy, detector=detector)
+    times, threads = time_oracle(w, 1, n_layers, K, warm=W, policy=policy, detector=detector,
+                                 fresh=fresh)
     sec = sum(times)
     scale = (1.0 / w.batch) * (n_layers / w.L)   # batch steps per sampled step
     return {"value": K * scale / sec, "sec": sec, "steps": K, "scale": scale,
             "threads": threads, "n_layers": n_layers,
-            "sample": "the first %d guarded decode steps of the GPU arm's timed trajectory, from "
-                      "its fresh cache (after %d warm-up step(s)), of sequence 0 of %d and its "
-                      "layers 0..%d of %d; value = steps x %.6f batch steps per sampled step / "
-                      "%.2f s" % (K, W, w.batch, n_layers - 1, w.L, scale, sec)}
+            "sample": "%s (after %d warm-up step(s)), of sequence 0 of %d and its layers 0..%d "
+                      "of %d; value = steps x %.6f batch steps per sampled step / %.2f s" % (
+                          "%d first guarded decode steps, each from a fresh cache" % K if fresh
+                          else "the first %d guarded decode steps of the GPU arm's timed "
+                               "trajectory, from its fresh cache" % K,
+                          W, w.batch, n_layers - 1, w.L, scale, sec)}
 
 
 def cpu_baseline(w, args):
     """the oracle on the host cores: the bounded sample of oracle_sample, as batch steps/s; and
     beside it the same trajectory's first steps on one thread (one layer, at most 2 steps, in a
     fresh interpreter: the oracle takes its thread count when it loads)"""
-    o = oracle_sample(w, args.steps, args.warmup, args.policy, detector=args.detector)
+    o = oracle_sample(w, args.steps, args.warmup, args.policy, detector=args.detector,
+                      fresh=args.fresh_each_step)
     line = {"value": round(o["value"], 6), "unit": UNIT, "cores": o["threads"],
             "kind": "oracle", "affinity_cores": len(os.sched_getaffinity(0)),
             "sample": o["sample"], "sample_scale": o["scale"],
@@ -1003,6 +1015,8 @@ def cpu_baseline(w, args):
                "--policy", args.policy, "--detector", args.detector]
         if args.batch:
             cmd += ["--batch", str(args.batch)]
+        if args.fresh_each_step:
+            cmd += ["--fresh-each-step"]
         r = subprocess.run(cmd, env=env, capture_output=True, text=True, timeout=600)
         one = json.loads(r.stdout.strip().splitlines()[-1])
         line["single_thread"] = {"value": round(one["value"], 6), "unit": UNIT,
@@ -1021,7 +1035,7 @@ def run_reference(args, ws, rank):
         return
     K, W = args.steps, args.warmup
     w = gpu_workload(args, rank)   # rank 0's batch: the GPU arm's, --batch included
-    o = oracle_sample(w, K, W, args.policy, detector=args.detector)
+    o = oracle_sample(w, K, W, args.policy, detector=args.detector, fresh=args.fresh_each_step)
     value = o["value"]
     line = {"impl": "reference", "metric": METRIC, "value": round(value, 6), "unit": UNIT,
             "n_gpus": ws, "steps": K, "warmup": W,
@@ -1067,7 +1081,7 @@ def main():
         # internal: the oracle's sample on this process's threads (one, from the environment)
         w = gpu_workload(args)
         o = oracle_sample(w, args.steps, 0, args.policy, target_s=0.0, max_layers=1,
-                          detector=args.detector)
+                          detector=args.detector, fresh=args.fresh_each_step)
         print(json.dumps({"value": o["value"], "threads": o["threads"], "sample": o["sample"]}),
               flush=True)
         return

@@ -47,11 +47,12 @@ def test_bench_line_keeps_the_contract():
     assert d["gpu_launches"] == 7 * 6
 
 
-@pytest.mark.parametrize("detector", ["kv", "token"])
-def test_reference_line_is_on_the_same_config(detector):
-    """the reference arm times the GPU arm's batch (--batch) and detector (--detector)"""
-    args = ["--workload", "2", "--batch", "2", "--steps", "4", "--warmup", "3", "--detector",
-            detector]
+@pytest.mark.parametrize("extra", [["--detector", "kv"], ["--detector", "token"],
+                                   ["--fresh-each-step"]])
+def test_reference_line_is_on_the_same_config(extra):
+    """the reference arm times the GPU arm's batch (--batch), detector (--detector) and steps
+    (--fresh-each-step)"""
+    args = ["--workload", "2", "--batch", "2", "--steps", "4", "--warmup", "3", *extra]
     d = _line(*args, "--no-cpu-baseline")
     r = _line(*args, "--impl", "reference")
     assert r["impl"] == "reference" and r["metric"] == d["metric"] and r["unit"] == d["unit"]
@@ -59,3 +60,5 @@ def test_reference_line_is_on_the_same_config(detector):
     assert r["value"] > 0 and r["cpu_baseline"]["kind"] == "oracle"
     assert r["e2e"]["h2d_bytes_per_step"] == 0 and r["e2e"]["d2h_bytes_per_step"] == 0
     assert "of 2" in r["cpu_baseline"]["sample"]   # sequence 0 of the GPU arm's 2
+    assert ("each from a fresh cache" in r["cpu_baseline"]["sample"]) == \
+        ("--fresh-each-step" in extra)
